@@ -1,0 +1,158 @@
+/*
+ * emu.h -- C-ABI of the GB300 (sm_103a) BF16 component-product GEMM emulation
+ * of arXiv 2609.04663, "BF16 Component-Product Emulation of FP32 and FP64 GEMM
+ * on Intel AMX".
+ *
+ *   FP32 mode: C = A.B for FP32 A, B.  Each operand is split into 3 BF16
+ *   slices (Eq. (fp32split)) and the 6 products with i + j <= 2 are kept
+ *   (Eq. (fp32six), Algorithm 1), accumulated in FP32.
+ *
+ *   FP64 mode: C = A.B for FP64 A, B inside the BF16 exponent range
+ *   (Eq. (bf16rangefp64)).  Each operand is split into 6 BF16 slices by the
+ *   fixed simplified Ozaki projection (Eq. (fp64split)); nprod = 6, 10, 15 or
+ *   21 products (i + j < d, d = 3..6, Eq. (fp64productcounts)) are kept.  Each
+ *   product is formed in FP32 per K-chunk of 256 and widened and accumulated
+ *   in FP64 (Eq. (fp64reconstruction), Algorithm 2).
+ *
+ * Common conventions
+ *   - Every pointer argument named as a matrix, plane set, workspace or v_out
+ *     is a DEVICE pointer owned by the caller.  The library never allocates,
+ *     frees or keeps a reference to caller memory after the call returns.
+ *   - Matrices are row-major with a leading dimension in elements (ld >= cols).
+ *   - All work is enqueued on `stream` and is asynchronous to the host; the
+ *     only host synchronisation is emu_read_flags.
+ *   - Synchronous errors (bad arguments, launch failures) are returned as an
+ *     emu_status before or while enqueuing.  Numerical-domain violations and
+ *     watchdog timeouts are found on the device: they set EMU_FLAG_* bits in
+ *     the flag word at the start of the workspace, which every call clears
+ *     first; read them with emu_read_flags.  The paper has no fallback for
+ *     such inputs (Sections 3.1, 3.2): results are then unspecified.
+ *   - M = 0 or N = 0 is a no-op; K = 0 writes zeros to C.
+ *   - Component planes ("comps"): BF16 bit patterns (uint16), plane r of
+ *     a set at comps + r * rows_out * ldcomp, each plane row-major
+ *     [rows_out][ldcomp].  For an A operand (transpose = 0) rows_out = rows of
+ *     X; for a B operand (transpose = 1) the plane is stored transposed,
+ *     [cols][rows] -- K-major, as the tensor-core GEMM reads both operands.
+ *   - Product-sum entry points take planes as written by the split with
+ *     ldcomp a multiple of 8 and 16-byte aligned plane bases (the tensor
+ *     memory accelerator requires 16-byte strides); otherwise
+ *     EMU_ERR_MISALIGNED.
+ *   - Requires an sm_103 (GB300) device; the library holds sm_103a code only.
+ */
+#ifndef EMU_H
+#define EMU_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; 0 is the legacy default stream. */
+typedef struct CUstream_st *emu_stream_t;
+
+typedef enum {
+    EMU_OK = 0,
+    EMU_ERR_INVALID_ARG = 1,          /* negative size, ld < cols, bad nprod, NULL pointer */
+    EMU_ERR_MISALIGNED = 2,           /* plane base / ldcomp not 16-byte compatible */
+    EMU_ERR_WORKSPACE_TOO_SMALL = 3,  /* ws_bytes below the *_workspace_bytes value */
+    EMU_ERR_CUDA = 4,                 /* a CUDA call or kernel launch failed */
+    EMU_ERR_UNSUPPORTED = 5           /* size beyond the library's limits */
+} emu_status;
+
+/* Asynchronous flag bits (emu_read_flags). */
+#define EMU_FLAG_NONFINITE 0x1u  /* an input entry is NaN or infinite */
+#define EMU_FLAG_RANGE     0x2u  /* an FP64 input entry is outside F64^B, Eq. (bf16rangefp64) */
+#define EMU_FLAG_SLICE     0x4u  /* a slice entry is not a normal BF16 value: FP64 mode,
+                                    Z != fl_BF16(Z), or Z nonzero with |Z| < 2^-126
+                                    (Section 4.3); FP32 mode, a non-finite slice */
+#define EMU_FLAG_TIMEOUT   0x8u  /* a bounded wait inside a kernel gave up (about 2 s);
+                                    the kernel stopped early and C is incomplete */
+
+/* v_out value of a level whose residual is all zero (Section 4.3). */
+#define EMU_ZERO_LEVEL INT32_MIN
+
+/* Bytes of workspace emu_split_f32 / emu_split_f64 need (flag word and the
+ * per-level maxima of the FP64 split).  mode is 32 or 64. */
+size_t emu_split_workspace_bytes(int mode);
+
+/* FP32 three-slice split, Eq. (fp32split) / Algorithm 1 (Split_FP32):
+ *   A_r = fl_BF16(A^(r)), A^(r+1) = fl32(A^(r) - A_r), r = 0, 1, 2,
+ * fl_BF16 = round to nearest, ties to even (Section 4.1).
+ * X: rows x cols FP32, leading dimension ldx (elements, >= cols).
+ * transpose = 0: comps holds 3 planes [rows][ldcomp] (ldcomp >= cols);
+ * transpose = 1: comps holds 3 planes [cols][ldcomp] (ldcomp >= rows).
+ * Padding columns of the planes are not written.  Bit-exact and
+ * deterministic.  Flags: EMU_FLAG_NONFINITE, EMU_FLAG_SLICE. */
+emu_status emu_split_f32(const float *X, int64_t rows, int64_t cols, int64_t ldx, int transpose,
+                         uint16_t *comps, int64_t ldcomp, void *ws, size_t ws_bytes,
+                         emu_stream_t stream);
+
+/* FP64 six-slice split, Eq. (fp64split) / Algorithm 2 (Split_FP64):
+ *   v^(r) = ceil(log2(max_ij |A^(r)_ij|)) over the whole matrix,
+ *   Z = fl64(fl64(A^(r) + 2^(v+45)) - 2^(v+45)), A_r = fl_BF16(Z),
+ *   A^(r+1) = fl64(A^(r) - A_r), r = 0..5; an all-zero residual makes its
+ *   slice and all later slices zero with v = EMU_ZERO_LEVEL.
+ * Layout as emu_split_f32 with 6 planes.  v_out: device int32[6] receiving
+ * v^(0..5).  Bit-exact and deterministic for inputs in the domain.  Flags:
+ * EMU_FLAG_NONFINITE, EMU_FLAG_RANGE, EMU_FLAG_SLICE (planes then unspecified). */
+emu_status emu_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ldx, int transpose,
+                         uint16_t *comps, int64_t ldcomp, int32_t *v_out, void *ws,
+                         size_t ws_bytes, emu_stream_t stream);
+
+/* Workspace bytes for emu_gemm_f32 (mode 32) / emu_gemm_f64 (mode 64):
+ * the flag word plus the slice planes of A (M x K) and B (K x N). */
+size_t emu_gemm_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K);
+
+/* FP32-mode emulated GEMM, Algorithm 1: C (M x N, ldc) = A (M x K, lda) . B
+ * (K x N, ldb), all FP32 row-major.  Splits A and B into the workspace, then
+ * runs the tensor-core product-sum: the 6 products of Eq. (fp32six) are
+ * accumulated in one FP32 accumulator over all of K (Section 5.3, FP32
+ * reconstruction), so C matches the oracle within FP32 reordering error. */
+emu_status emu_gemm_f32(int64_t M, int64_t N, int64_t K, const float *A, int64_t lda,
+                        const float *B, int64_t ldb, float *C, int64_t ldc, void *ws,
+                        size_t ws_bytes, emu_stream_t stream);
+
+/* FP64-mode emulated GEMM, Algorithm 2: C = A . B for FP64 inputs, nprod in
+ * {6, 10, 15, 21}.  Per K-chunk of 256 each retained product's partial is
+ * formed in FP32 on the tensor cores and added into an FP64 accumulator in
+ * the oracle's order (chunk outer, diagonal order inner), so C equals the
+ * oracle bit for bit. */
+emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda,
+                        const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,
+                        void *ws, size_t ws_bytes, emu_stream_t stream);
+
+/* Product-sum alone, from planes already split (A: [3][M][ldcomp],
+ * B: [3][N][ldcomp], i.e. split with transpose = 1).  Eq. (fp32six),
+ * Section 5.3.  ws: at least emu_split_workspace_bytes(32) (flag word). */
+emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acomps,
+                           const uint16_t *Bcomps, int64_t ldcomp, float *C, int64_t ldc,
+                           void *ws, size_t ws_bytes, emu_stream_t stream);
+
+/* Product-sum alone for FP64 mode, Eq. (fp64reconstruction): A planes
+ * [6][M][ldcomp], B planes [6][N][ldcomp]; nprod in {6, 10, 15, 21}.
+ * ws: at least emu_split_workspace_bytes(64). */
+emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acomps,
+                           const uint16_t *Bcomps, int64_t ldcomp, int nprod, double *C,
+                           int64_t ldc, void *ws, size_t ws_bytes, emu_stream_t stream);
+
+/* Copies the flag word of the last call that used `ws` to *host_flags after
+ * synchronising `stream`.  ws: device workspace; host_flags: host pointer. */
+emu_status emu_read_flags(const void *ws, uint32_t *host_flags, emu_stream_t stream);
+
+/* Watchdog self-test: launches one kernel that waits, with the same bounded
+ * wait the GEMM kernels use, on a barrier that nothing completes; after
+ * timeout_us microseconds it gives up, sets EMU_FLAG_TIMEOUT in the
+ * workspace flag word and returns, leaving the context usable.
+ * timeout_us in [1, 10^6]. */
+emu_status emu_selftest_timeout(void *ws, size_t ws_bytes, uint32_t timeout_us,
+                                emu_stream_t stream);
+
+/* Static description of an emu_status value. */
+const char *emu_status_string(emu_status status);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* EMU_H */

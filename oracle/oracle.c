@@ -10,8 +10,8 @@
  * Build: gcc -O2 -ffp-contract=off -fopenmp (no fast-math), so every fl32 /
  * fl64 of the paper is exactly one IEEE-754 operation in the stated format and
  * nothing is contracted into an FMA or reassociated.  OpenMP only splits
- * independent output rows (or independent elements) between threads; it never
- * changes the order of any floating-point sum.
+ * independent output elements (or independent input entries) between threads;
+ * it never changes the order of any floating-point sum.
  *
  * Layouts (all row-major, dense):
  *   A planes  [s][M][K]  BF16 bit patterns (uint16), slice r at offset r*M*K
@@ -245,7 +245,7 @@ void oracle_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, con
     oracle_products(32, 6, pairs);
     float *a = expand_a(Ap, 3, M, K, r0, nr);
     float *b = expand_bt(Bp, 3, K, N);
-    #pragma omp parallel for schedule(dynamic, 1)
+    #pragma omp parallel for collapse(2) schedule(dynamic, 16)
     for (int64_t i = 0; i < nr; ++i) {
         for (int64_t n = 0; n < N; ++n) {
             float c32 = 0.0f;
@@ -287,7 +287,7 @@ void oracle_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, con
     float *a = expand_a(Ap, 6, M, K, r0, nr);
     float *b = expand_bt(Bp, 6, K, N);
     int64_t bad = 0;
-    #pragma omp parallel for schedule(dynamic, 1) reduction(+:bad)
+    #pragma omp parallel for collapse(2) schedule(dynamic, 16) reduction(+:bad)
     for (int64_t i = 0; i < nr; ++i) {
         for (int64_t n = 0; n < N; ++n) {
             double c64 = 0.0;
@@ -328,10 +328,10 @@ void oracle_ref_dd(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda
     #pragma omp parallel for schedule(static)
     for (int64_t n = 0; n < N; ++n)
         for (int64_t k = 0; k < K; ++k) bt[n * K + k] = B[k * ldb + n];
-    #pragma omp parallel for schedule(dynamic, 1)
+    #pragma omp parallel for collapse(2) schedule(dynamic, 16)
     for (int64_t i = 0; i < nr; ++i) {
-        const double *ar = A + (r0 + i) * lda;
         for (int64_t n = 0; n < N; ++n) {
+            const double *ar = A + (r0 + i) * lda;
             const double *bc = bt + n * K;
             double sh = 0.0, sl = 0.0;
             for (int64_t k = 0; k < K; ++k) {

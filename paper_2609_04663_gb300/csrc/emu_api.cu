@@ -1,0 +1,229 @@
+// C-ABI of the emulation library (declared in include/emu.h): argument
+// checks, workspace layout and the launch sequence of each entry point.
+#include "common.cuh"
+
+namespace emu {
+cudaError_t launch_split_f32(const float *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
+                             uint16_t *comps, int64_t ldcomp, WsHeader *ws, cudaStream_t st);
+cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
+                             uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
+                             cudaStream_t st);
+cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
+                               int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st);
+cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
+                               int64_t ldcomp, int nprod, double *C, int64_t ldc, uint32_t *flags,
+                               cudaStream_t st);
+cudaError_t launch_timeout_selftest(uint32_t *flags, uint32_t timeout_us, cudaStream_t st);
+}  // namespace emu
+
+using namespace emu;
+
+namespace {
+
+constexpr int64_t kMaxDim = (int64_t)1 << 31;      // kernels index with 32-bit coordinates
+
+int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+// K-major plane leading dimension used inside the GEMM workspace: TMA needs
+// row strides that are multiples of 16 bytes.
+int64_t gemm_ldk(int64_t K) { return round_up(K < 1 ? 1 : K, 8); }
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+emu_status cuda_status(cudaError_t e) { return e == cudaSuccess ? EMU_OK : EMU_ERR_CUDA; }
+
+emu_status check_planes(const void *Ap, const void *Bp, int64_t ldcomp, int64_t K)
+{
+    if (!Ap || !Bp || ldcomp < K || ldcomp < 1) return EMU_ERR_INVALID_ARG;
+    if ((ldcomp & 7) != 0 || !aligned16(Ap) || !aligned16(Bp)) return EMU_ERR_MISALIGNED;
+    return EMU_OK;
+}
+
+emu_status check_gemm_dims(int64_t M, int64_t N, int64_t K, int64_t lda, int64_t ldb, int64_t ldc)
+{
+    if (M < 0 || N < 0 || K < 0) return EMU_ERR_INVALID_ARG;
+    if (lda < (K > 0 ? K : 1) || ldb < (N > 0 ? N : 1) || ldc < (N > 0 ? N : 1)) return EMU_ERR_INVALID_ARG;
+    if (M >= kMaxDim || N >= kMaxDim || K >= kMaxDim) return EMU_ERR_UNSUPPORTED;
+    return EMU_OK;
+}
+
+// C = 0 for K = 0 (rows of N elements with pitch ldc).
+template <typename T>
+emu_status zero_c(T *C, int64_t M, int64_t N, int64_t ldc, cudaStream_t st)
+{
+    return cuda_status(cudaMemset2DAsync(C, (size_t)ldc * sizeof(T), 0, (size_t)N * sizeof(T), (size_t)M, st));
+}
+
+size_t gemm_ws_bytes(int s, int64_t M, int64_t N, int64_t K)
+{
+    const int64_t ldk = gemm_ldk(K);
+    return kWsHeaderBytes + (size_t)round_up((int64_t)s * M * ldk * 2, 256) + (size_t)round_up((int64_t)s * N * ldk * 2, 256);
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t emu_split_workspace_bytes(int mode)
+{
+    (void)mode;
+    return kWsHeaderBytes;
+}
+
+emu_status emu_split_f32(const float *X, int64_t rows, int64_t cols, int64_t ldx, int transpose, uint16_t *comps,
+                         int64_t ldcomp, void *ws, size_t ws_bytes, emu_stream_t stream)
+{
+    if (rows < 0 || cols < 0 || ldx < (cols > 0 ? cols : 1) || !ws) return EMU_ERR_INVALID_ARG;
+    if (ldcomp < (transpose ? rows : cols) || ldcomp < 1) return EMU_ERR_INVALID_ARG;
+    if (rows > 0 && cols > 0 && (!X || !comps)) return EMU_ERR_INVALID_ARG;
+    if (ws_bytes < kWsHeaderBytes) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
+    if (e == cudaSuccess) e = launch_split_f32(X, rows, cols, ldx, transpose != 0, comps, ldcomp, h, st);
+    return cuda_status(e);
+}
+
+emu_status emu_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ldx, int transpose, uint16_t *comps,
+                         int64_t ldcomp, int32_t *v_out, void *ws, size_t ws_bytes, emu_stream_t stream)
+{
+    if (rows < 0 || cols < 0 || ldx < (cols > 0 ? cols : 1) || !ws || !v_out) return EMU_ERR_INVALID_ARG;
+    if (ldcomp < (transpose ? rows : cols) || ldcomp < 1) return EMU_ERR_INVALID_ARG;
+    if (rows > 0 && cols > 0 && (!X || !comps)) return EMU_ERR_INVALID_ARG;
+    if (ws_bytes < kWsHeaderBytes) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
+    if (e == cudaSuccess) e = launch_split_f64(X, rows, cols, ldx, transpose != 0, comps, ldcomp, v_out, h, 0, st);
+    return cuda_status(e);
+}
+
+size_t emu_gemm_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K)
+{
+    if (M < 0 || N < 0 || K < 0) return 0;
+    return gemm_ws_bytes(mode == 64 ? 6 : 3, M, N, K);
+}
+
+emu_status emu_gemm_f32(int64_t M, int64_t N, int64_t K, const float *A, int64_t lda, const float *B, int64_t ldb,
+                        float *C, int64_t ldc, void *ws, size_t ws_bytes, emu_stream_t stream)
+{
+    emu_status s = check_gemm_dims(M, N, K, lda, ldb, ldc);
+    if (s != EMU_OK) return s;
+    if (!ws || (M > 0 && N > 0 && (!C || (K > 0 && (!A || !B))))) return EMU_ERR_INVALID_ARG;
+    if (ws_bytes < gemm_ws_bytes(3, M, N, K)) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
+    if (e != cudaSuccess) return EMU_ERR_CUDA;
+    if (M == 0 || N == 0) return EMU_OK;
+    if (K == 0) return zero_c(C, M, N, ldc, st);
+    const int64_t ldk = gemm_ldk(K);
+    uint16_t *Ap = reinterpret_cast<uint16_t *>(static_cast<char *>(ws) + kWsHeaderBytes);
+    uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(3 * M * ldk * 2, 256));
+    e = launch_split_f32(A, M, K, lda, false, Ap, ldk, h, st);
+    if (e == cudaSuccess) e = launch_split_f32(B, K, N, ldb, true, Bp, ldk, h, st);
+    if (e == cudaSuccess) e = launch_prodsum_f32(M, N, K, Ap, Bp, ldk, C, ldc, &h->flags, st);
+    return cuda_status(e);
+}
+
+emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda, const double *B,
+                        int64_t ldb, double *C, int64_t ldc, int nprod, void *ws, size_t ws_bytes,
+                        emu_stream_t stream)
+{
+    emu_status s = check_gemm_dims(M, N, K, lda, ldb, ldc);
+    if (s != EMU_OK) return s;
+    if (nprod != 6 && nprod != 10 && nprod != 15 && nprod != 21) return EMU_ERR_INVALID_ARG;
+    if (!ws || (M > 0 && N > 0 && (!C || (K > 0 && (!A || !B))))) return EMU_ERR_INVALID_ARG;
+    if (ws_bytes < gemm_ws_bytes(6, M, N, K)) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
+    if (e != cudaSuccess) return EMU_ERR_CUDA;
+    if (M == 0 || N == 0) return EMU_OK;
+    if (K == 0) return zero_c(C, M, N, ldc, st);
+    const int64_t ldk = gemm_ldk(K);
+    uint16_t *Ap = reinterpret_cast<uint16_t *>(static_cast<char *>(ws) + kWsHeaderBytes);
+    uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(6 * M * ldk * 2, 256));
+    e = launch_split_f64(A, M, K, lda, false, Ap, ldk, nullptr, h, 0, st);
+    if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, nullptr, h, 1, st);
+    if (e == cudaSuccess) e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, nprod, C, ldc, &h->flags, st);
+    return cuda_status(e);
+}
+
+emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acomps, const uint16_t *Bcomps,
+                           int64_t ldcomp, float *C, int64_t ldc, void *ws, size_t ws_bytes, emu_stream_t stream)
+{
+    if (M < 0 || N < 0 || K < 0 || ldc < (N > 0 ? N : 1) || !ws) return EMU_ERR_INVALID_ARG;
+    if (M >= kMaxDim || N >= kMaxDim || K >= kMaxDim) return EMU_ERR_UNSUPPORTED;
+    if (ws_bytes < kWsHeaderBytes) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    if (cudaMemsetAsync(&h->flags, 0, sizeof(uint32_t), st) != cudaSuccess) return EMU_ERR_CUDA;
+    if (M == 0 || N == 0) return EMU_OK;
+    if (!C) return EMU_ERR_INVALID_ARG;
+    if (K == 0) return zero_c(C, M, N, ldc, st);
+    emu_status s = check_planes(Acomps, Bcomps, ldcomp, K);
+    if (s != EMU_OK) return s;
+    return cuda_status(launch_prodsum_f32(M, N, K, Acomps, Bcomps, ldcomp, C, ldc, &h->flags, st));
+}
+
+emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acomps, const uint16_t *Bcomps,
+                           int64_t ldcomp, int nprod, double *C, int64_t ldc, void *ws, size_t ws_bytes,
+                           emu_stream_t stream)
+{
+    if (M < 0 || N < 0 || K < 0 || ldc < (N > 0 ? N : 1) || !ws) return EMU_ERR_INVALID_ARG;
+    if (nprod != 6 && nprod != 10 && nprod != 15 && nprod != 21) return EMU_ERR_INVALID_ARG;
+    if (M >= kMaxDim || N >= kMaxDim || K >= kMaxDim) return EMU_ERR_UNSUPPORTED;
+    if (ws_bytes < kWsHeaderBytes) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    if (cudaMemsetAsync(&h->flags, 0, sizeof(uint32_t), st) != cudaSuccess) return EMU_ERR_CUDA;
+    if (M == 0 || N == 0) return EMU_OK;
+    if (!C) return EMU_ERR_INVALID_ARG;
+    if (K == 0) return zero_c(C, M, N, ldc, st);
+    emu_status s = check_planes(Acomps, Bcomps, ldcomp, K);
+    if (s != EMU_OK) return s;
+    return cuda_status(launch_prodsum_f64(M, N, K, Acomps, Bcomps, ldcomp, nprod, C, ldc, &h->flags, st));
+}
+
+emu_status emu_read_flags(const void *ws, uint32_t *host_flags, emu_stream_t stream)
+{
+    if (!ws || !host_flags) return EMU_ERR_INVALID_ARG;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemcpyAsync(host_flags, &static_cast<const WsHeader *>(ws)->flags, sizeof(uint32_t),
+                                    cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    return cuda_status(e);
+}
+
+emu_status emu_selftest_timeout(void *ws, size_t ws_bytes, uint32_t timeout_us, emu_stream_t stream)
+{
+    if (!ws || timeout_us < 1 || timeout_us > 1000000) return EMU_ERR_INVALID_ARG;
+    if (ws_bytes < kWsHeaderBytes) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(&h->flags, 0, sizeof(uint32_t), st);
+    if (e == cudaSuccess) e = launch_timeout_selftest(&h->flags, timeout_us, st);
+    return cuda_status(e);
+}
+
+const char *emu_status_string(emu_status status)
+{
+    switch (status) {
+    case EMU_OK: return "ok";
+    case EMU_ERR_INVALID_ARG: return "invalid argument";
+    case EMU_ERR_MISALIGNED: return "misaligned pointer or leading dimension";
+    case EMU_ERR_WORKSPACE_TOO_SMALL: return "workspace too small";
+    case EMU_ERR_CUDA: return "CUDA error";
+    case EMU_ERR_UNSUPPORTED: return "unsupported size";
+    }
+    return "unknown status";
+}
+
+}  // extern "C"

@@ -1,0 +1,445 @@
+// Split kernels: FP32 three-slice residual split (Eq. (fp32split)) and FP64
+// fixed six-slice simplified Ozaki split (Eq. (fp64split)), writing BF16
+// component planes row-major or transposed (K-major for the B operand).
+//
+// Both are HBM-bound elementwise passes.  A 64 x 64 tile of X is read with
+// coalesced vector loads, split in registers, staged in shared memory and
+// written as 16-byte chunks of whole plane rows, so the transposed B planes
+// are written as coalesced as the row-major A planes.
+//
+// FP64 level exponents need a whole-matrix max per level (v^(r) of
+// Eq. (fp64split)), i.e. six dependent grid-wide reductions.  The split does
+// them speculatively in one pass: after the exact max of level 0, the fused
+// pass assumes v^(r) = v^(0) - 8r (a residual always shrinks by at least 2^-8
+// per level, and on full-size dense data by exactly that), writes all six
+// planes and records the true per-level maxima.  A one-thread kernel then
+// checks the assumption level by level; only if it fails do the gated fix
+// kernels recompute the remaining levels literally.  The result is
+// identical to the literal definition in every case.
+#include "common.cuh"
+
+namespace emu {
+
+namespace {
+
+constexpr int kTile = 64;            // tile edge (elements)
+constexpr int kSRow = kTile + 2;     // shared-memory row pitch in uint16 (odd word pitch)
+constexpr int kThreads = 256;
+
+// --------------------------------------------------------------- rounding
+// fl_BF16 of an FP32 value (round to nearest, ties to even) on its bit
+// pattern: add 0x7FFF plus the lowest kept bit, keep the upper half.
+__device__ __forceinline__ uint32_t bf16_rne_f32bits(float x)
+{
+    uint32_t u = __float_as_uint(x);
+    u += 0x7FFFu + ((u >> 16) & 1u);
+    return u >> 16;
+}
+
+__device__ __forceinline__ float bf16_as_float(uint32_t s) { return __uint_as_float(s << 16); }
+
+// fl_BF16 of an FP64 value, one rounding, by integer arithmetic on its bits:
+// the BF16 quantum is 2^(max(e, -126) - 7) for a leading-bit exponent e;
+// subnormal BF16 spacing 2^-133; overflow to infinity.
+__device__ uint16_t bf16_rne_f64(double z)
+{
+    const uint64_t b = (uint64_t)__double_as_longlong(z);
+    const uint16_t sign = (uint16_t)((b >> 48) & 0x8000u);
+    const uint64_t a = b & 0x7FFFFFFFFFFFFFFFull;
+    if (a > 0x7FF0000000000000ull) return 0x7FC0u;
+    if (a == 0x7FF0000000000000ull) return (uint16_t)(sign | 0x7F80u);
+    if (a == 0) return sign;
+    int E = (int)(a >> 52);
+    uint64_t m = a & 0x000FFFFFFFFFFFFFull;
+    int e;                                        // exponent of the leading bit
+    if (E) { m |= 1ull << 52; e = E - 1023; }
+    else { E = 1; e = -1022 - (__clzll((long long)m) - 11); }
+    const int qe = (e < -126 ? -126 : e) - 7;     // quantum exponent
+    const int s = qe - (E - 1075);                // value = m * 2^(E-1075)
+    uint64_t n;
+    if (s <= 0) n = m << (-s);
+    else if (s >= 64) n = 0;
+    else {
+        n = m >> s;
+        const uint64_t rem = m & ((1ull << s) - 1ull), half = 1ull << (s - 1);
+        if (rem > half || (rem == half && (n & 1ull))) ++n;
+    }
+    if (qe == -133) return (uint16_t)(sign | (uint16_t)n);   // subnormal (n <= 128)
+    int ebits = qe + 7 + 127;
+    if (n == 256) { n = 128; ++ebits; }
+    if (ebits >= 255) return (uint16_t)(sign | 0x7F80u);
+    return (uint16_t)(sign | (uint16_t)(ebits << 7) | (uint16_t)(n - 128));
+}
+
+__device__ __forceinline__ double pow2_d(int e)
+{
+    e = e < -1022 ? -1022 : (e > 1023 ? 1023 : e);
+    return __longlong_as_double((long long)(e + 1023) << 52);
+}
+
+// ceil(log2(m)) for m > 0 given as the bit pattern of a non-negative double.
+__device__ __host__ __forceinline__ int ceil_log2_bits(unsigned long long b)
+{
+    const int E = (int)(b >> 52) & 0x7FF;
+    const unsigned long long f = b & 0x000FFFFFFFFFFFFFull;
+    if (E == 0) {                                 // subnormal
+#ifdef __CUDA_ARCH__
+        const int msb = 63 - __clzll((long long)f);
+#else
+        const int msb = 63 - __builtin_clzll(f);
+#endif
+        return ((f & (f - 1)) == 0 ? msb : msb + 1) - 1074;
+    }
+    return (E - 1023) + (f != 0 ? 1 : 0);
+}
+
+// One level of Eq. (fp64split) for one entry: Z = (R + 2^(v+45)) - 2^(v+45)
+// in FP64 round-to-nearest (no contraction), A_r = fl_BF16(Z),
+// R <- R - A_r.  Sets *bad if A_r is not exactly Z or is a nonzero value
+// below the normal BF16 range.
+__device__ __forceinline__ uint16_t f64_level(double &R, int v, bool &bad)
+{
+    if (v == kZeroLevel) return 0;                // residual is zero here
+    const double sigma = pow2_d(v + 45);
+    const double Z = __dsub_rn(__dadd_rn(R, sigma), sigma);
+    const float f = __double2float_rn(Z);
+    const uint32_t fb = __float_as_uint(f);
+    uint16_t s;
+    if ((double)f == Z && (fb & 0xFFFFu) == 0u && (Z == 0.0 || (fb & 0x7F800000u) != 0u) &&
+        (fb & 0x7F800000u) != 0x7F800000u) {
+        s = (uint16_t)(fb >> 16);
+    } else {
+        bad = true;
+        s = bf16_rne_f64(Z);
+    }
+    const double sv = (double)bf16_as_float(s);
+    R = __dsub_rn(R, sv);
+    return s;
+}
+
+// Final v^(0..5) of operand `slot` once verification and fix passes ran
+// (levels up to fix_from come from the verifier, later ones from the fix
+// maxima).  Levels past an all-zero residual are kZeroLevel.
+__device__ __forceinline__ void final_levels(const WsHeader *ws, int slot, int upto, int (&v)[6])
+{
+    const int ff = ws->fix_from[slot];
+    bool zero = false;
+    for (int r = 0; r < 6; ++r) {
+        if (r >= upto || zero) { v[r] = kZeroLevel; continue; }
+        if (r <= ff) v[r] = ws->v[slot][r];
+        else {
+            const unsigned long long m = ws->fixmax[slot][r];
+            v[r] = m ? ceil_log2_bits(m) : kZeroLevel;
+        }
+        if (v[r] == kZeroLevel) zero = true;
+    }
+}
+
+__device__ __forceinline__ double warp_max(double x)
+{
+    for (int o = 16; o; o >>= 1) x = fmax(x, __shfl_xor_sync(0xFFFFFFFFu, x, o));
+    return x;
+}
+
+// Block-wide max of one value per thread, then one atomicMax on the bit
+// pattern (non-negative doubles order like their bit patterns).
+__device__ __forceinline__ void block_max_to(double x, unsigned long long *dst, double *red)
+{
+    x = warp_max(x);
+    const int w = threadIdx.x >> 5;
+    if (lane_id() == 0) red[w] = x;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double m = 0.0;
+        for (int i = 0; i < kThreads / 32; ++i) m = fmax(m, red[i]);
+        if (m > 0.0) atomicMax(dst, (unsigned long long)__double_as_longlong(m));
+    }
+    __syncthreads();
+}
+
+// ------------------------------------------------------------ tile kernel
+// MODE 0: FP32 split.  MODE 1: FP64 speculative split (v^(r) = v0 - 8r,
+// records the maxima of |A^(r)|, r = 1..5).  MODE 2: FP64 rewrite with the
+// final levels (runs only when verification failed).
+template <typename T, int MODE, bool TRANSPOSE>
+__global__ void __launch_bounds__(kThreads)
+split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                  uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
+{
+    constexpr int NS = (MODE == 0) ? 3 : 6;
+    extern __shared__ __align__(16) uint16_t smdyn[];    // [NS][kTile][kSRow]
+    auto sm = [&](int r, int row, int col) -> uint16_t & {
+        return smdyn[((size_t)r * kTile + row) * kSRow + col];
+    };
+    __shared__ double red[kThreads / 32];
+
+    int v[6] = {0, 0, 0, 0, 0, 0};
+    if constexpr (MODE == 1) {
+        const unsigned long long m0 = ws->maxbits[slot][0];
+        const int v0 = m0 ? ceil_log2_bits(m0) : kZeroLevel;
+        for (int r = 0; r < 6; ++r) v[r] = (v0 == kZeroLevel) ? kZeroLevel : v0 - 8 * r;
+    } else if constexpr (MODE == 2) {
+        if (ws->fix_from[slot] >= 6) return;     // speculation held: nothing to redo
+        final_levels(ws, slot, 6, v);
+    }
+
+    double mx[5] = {0.0, 0.0, 0.0, 0.0, 0.0};
+    uint32_t badmask = 0, flagbits = 0;
+    const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;   // 16 x 16 threads
+
+    for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
+        const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
+        // ---- load, split, stage: thread (ty, tx) owns rows ty + 16p, columns 4tx..4tx+3
+#pragma unroll
+        for (int p = 0; p < 4; ++p) {
+            const int li = ty + 16 * p;
+            const int64_t gi = r0 + li;
+            T x[4];
+            const int64_t gj = c0 + 4 * tx;
+            const T *src = X + gi * ldx + gj;
+            const bool row_ok = gi < rows;
+            if (row_ok && gj + 4 <= cols && ((reinterpret_cast<uintptr_t>(src) & 15u) == 0)) {
+                if constexpr (sizeof(T) == 4) {
+                    const float4 q = *reinterpret_cast<const float4 *>(src);
+                    x[0] = q.x; x[1] = q.y; x[2] = q.z; x[3] = q.w;
+                } else {
+                    const double2 q0 = reinterpret_cast<const double2 *>(src)[0];
+                    const double2 q1 = reinterpret_cast<const double2 *>(src)[1];
+                    x[0] = q0.x; x[1] = q0.y; x[2] = q1.x; x[3] = q1.y;
+                }
+            } else {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) x[e] = (row_ok && gj + e < cols) ? src[e] : T(0);
+            }
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int lj = 4 * tx + e;
+                uint16_t s[NS];
+                if constexpr (MODE == 0) {
+                    float a = x[e];
+                    if (!isfinite(a)) flagbits |= EMU_FLAG_NONFINITE;
+#pragma unroll
+                    for (int r = 0; r < 3; ++r) {
+                        const uint32_t b = bf16_rne_f32bits(a);
+                        s[r] = (uint16_t)b;
+                        if ((b & 0x7F80u) == 0x7F80u) flagbits |= EMU_FLAG_SLICE;
+                        a = __fsub_rn(a, bf16_as_float(b));
+                    }
+                } else {
+                    double R = x[e];
+#pragma unroll
+                    for (int r = 0; r < 6; ++r) {
+                        if constexpr (MODE == 1) {
+                            if (r > 0) mx[r - 1] = fmax(mx[r - 1], fabs(R));
+                        }
+                        bool bad = false;
+                        s[r] = f64_level(R, v[r], bad);
+                        if (bad) badmask |= 1u << r;
+                    }
+                }
+#pragma unroll
+                for (int r = 0; r < NS; ++r) {
+                    if (TRANSPOSE) sm(r, lj, li) = s[r];
+                    else sm(r, li, lj) = s[r];
+                }
+            }
+        }
+        __syncthreads();
+        // ---- write plane rows in 16-byte chunks (8 BF16 per chunk)
+        const int64_t orow0 = TRANSPOSE ? c0 : r0, ocol0 = TRANSPOSE ? r0 : c0;
+        const int64_t orows = TRANSPOSE ? cols : rows, ocols = TRANSPOSE ? rows : cols;
+        for (int c = threadIdx.x; c < NS * kTile * (kTile / 8); c += kThreads) {
+            const int r = c / (kTile * (kTile / 8));
+            const int rem = c % (kTile * (kTile / 8));
+            const int orow = rem / (kTile / 8), ch = rem % (kTile / 8);
+            const int64_t go = orow0 + orow, gc = ocol0 + 8 * ch;
+            if (go >= orows || gc >= ocols) continue;
+            uint16_t *dst = comps + r * plane + go * ldcomp + gc;
+            const uint32_t *w = reinterpret_cast<const uint32_t *>(&sm(r, orow, 8 * ch));
+            if (gc + 8 <= ocols && ((reinterpret_cast<uintptr_t>(dst) & 15u) == 0)) {
+                *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+            } else {
+                for (int e = 0; e < 8 && gc + e < ocols; ++e) dst[e] = sm(r, orow, 8 * ch + e);
+            }
+        }
+        __syncthreads();
+    }
+
+    if constexpr (MODE == 0) {
+        flagbits = __reduce_or_sync(0xFFFFFFFFu, flagbits);
+        if (flagbits && lane_id() == 0) atomicOr(&ws->flags, flagbits);
+    } else {
+        badmask = __reduce_or_sync(0xFFFFFFFFu, badmask);
+        if (badmask && lane_id() == 0) atomicOr(&ws->slice_bad[slot], MODE == 1 ? badmask : badmask << 8);
+    }
+    if constexpr (MODE == 1) {
+#pragma unroll
+        for (int r = 0; r < 5; ++r) block_max_to(mx[r], &ws->maxbits[slot][r + 1], red);
+    }
+}
+
+// --------------------------------------------- row-segment FP64 passes
+// LEVEL = 0: max |x| and the input-domain checks of Eq. (bf16rangefp64).
+// LEVEL = L in 2..5: max |A^(L)| recomputed literally from x with the final
+// levels 0..L-1 (only when verification failed before level L).
+template <int LEVEL>
+__global__ void __launch_bounds__(kThreads)
+f64_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, WsHeader *ws,
+               int slot)
+{
+    __shared__ double red[kThreads / 32];
+    int v[6] = {0, 0, 0, 0, 0, 0};
+    if constexpr (LEVEL > 0) {
+        if (ws->fix_from[slot] >= LEVEL) return;
+        final_levels(ws, slot, LEVEL, v);
+        if (v[LEVEL - 1] == kZeroLevel) return;   // residual already zero
+    }
+    const double lo = 0x1p-126, hi = 0x1.fcp127;  // (2 - 2^-7) * 2^127
+    double m = 0.0;
+    uint32_t flagbits = 0;
+    const int64_t segs = (cols + 4 * kThreads - 1) / (4 * kThreads);
+    for (int64_t it = blockIdx.x; it < rows * segs; it += gridDim.x) {
+        const int64_t i = it / segs, j0 = (it % segs) * (4 * kThreads) + 4 * threadIdx.x;
+        const double *src = X + i * ldx + j0;
+        double x[4];
+        if (j0 + 4 <= cols && ((reinterpret_cast<uintptr_t>(src) & 15u) == 0)) {
+            const double2 q0 = reinterpret_cast<const double2 *>(src)[0];
+            const double2 q1 = reinterpret_cast<const double2 *>(src)[1];
+            x[0] = q0.x; x[1] = q0.y; x[2] = q1.x; x[3] = q1.y;
+        } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) x[e] = (j0 + e < cols) ? src[e] : 0.0;
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            double R = x[e];
+            if constexpr (LEVEL == 0) {
+                const double a = fabs(R);
+                if (!isfinite(R)) flagbits |= EMU_FLAG_NONFINITE;
+                else if (R != 0.0 && (a < lo || a > hi)) flagbits |= EMU_FLAG_RANGE;
+                if (!isnan(R)) m = fmax(m, a);
+            } else {
+                bool bad = false;
+#pragma unroll
+                for (int r = 0; r < LEVEL; ++r) (void)f64_level(R, v[r], bad);
+                m = fmax(m, fabs(R));
+            }
+        }
+    }
+    if constexpr (LEVEL == 0) {
+        flagbits = __reduce_or_sync(0xFFFFFFFFu, flagbits);
+        if (flagbits && lane_id() == 0) atomicOr(&ws->flags, flagbits);
+        block_max_to(m, &ws->maxbits[slot][0], red);
+    } else {
+        block_max_to(m, &ws->fixmax[slot][LEVEL], red);
+    }
+}
+
+// One thread: checks the speculative levels in order.  Level r's max from
+// the fused pass is literal as long as levels < r were right, so the first
+// mismatch r gives the true v^(r) directly; levels from r on are redone.
+__global__ void f64_verify_kernel(WsHeader *ws, int slot)
+{
+    int ff = 6;
+    const unsigned long long m0 = ws->maxbits[slot][0];
+    if (m0 == 0) {
+        for (int r = 0; r < 6; ++r) ws->v[slot][r] = kZeroLevel;
+    } else {
+        const int v0 = ceil_log2_bits(m0);
+        ws->v[slot][0] = v0;
+        bool zero = false;
+        for (int r = 1; r < 6; ++r) {
+            if (zero) { ws->v[slot][r] = kZeroLevel; continue; }
+            const unsigned long long m = ws->maxbits[slot][r];
+            if (m == 0) { ws->v[slot][r] = kZeroLevel; zero = true; continue; }
+            const int vr = ceil_log2_bits(m);
+            ws->v[slot][r] = vr;
+            if (vr != v0 - 8 * r) { ff = r; break; }
+        }
+    }
+    ws->fix_from[slot] = ff;
+}
+
+// One thread: publishes v_out and the slice flag of the levels actually used.
+__global__ void f64_finalize_kernel(WsHeader *ws, int slot, int32_t *v_out)
+{
+    int v[6];
+    final_levels(ws, slot, 6, v);
+    if (v_out)
+        for (int r = 0; r < 6; ++r) v_out[r] = v[r];
+    const int ff = ws->fix_from[slot];
+    const uint32_t keep = (1u << ff) - 1u;                       // levels taken from the fused pass
+    const uint32_t sb = ws->slice_bad[slot];
+    const uint32_t bad = (sb & keep & 0x3Fu) | ((sb >> 8) & ~keep & 0x3Fu);
+    if (bad) atomicOr(&ws->flags, (uint32_t)EMU_FLAG_SLICE);
+}
+
+size_t smem_bytes(int ns) { return (size_t)ns * kTile * kSRow * sizeof(uint16_t); }
+
+int grid_for(int64_t work_items, int max_blocks)
+{
+    int64_t g = work_items < 1 ? 1 : work_items;
+    return (int)(g < max_blocks ? g : max_blocks);
+}
+
+}  // namespace
+
+// ----------------------------------------------------------- host launchers
+cudaError_t launch_split_f32(const float *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
+                             uint16_t *comps, int64_t ldcomp, WsHeader *ws, cudaStream_t st)
+{
+    if (rows == 0 || cols == 0) return cudaSuccess;
+    const int64_t plane = (transpose ? cols : rows) * ldcomp;
+    const int64_t tiles = ((rows + kTile - 1) / kTile) * ((cols + kTile - 1) / kTile);
+    const int grid = grid_for(tiles, 152 * 16);
+    const size_t sm = smem_bytes(3);
+    if (transpose)
+        split_tile_kernel<float, 0, true><<<grid, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, 0);
+    else
+        split_tile_kernel<float, 0, false><<<grid, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, 0);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
+                             uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
+                             cudaStream_t st)
+{
+    const int64_t plane = (transpose ? cols : rows) * ldcomp;
+    if (rows > 0 && cols > 0) {
+        const int64_t segs = rows * ((cols + 4 * kThreads - 1) / (4 * kThreads));
+        const int gmax = grid_for(segs, 152 * 8);
+        const int64_t tiles = ((rows + kTile - 1) / kTile) * ((cols + kTile - 1) / kTile);
+        const int gt = grid_for(tiles, 152 * 8);
+        const size_t sm = smem_bytes(6);
+        cudaError_t e = cudaSuccess;
+        if (transpose) {
+            e = cudaFuncSetAttribute(split_tile_kernel<double, 1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+            if (e == cudaSuccess) e = cudaFuncSetAttribute(split_tile_kernel<double, 2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+        } else {
+            e = cudaFuncSetAttribute(split_tile_kernel<double, 1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+            if (e == cudaSuccess) e = cudaFuncSetAttribute(split_tile_kernel<double, 2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+        }
+        if (e != cudaSuccess) return e;
+        f64_max_kernel<0><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
+        if (transpose)
+            split_tile_kernel<double, 1, true><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot);
+        else
+            split_tile_kernel<double, 1, false><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot);
+        f64_verify_kernel<<<1, 1, 0, st>>>(ws, slot);
+        f64_max_kernel<2><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
+        f64_max_kernel<3><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
+        f64_max_kernel<4><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
+        f64_max_kernel<5><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
+        if (transpose)
+            split_tile_kernel<double, 2, true><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot);
+        else
+            split_tile_kernel<double, 2, false><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot);
+    } else {
+        f64_verify_kernel<<<1, 1, 0, st>>>(ws, slot);
+    }
+    f64_finalize_kernel<<<1, 1, 0, st>>>(ws, slot, v_out);
+    return cudaGetLastError();
+}
+
+}  // namespace emu

@@ -1,0 +1,66 @@
+"""The C-ABI library loads without a GPU, exports every entry point that
+include/emu.h declares, and rejects bad arguments on the host before any
+CUDA call."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2609_04663_gb300 as emu
+from paper_2609_04663_gb300 import _build
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "emu.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(emu_[a-z0-9_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    _build.build()
+    return emu.load()
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("emu_split_f32", "emu_split_f64", "emu_gemm_f32", "emu_gemm_f64",
+                     "emu_prodsum_f32", "emu_prodsum_f64", "emu_read_flags"):
+        assert required in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+        assert name in emu._SIGS, f"binding lacks {name}"
+
+
+def test_library_is_built_for_sm103a_only():
+    assert "arch=compute_103a,code=sm_103a" in " ".join(_build.ARCH)
+
+
+def test_status_strings_and_sizes(lib):
+    assert emu.emu_status_string(0) == b"ok"
+    assert emu.emu_status_string(3) == b"workspace too small"
+    assert emu.emu_split_workspace_bytes(64) >= 256
+    M, N, K = 300, 200, 700
+    ldk = emu.gemm_ldk(K)
+    assert ldk == 704
+    need = emu.emu_gemm_workspace_bytes(64, M, N, K)
+    assert need >= 6 * (M + N) * ldk * 2
+    assert emu.emu_gemm_workspace_bytes(32, M, N, K) < need
+
+
+def test_host_argument_checks_need_no_gpu(lib):
+    # every call below fails validation before touching CUDA
+    P = 16  # a dummy, 16-byte aligned, never dereferenced
+    assert emu.emu_gemm_f32(-1, 4, 4, P, 4, P, 4, P, 4, P, 1 << 20, None) == 1
+    assert emu.emu_gemm_f32(4, 4, 4, P, 3, P, 4, P, 4, P, 1 << 20, None) == 1       # lda < K
+    assert emu.emu_gemm_f64(4, 4, 4, P, 4, P, 4, P, 4, 7, P, 1 << 20, None) == 1    # nprod
+    assert emu.emu_gemm_f64(4, 4, 4, P, 4, P, 4, P, 4, 6, P, 16, None) == 3         # workspace
+    assert emu.emu_gemm_f32(1 << 31, 4, 4, P, 4, P, 4, P, 4, P, 1 << 62, None) == 5  # size limit
+    assert emu.emu_split_f64(P, 4, 4, 2, 0, P, 4, P, P, 4096, None) == 1              # ldx < cols
+    assert emu.emu_selftest_timeout(P, 4096, 0, None) == 1

@@ -1,0 +1,144 @@
+"""GPU split kernels against the oracle: bit-exact planes, levels and flags.
+
+Eq. (fp32split) and Eq. (fp64split) are integer-valued decisions on FP32/FP64
+arithmetic, so the bar is bit equality.  B operands are split transposed
+(K-major planes); they are compared with the oracle's planes transposed.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+import paper_2609_04663_gb300 as emu
+from helpers import device, planes_np, random_finite_f32, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dev():
+    return device()
+
+
+def _check_f32(X, dev, transpose, pad, ld_pad=0):
+    rows, cols = X.shape
+    rows_out, cols_out = (cols, rows) if transpose else (rows, cols)
+    ldcomp = cols_out + pad
+    planes, ws = emu.split_f32(to_dev(X, dev, ld_pad), transpose=transpose, ldcomp=ldcomp)
+    flags = emu.read_flags(ws)
+    want, wflags = oracle.split_f32(X)
+    if transpose:
+        want = want.transpose(0, 2, 1)
+    got = planes_np(planes)
+    assert flags == wflags
+    assert np.array_equal(got[:, :rows_out, :cols_out], want)
+    assert not got[:, :, cols_out:].any()          # padding untouched (zero-initialised)
+
+
+@pytest.mark.parametrize("shape", [(1, 1), (37, 129), (64, 64), (65, 3), (300, 700), (129, 1000)])
+@pytest.mark.parametrize("transpose", [False, True])
+def test_split_f32_uniform_bitexact(dev, shape, transpose):
+    X = synth.uniform_f32(7, 0, shape)
+    _check_f32(X, dev, transpose, pad=0)
+
+
+@pytest.mark.parametrize("transpose", [False, True])
+@pytest.mark.parametrize("pad,ld_pad", [(0, 0), (3, 5), (8, 4)])
+def test_split_f32_bit_patterns(dev, transpose, pad, ld_pad):
+    """Zeros, subnormals, ties and large magnitudes; odd leading dimensions."""
+    X = random_finite_f32((131, 203), 3)
+    _check_f32(X, dev, transpose, pad, ld_pad)
+
+
+def test_split_f32_flags(dev):
+    X = synth.uniform_f32(1, 0, (40, 50))
+    X[5, 7] = np.nan
+    planes, ws = emu.split_f32(to_dev(X, dev))
+    assert emu.read_flags(ws) & emu.FLAG_NONFINITE
+    X = synth.uniform_f32(1, 0, (40, 50))
+    X[0, 0] = np.float32(3.4e38)                   # the first slice rounds past the largest BF16
+    planes, ws = emu.split_f32(to_dev(X, dev))
+    assert emu.read_flags(ws) == oracle.split_f32(X)[1] == emu.FLAG_SLICE
+
+
+def _check_f64(X, dev, transpose, pad=0, ld_pad=0):
+    rows, cols = X.shape
+    rows_out, cols_out = (cols, rows) if transpose else (rows, cols)
+    planes, v, ws = emu.split_f64(to_dev(X, dev, ld_pad), transpose=transpose, ldcomp=cols_out + pad)
+    flags = emu.read_flags(ws)
+    want, wv, wflags = oracle.split_f64(X)
+    if transpose:
+        want = want.transpose(0, 2, 1)
+    assert flags == wflags
+    assert np.array_equal(v.cpu().numpy(), wv)
+    if wflags == 0:
+        assert np.array_equal(planes_np(planes)[:, :rows_out, :cols_out], want)
+    return wv
+
+
+@pytest.mark.parametrize("shape", [(1, 1), (12, 17), (64, 64), (300, 700), (257, 513)])
+@pytest.mark.parametrize("transpose", [False, True])
+def test_split_f64_uniform_bitexact(dev, shape, transpose):
+    wv = _check_f64(synth.uniform_f64(1, 0, shape), dev, transpose)
+    if shape[0] * shape[1] >= 4096:
+        assert list(np.diff(wv)) == [-8] * 5           # the speculative levels held
+
+
+@pytest.mark.parametrize("phi", [0.5, 2.0, 4.0])
+@pytest.mark.parametrize("transpose", [False, True])
+def test_split_f64_scaled_class_bitexact(dev, phi, transpose):
+    _check_f64(synth.scaled_f64(5, 0, phi, (190, 333)), dev, transpose, pad=5, ld_pad=3)
+
+
+@pytest.mark.parametrize("transpose", [False, True])
+def test_split_f64_fix_path_levels(dev, transpose):
+    """Inputs whose residual shrinks by far more than 2^-8 per level: the
+    speculative levels fail and the gated literal passes take over."""
+    rng = np.random.default_rng(9)
+    a = rng.integers(-127, 128, size=(150, 90)).astype(np.float64)
+    b = rng.integers(-127, 128, size=(150, 90)).astype(np.float64)
+    c = rng.integers(-127, 128, size=(150, 90)).astype(np.float64)
+    X = a * 2.0**10 + b * 2.0**-20 + c * 2.0**-50
+    X[0, 0] = 127 * 2.0**10
+    wv = _check_f64(X, dev, transpose)
+    assert wv[1] != wv[0] - 8                           # the fix path really ran
+    # integers: one slice, then zero levels (verifier stops at the zero residual)
+    Y = rng.integers(-100, 101, size=(70, 33)).astype(np.float64)
+    Y[3, 3] = 100.0
+    wv = _check_f64(Y, dev, transpose)
+    assert wv[1] == oracle.ZERO_LEVEL
+    _check_f64(np.zeros((20, 30)), dev, transpose)
+
+
+def test_split_f64_flags(dev):
+    X = synth.uniform_f64(3, 0, (33, 47))
+    for val in (np.nan, np.inf, 2.0**-127, 2.0**129):
+        Y = X.copy()
+        Y[4, 5] = val
+        planes, v, ws = emu.split_f64(to_dev(Y, dev))
+        assert emu.read_flags(ws) == oracle.split_f64(Y)[2] != 0, val
+    Y = np.full((4, 4), 2.0**-120)
+    Y[0, 0] = 2.0**-120 + 2.0**-140                    # a nonzero slice below 2^-126
+    _check_f64(Y, dev, False)
+    assert oracle.split_f64(Y)[2] == emu.FLAG_SLICE
+
+
+def test_split_fullsize_fp32_a_plane_bitexact(dev):
+    """Full size (M = K = 16384, FP32 sweep top): every plane bit-exact."""
+    n = 16384
+    A = synth.uniform_f32(n, 0, (n, n))
+    planes, ws = emu.split_f32(to_dev(A, dev))
+    assert emu.read_flags(ws) == 0
+    want, _ = oracle.split_f32(A)
+    assert np.array_equal(planes_np(planes), want)
+
+
+def test_split_fullsize_fp64_scaled_b_transposed_bitexact(dev):
+    """Full size (8192 x 8192, scaled class phi = 4), B orientation."""
+    n = 8192
+    B = synth.scaled_f64(5, n * n, 4.0, (n, n))
+    planes, v, ws = emu.split_f64(to_dev(B, dev), transpose=True)
+    assert emu.read_flags(ws) == 0
+    want, wv, _ = oracle.split_f64(B)
+    assert np.array_equal(v.cpu().numpy(), wv)
+    assert np.array_equal(planes_np(planes), want.transpose(0, 2, 1))
