@@ -1,0 +1,490 @@
+#!/usr/bin/env python3
+"""Throughput of the BF16 component-product GEMM emulation on GB300.
+
+Metric: emulated GEMM TFLOP/s = 2 M N K / t per step, where a step is one
+pass of the whole hot path on resident inputs: split A, split B (transposed)
+and the tensor-core product-sum.  The headline workload is FP32 mode (6
+products) at M = N = K = 16384, the top of the paper's square sweep; FP64
+mode at M = N = K = 4096 with 6, 10, 15 and 21 products and the other
+workloads are reported under "variants".
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   (the CPU oracle on the host cores)
+
+Multi-GPU (torchrun, one rank per GPU): every rank runs its own independent
+GEMM of the same size (replicas, weak scaling); no data moves between ranks.
+Rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "emulated GEMM TFLOP/s (2MNK/t) FP32-6p & FP64-6/10/15/21p; tensor-pipe % peak"
+DEFAULT_WORKLOAD = "fp32_n16384"
+L2_BYTES = 129 * 1024 * 1024
+
+
+# ------------------------------------------------------------ distributed
+def dist_init():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    """Max of a per-rank scalar (the slowest rank sets the job time)."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(flop_per_rank_step: float, steps: int, world: int, t_max_s: float) -> float:
+    """Whole-job TFLOP/s: the work of all ranks over the slowest rank's time."""
+    return flop_per_rank_step * steps * world / t_max_s / 1e12
+
+
+# ------------------------------------------------------------ clock sampler
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+                 "-i", str(self.gpu)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        for line in out.splitlines():
+            f = [t.strip() for t in line.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, val in zip(self.NAMES, f[4:8]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------ workloads
+def workload(name: str):
+    import synth
+    kind, M, N, K, seed, phi, nprods = synth.WORKLOADS[name]
+    return kind, M, N, K, seed, phi, nprods
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"bf16_sustained": p["bf16_tflops_sustained"], "bf16_burst": p["bf16_tflops"],
+                "hbm": p["hbm_gbs"], "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"bf16_sustained": 1700.0, "bf16_burst": 1900.0, "hbm": 6800.0, "source": "fallback"}
+
+
+def kernel_traffic(kernel: str, workload_name: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on
+    the current source of the kernel (else None)."""
+    src = os.path.join(ROOT, "paper_2609_04663_gb300", "csrc", "prodsum.cu")
+    try:
+        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        with open(os.path.join(ROOT, "profiles", "traffic.txt")) as f:
+            for line in f:
+                t = line.split()
+                if len(t) >= 4 and not line.startswith("#") and t[0] == kernel and t[1] == workload_name \
+                        and t[2] == digest:
+                    return float(t[3])
+    except OSError:
+        pass
+    return None
+
+
+class Case:
+    """Device-resident inputs, planes and output of one GEMM workload."""
+
+    def __init__(self, name: str, rank: int, nprod: int | None = None):
+        import numpy as np
+        import torch
+        import synth
+        import paper_2609_04663_gb300 as emu
+        self.emu, self.torch = emu, torch
+        self.name = name
+        kind, M, N, K, seed, phi, nprods = workload(name)
+        self.kind, self.M, self.N, self.K = kind, M, N, K
+        self.mode = 32 if kind == "f32" else 64
+        self.nprod = nprod or nprods[0]
+        # each rank draws its own problem (replicas): offset the seed by the rank
+        A, B = synth.gemm_inputs(kind, M, N, K, seed + 1000003 * rank, phi=phi)
+        self.A_host, self.B_host = A, B
+        dev = torch.device("cuda")
+        self.A = torch.from_numpy(A).to(dev)
+        self.B = torch.from_numpy(B).to(dev)
+        self.ldk = emu.gemm_ldk(K)
+        s = 3 if self.mode == 32 else 6
+        self.Ap = torch.empty((s, M, self.ldk), dtype=torch.int16, device=dev)
+        self.Bp = torch.empty((s, N, self.ldk), dtype=torch.int16, device=dev)
+        self.v = torch.empty(12, dtype=torch.int32, device=dev)
+        self.C = torch.empty((M, N), dtype=torch.float32 if self.mode == 32 else torch.float64, device=dev)
+        self.ws = emu.workspace(emu.emu_split_workspace_bytes(self.mode), dev)
+        self.gemm_ws = None
+        self.flop = 2.0 * M * N * K
+        self.exec_flop = self.flop * (6 if self.mode == 32 else self.nprod)
+        # kernels of ours per step: FP32 split = 1 launch, FP64 split = 9, product-sum = 1
+        self.launches = (2 * 1 + 1) if self.mode == 32 else (2 * 9 + 1)
+        del np
+
+    def split(self, stream):
+        emu, st = self.emu, stream.cuda_stream
+        ws, n = self.ws.data_ptr(), self.ws.numel()
+        if self.mode == 32:
+            r = emu.emu_split_f32(self.A.data_ptr(), self.M, self.K, self.A.stride(0), 0, self.Ap.data_ptr(),
+                                  self.ldk, ws, n, st)
+            r |= emu.emu_split_f32(self.B.data_ptr(), self.K, self.N, self.B.stride(0), 1, self.Bp.data_ptr(),
+                                   self.ldk, ws, n, st)
+        else:
+            r = emu.emu_split_f64(self.A.data_ptr(), self.M, self.K, self.A.stride(0), 0, self.Ap.data_ptr(),
+                                  self.ldk, self.v.data_ptr(), ws, n, st)
+            r |= emu.emu_split_f64(self.B.data_ptr(), self.K, self.N, self.B.stride(0), 1, self.Bp.data_ptr(),
+                                   self.ldk, self.v.data_ptr() + 24, ws, n, st)
+        assert r == 0, r
+
+    def prodsum(self, stream):
+        emu, st = self.emu, stream.cuda_stream
+        if self.mode == 32:
+            r = emu.emu_prodsum_f32(self.M, self.N, self.K, self.Ap.data_ptr(), self.Bp.data_ptr(), self.ldk,
+                                    self.C.data_ptr(), self.N, self.ws.data_ptr(), self.ws.numel(), st)
+        else:
+            r = emu.emu_prodsum_f64(self.M, self.N, self.K, self.Ap.data_ptr(), self.Bp.data_ptr(), self.ldk,
+                                    self.nprod, self.C.data_ptr(), self.N, self.ws.data_ptr(), self.ws.numel(), st)
+        assert r == 0, r
+
+    def split_bytes(self):
+        """Algorithmic HBM bytes of the two splits: FP32 4 B read + 6 B written
+        per entry; FP64 8 B (level-0 max) + 8 B (fused pass) read + 12 B written."""
+        per = 10 if self.mode == 32 else 28
+        return per * (self.M * self.K + self.K * self.N)
+
+
+def time_device(case: Case, steps: int, warmup: int, world: int, flush: bool):
+    """Time `steps` whole-path steps with CUDA events on the launching stream."""
+    torch = case.torch
+    stream = torch.cuda.current_stream()
+    scratch = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device="cuda") if flush else None
+    for _ in range(warmup):
+        case.split(stream)
+        case.prodsum(stream)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for i in range(steps):
+        if flush:
+            scratch.fill_(i & 0xFF)              # evict the previous step from L2 (not timed)
+        ev[i][0].record(stream)
+        case.split(stream)
+        ev[i][1].record(stream)
+        case.prodsum(stream)
+        ev[i][2].record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    split_ms = [a.elapsed_time(b) for a, b, _ in ev]
+    prod_ms = [b.elapsed_time(c) for _, b, c in ev]
+    step_ms = [a.elapsed_time(c) for a, _, c in ev]
+    return {"step_ms": step_ms, "split_ms": split_ms, "prodsum_ms": prod_ms, "wall_s": wall}
+
+
+def time_e2e(case: Case, steps: int, warmup: int, world: int):
+    """Same metric through the public C-ABI call (emu_gemm_*) with host
+    buffers: pinned H2D of A and B, the GEMM, D2H of C, all inside the timing."""
+    torch, emu = case.torch, case.emu
+    stream = torch.cuda.current_stream()
+    A_h = torch.from_numpy(case.A_host).pin_memory()
+    B_h = torch.from_numpy(case.B_host).pin_memory()
+    C_h = torch.empty(case.C.shape, dtype=case.C.dtype).pin_memory()
+    need = emu.emu_gemm_workspace_bytes(case.mode, case.M, case.N, case.K)
+    ws = emu.workspace(need, "cuda")
+
+    def step():
+        case.A.copy_(A_h, non_blocking=True)
+        case.B.copy_(B_h, non_blocking=True)
+        st = stream.cuda_stream
+        if case.mode == 32:
+            r = emu.emu_gemm_f32(case.M, case.N, case.K, case.A.data_ptr(), case.K, case.B.data_ptr(), case.N,
+                                 case.C.data_ptr(), case.N, ws.data_ptr(), ws.numel(), st)
+        else:
+            r = emu.emu_gemm_f64(case.M, case.N, case.K, case.A.data_ptr(), case.K, case.B.data_ptr(), case.N,
+                                 case.C.data_ptr(), case.N, case.nprod, ws.data_ptr(), ws.numel(), st)
+        assert r == 0, r
+        C_h.copy_(case.C, non_blocking=True)
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize()
+    barrier(world)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for _ in range(steps):
+        step()
+    end.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    t = max_over_ranks(start.elapsed_time(end) / 1e3, world)
+    h2d = case.A_host.nbytes + case.B_host.nbytes
+    d2h = C_h.numel() * C_h.element_size()
+    del ws, A_h, B_h, C_h
+    return {"value": job_throughput(case.flop, steps, world, t), "unit": "TFLOP/s",
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+
+
+# ------------------------------------------------------------ CPU oracle
+class OracleSampler:
+    """Times the CPU oracle (as it stands) on a bounded sample of a workload.
+
+    One sample: the split of B (FP32: a block of B's rows, scaled to all K
+    rows -- the FP32 split is elementwise; FP64: the whole of B, because its
+    levels are global), the split of A (FP32: the sampled rows; FP64: the
+    whole of A), each pro-rated to the sampled output rows, plus the
+    product-sum of the sampled rows.  Value = 2 * rows * N * K / time."""
+
+    def __init__(self, name: str, nprod: int | None = None):
+        import synth
+        kind, M, N, K, seed, phi, nprods = workload(name)
+        self.name, self.kind, self.M, self.N, self.K = name, kind, M, N, K
+        self.nprod = nprod or nprods[0]
+        self.A, self.B = synth.gemm_inputs(kind, M, N, K, seed, phi=phi)
+        self.rows = 2
+        self.Bp = None
+
+    def _split(self, X):
+        import oracle
+        return oracle.split_f32(X)[0] if self.kind == "f32" else oracle.split_f64(X)[0]
+
+    def sample(self, budget_s: float):
+        import numpy as np
+        import oracle
+        M, N, K = self.M, self.N, self.K
+        t0 = time.perf_counter()
+        if self.kind == "f32":
+            kb = min(K, 1024)
+            self._split(self.B[:kb])
+            t_b = (time.perf_counter() - t0) * K / kb
+            if self.Bp is None:
+                self.Bp = self._split(self.B)
+        else:
+            self.Bp = self._split(self.B)
+            t_b = time.perf_counter() - t0
+            t0 = time.perf_counter()
+            self.Ap = self._split(self.A)
+            t_a_full = time.perf_counter() - t0
+        while True:
+            sel = np.arange(self.rows)
+            t0 = time.perf_counter()
+            if self.kind == "f32":
+                oracle.prodsum_f32(self._split(self.A[sel]), self.Bp)
+            else:
+                oracle.prodsum_f64(self.Ap[:, sel], self.Bp, self.nprod)
+            t_rows = time.perf_counter() - t0
+            if t_rows >= budget_s / 3 or self.rows >= M:
+                break
+            self.rows = min(M, self.rows * 2)
+        share = self.rows / M
+        t = t_rows + t_b * share + (0.0 if self.kind == "f32" else t_a_full * share)
+        cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+        return {"value": 2.0 * self.rows * N * K / t / 1e12, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+                "sample": f"{self.rows} of {M} output rows of {self.name} (nprod "
+                          f"{6 if self.kind == 'f32' else self.nprod}); operand splits timed and pro-rated to "
+                          f"those rows; {t:.2f} s of CPU work"}
+
+
+def oracle_sample(name: str, target_s: float = 15.0):
+    return OracleSampler(name).sample(target_s)
+
+
+# ------------------------------------------------------------ arms
+def reference_arm(args, rank, world):
+    if rank != 0:
+        return 0
+    name = args.workload
+    kind, M, N, K, *_ = workload(name)
+    sampler = OracleSampler(name)
+    budget = min(args.ref_seconds, 120.0 / max(args.steps + args.warmup, 1))
+    for _ in range(args.warmup):
+        sampler.sample(budget)
+    vals = []
+    t_start = time.perf_counter()
+    for _ in range(args.steps):
+        vals.append(sampler.sample(budget))
+    wall = time.perf_counter() - t_start
+    v = statistics.mean(x["value"] for x in vals)
+    cpu = dict(vals[-1])
+    cpu["value"] = v
+    line = {
+        "impl": "reference", "metric": METRIC, "value": v, "unit": "TFLOP/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * wall / max(args.steps, 1),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32" if kind == "f32" else "f64", "data": "synthetic",
+        "config": {"workload": name, "M": M, "N": N, "K": K},
+        "cpu_baseline": cpu,
+        "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def gpu_arm(args, rank, world, local):
+    import torch
+    torch.cuda.set_device(local)
+    import __graft_entry__
+    __graft_entry__.build()
+    pk = peaks()
+    name = args.workload
+    case = Case(name, rank)
+    clocks = ClockSampler(local)
+    clocks.start()
+    res = time_device(case, args.steps, args.warmup, world, flush=False)
+    clk = clocks.stop()
+    t_job = max_over_ranks(sum(res["step_ms"]) / 1e3, world)
+    value = job_throughput(case.flop, args.steps, world, t_job)
+    prod_ms = statistics.mean(res["prodsum_ms"])
+    split_ms = statistics.mean(res["split_ms"])
+    achieved = case.exec_flop / (prod_ms / 1e3) / 1e12
+    # the timed region is well under the seconds-long loop of the sustained
+    # figure, so the (higher) burst peak is the denominator
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": pk["bf16_burst"], "unit": "TFLOP/s",
+                "frac": achieved / pk["bf16_burst"],
+                "peak_source": f"{pk['source']} bf16 burst (cuBLAS 8192^3); sustained {pk['bf16_sustained']}",
+                "kernel": "prodsum_f32_kernel" if case.mode == 32 else "prodsum_f64_kernel",
+                "traffic": kernel_traffic("prodsum_f32" if case.mode == 32 else "prodsum_f64", name)}
+    flags = case.emu.read_flags(case.ws)
+    e2e = None if args.no_e2e else time_e2e(case, max(2, min(args.steps, 5)), 1, world)
+    split_gbs = case.split_bytes() / (split_ms / 1e3) / 1e9
+    line = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * t_job / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": name, "mode": f"fp{case.mode}", "nprod": case.nprod if case.mode == 64 else 6,
+                   "M": case.M, "N": case.N, "K": case.K, "parallelism": f"replicas{world}",
+                   "l2": "inputs larger than L2 (no flush needed)"},
+        "breakdown": {"split_ms": split_ms, "prodsum_ms": prod_ms, "split_gbs": split_gbs,
+                      "split_frac_hbm": split_gbs / pk["hbm"], "executed_tflops": achieved,
+                      "effective_prodsum_only_tflops": case.flop / (prod_ms / 1e3) / 1e12},
+        "roofline": roofline, "clocks": clk, "e2e": e2e, "gpu_launches": case.launches * args.steps,
+        "flags": flags,
+    }
+    del case
+    torch.cuda.empty_cache()
+    if not args.no_variants:
+        line["variants"] = variants(args, rank, world, pk)
+    if rank == 0 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = oracle_sample(name, target_s=args.ref_seconds)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
+def variants(args, rank, world, pk):
+    """The other workloads, a few steps each, L2 flushed between steps."""
+    out = {}
+    todo = [("fp32_n8192", None), ("fp64_n4096", 6), ("fp64_n4096", 10), ("fp64_n4096", 15), ("fp64_n4096", 21)]
+    if args.all_variants:
+        todo += [("fp32_n1024", None), ("fp32_n2048", None), ("fp32_n4096", None), ("fp32_largek", None),
+                 ("fp64_scaled_phi4_n8192", 21), ("fp64_scaled_phi4_n8192", 10), ("fp64_largek", 21)]
+    torch = __import__("torch")
+    for name, nprod in todo:
+        case = Case(name, rank, nprod)
+        res = time_device(case, max(3, args.variant_steps), 2, world, flush=True)
+        t = max_over_ranks(sum(res["step_ms"]) / 1e3, world)
+        pm = statistics.mean(res["prodsum_ms"])
+        key = f"{name}" + (f"_np{case.nprod}" if case.mode == 64 else "")
+        out[key] = {"tflops": job_throughput(case.flop, len(res["step_ms"]), world, t),
+                    "ms_per_step": 1e3 * t / len(res["step_ms"]),
+                    "prodsum_ms": pm, "split_ms": statistics.mean(res["split_ms"]),
+                    "executed_tflops": case.exec_flop / (pm / 1e3) / 1e12,
+                    "frac_of_bf16_peak": case.exec_flop / (pm / 1e3) / 1e12 / pk["bf16_burst"],
+                    "flags": case.emu.read_flags(case.ws)}
+        del case
+        torch.cuda.empty_cache()
+    return out
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--variant-steps", type=int, default=5)
+    ap.add_argument("--all-variants", action="store_true")
+    ap.add_argument("--no-variants", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--ref-seconds", type=float, default=15.0)
+    args = ap.parse_args(argv)
+    if args.warmup < 3 and args.impl == "ours":
+        ap.error("--warmup must be at least 3")
+    rank, world, local = dist_init()
+    if args.impl == "reference":
+        return reference_arm(args, rank, world)
+    return gpu_arm(args, rank, world, local)
+
+
+if __name__ == "__main__":
+    sys.exit(main())
