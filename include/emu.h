@@ -137,6 +137,29 @@ emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
                            const uint16_t *Bcomps, int64_t ldcomp, int nprod, double *C,
                            int64_t ldc, void *ws, size_t ws_bytes, emu_stream_t stream);
 
+/* FP64-mode emulated GEMM that allocates nothing and takes no workspace.
+ * The paper has no counterpart: this entry point exists for callers that
+ * cannot allocate device memory -- plugins inside host programs that own the
+ * whole device memory budget and forbid allocation calls after start-up, or
+ * latency-critical paths that cannot accept the implicit synchronisation of
+ * cudaMalloc.  It computes exactly what emu_gemm_f64 computes (same kernels,
+ * same results), with its scratch (flag word, level maxima, BF16 planes) in a
+ * static device array of EMU_NOALLOC_SCRATCH_BYTES that every GPU loading
+ * the library holds until the library is unloaded.
+ * Limit: 512 + 12 * (M + N) * roundup(K, 8) bytes (256-byte rounding per
+ * operand) must fit the array, e.g. M = N = K = 1024; larger problems
+ * return EMU_ERR_UNSUPPORTED before any work is enqueued.
+ * flags_out: device pointer receiving the EMU_FLAG_* word of this call
+ * (may be NULL).  The first call on each device looks up the array's device
+ * address (with that device current); make that first call before any
+ * stream capture.  All calls on a device share the array: calls whose work
+ * may overlap on the GPU (different streams or host threads without
+ * ordering) race and must be serialised by the caller. */
+#define EMU_NOALLOC_SCRATCH_BYTES (32u << 20)
+emu_status emu_gemm_f64_noalloc(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda,
+                                const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,
+                                uint32_t *flags_out, emu_stream_t stream);
+
 /* Copies the flag word of the last call that used `ws` to *host_flags after
  * synchronising `stream`.  ws: device workspace; host_flags: host pointer. */
 emu_status emu_read_flags(const void *ws, uint32_t *host_flags, emu_stream_t stream);

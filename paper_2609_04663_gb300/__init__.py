@@ -35,6 +35,7 @@ _SIGS = {
     "emu_gemm_f64": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "size", "p"]),
     "emu_prodsum_f32": ("i", ["l", "l", "l", "p", "p", "l", "p", "l", "p", "size", "p"]),
     "emu_prodsum_f64": ("i", ["l", "l", "l", "p", "p", "l", "i", "p", "l", "p", "size", "p"]),
+    "emu_gemm_f64_noalloc": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "p"]),
     "emu_read_flags": ("i", ["p", "p", "p"]),
     "emu_selftest_timeout": ("i", ["p", "size", "u32", "p"]),
     "emu_status_string": ("str", ["i"]),
@@ -85,6 +86,7 @@ emu_gemm_f32 = _mk("emu_gemm_f32")
 emu_gemm_f64 = _mk("emu_gemm_f64")
 emu_prodsum_f32 = _mk("emu_prodsum_f32")
 emu_prodsum_f64 = _mk("emu_prodsum_f64")
+emu_gemm_f64_noalloc = _mk("emu_gemm_f64_noalloc")
 emu_read_flags = _mk("emu_read_flags")
 emu_selftest_timeout = _mk("emu_selftest_timeout")
 emu_status_string = _mk("emu_status_string")

@@ -1,0 +1,68 @@
+"""emu_gemm_f64_noalloc: the FP64-mode GEMM for callers that cannot allocate
+device memory (it keeps its scratch in a static device array instead of a
+caller-provided workspace).  It must give what emu_gemm_f64 gives -- FP64
+mode is bit-exact, so the bar here is equality -- on consecutive calls that
+reuse the shared array, and refuse problems too large for the array.
+
+This file is collected last on purpose: it also runs after every other test
+in the same process, and on its own in a fresh one."""
+import ctypes
+
+import numpy as np
+import pytest
+
+import synth
+import paper_2609_04663_gb300 as emu
+from helpers import device, to_dev
+
+pytestmark = pytest.mark.gpu
+
+SCRATCH_BYTES = 32 << 20
+
+
+def _noalloc(A, B, nprod, flags):
+    torch = emu._torch()
+    M, K = A.shape
+    N = B.shape[1]
+    C = torch.full((M, N), np.nan, dtype=torch.float64, device=A.device)
+    st = emu.emu_gemm_f64_noalloc(M, N, K, A.data_ptr(), A.stride(0), B.data_ptr(), B.stride(0), C.data_ptr(),
+                                  C.stride(0), nprod, flags.data_ptr(), emu._stream(None))
+    return st, C
+
+
+def test_noalloc_matches_workspace_entry_point_twice():
+    dev = device()
+    torch = emu._torch()
+    flags = torch.full((1,), 0xFFFF, dtype=torch.int32, device=dev)
+    # two calls in a row with different shapes and data reuse the shared scratch
+    for (M, N, K, seed, nprod) in [(200, 136, 300, 1, 21), (129, 257, 520, 2, 10)]:
+        A, B = synth.gemm_inputs("f64", M, N, K, seed)
+        Ad, Bd = to_dev(A, dev), to_dev(B, dev)
+        st, C = _noalloc(Ad, Bd, nprod, flags)
+        assert st == 0
+        Cref, ws = emu.gemm_f64(Ad, Bd, nprod)
+        assert emu.read_flags(ws) == 0
+        assert int(flags.item()) == 0
+        assert np.array_equal(C.cpu().numpy(), Cref.cpu().numpy())
+
+
+def test_noalloc_limit_and_flags():
+    dev = device()
+    torch = emu._torch()
+    flags = torch.zeros((1,), dtype=torch.int32, device=dev)
+    # largest square problem that fits: 512 + 2 * 12 * n * n <= 32 MiB  ->  n = 1024 fits, 1184 does not
+    n = 1024
+    assert 512 + 2 * 6 * n * n * 2 <= SCRATCH_BYTES
+    A, B = synth.gemm_inputs("f64", n, n, n, 3)
+    Ad, Bd = to_dev(A, dev), to_dev(B, dev)
+    st, C = _noalloc(Ad, Bd, 6, flags)
+    assert st == 0
+    Cref, _ = emu.gemm_f64(Ad, Bd, 6)
+    assert np.array_equal(C.cpu().numpy(), Cref.cpu().numpy())
+    big = torch.zeros((1184, 1184), dtype=torch.float64, device=dev)
+    st, _ = _noalloc(big, big, 6, flags)
+    assert st == 5                                       # EMU_ERR_UNSUPPORTED: beyond the static scratch
+    # a domain violation is reported through flags_out
+    A[5, 5] = 2.0**-130
+    st, _ = _noalloc(to_dev(A[:64, :64], dev), to_dev(B[:64, :64], dev), 6, flags)
+    assert st == 0 and int(flags.item()) & emu.FLAG_RANGE
