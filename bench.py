@@ -139,7 +139,7 @@ def peaks():
 def kernel_traffic(kernel: str, workload_name: str):
     """DRAM bytes per launch from the committed ncu summary, if it was taken on
     the current source of the kernel (else None)."""
-    src = os.path.join(ROOT, "paper_2609_04663_gb300", "csrc", "prodsum.cu")
+    src = os.path.join(ROOT, "paper_2609_04663_gb300", "csrc", kernel + ".cu")
     try:
         digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
         with open(os.path.join(ROOT, "profiles", "traffic.txt")) as f:
@@ -395,7 +395,7 @@ def gpu_arm(args, rank, world, local):
     __graft_entry__.build()
     pk = peaks()
     name = args.workload
-    case = Case(name, rank)
+    case = Case(name, rank, args.nprod)
     clocks = ClockSampler(local)
     clocks.start()
     res = time_device(case, args.steps, args.warmup, world, flush=False)
@@ -471,6 +471,7 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--nprod", type=int, default=None, help="FP64 product count (6, 10, 15, 21)")
     ap.add_argument("--variant-steps", type=int, default=5)
     ap.add_argument("--all-variants", action="store_true")
     ap.add_argument("--no-variants", action="store_true")

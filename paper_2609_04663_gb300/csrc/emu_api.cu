@@ -13,7 +13,25 @@ cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, int nprod, double *C, int64_t ldc, uint32_t *flags,
                                cudaStream_t st);
-cudaError_t launch_timeout_selftest(uint32_t *flags, uint32_t timeout_us, cudaStream_t st);
+
+// Watchdog self-test: one bounded wait on a barrier that nothing completes.
+namespace {
+__global__ void timeout_selftest_kernel(uint32_t *flags, unsigned long long limit_ns)
+{
+    __shared__ __align__(8) uint64_t bar;
+    const uint32_t b = smem_u32(&bar);
+    if (threadIdx.x == 0) { mbar_init(b, 1); fence_mbar_init(); }
+    __syncthreads();
+    if (threadIdx.x == 0) (void)mbar_wait(b, 0, flags, limit_ns);   // nothing ever arrives
+    __syncthreads();
+}
+}  // namespace
+
+cudaError_t launch_timeout_selftest(uint32_t *flags, uint32_t timeout_us, cudaStream_t st)
+{
+    timeout_selftest_kernel<<<1, 32, 0, st>>>(flags, 1000ull * timeout_us);
+    return cudaGetLastError();
+}
 }  // namespace emu
 
 using namespace emu;

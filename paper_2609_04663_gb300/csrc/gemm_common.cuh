@@ -1,0 +1,69 @@
+// Shared pieces of the tensor-core product-sum kernels: output-tile
+// rasterisation, the bounded drain of in-flight TMA copies, and the host-side
+// tensor-map encoding of a BF16 plane set.
+#pragma once
+
+#include "common.cuh"
+
+namespace emu {
+
+constexpr int kBM = 128;
+constexpr int kGroupM = 8;       // rasterisation: 8 tile rows walk the N tiles together
+
+__device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, int &tm, int &tn)
+{
+    const int group_size = kGroupM * tiles_n;
+    const int first_m = (tile / group_size) * kGroupM;
+    const int gm = min(tiles_m - first_m, kGroupM);
+    const int local = tile % group_size;
+    tm = first_m + local % gm;
+    tn = local / gm;
+}
+
+// Wait (bounded) for the TMA loads the producer issued that the MMA warp may
+// not have consumed: used only when a wait already timed out, so that no
+// copy into shared memory is left in flight when the CTA exits.
+__device__ __forceinline__ void drain_inflight(uint32_t full0, int stages, long issued, uint32_t *flags)
+{
+    for (long L = issued - stages < 0 ? 0 : issued - stages; L < issued; ++L)
+        (void)mbar_wait(full0 + 8u * (uint32_t)(L % stages), (uint32_t)((L / stages) & 1), flags, 100000000ull);
+}
+
+// ------------------------------------------------------------ host side
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
+                                   CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                   CUtensorMapFloatOOBfill);
+
+inline EncodeTiledFn encode_fn()
+{
+    static EncodeTiledFn fn = []() -> EncodeTiledFn {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            return nullptr;
+        return reinterpret_cast<EncodeTiledFn>(p);
+    }();
+    return fn;
+}
+
+// Tensor map over a plane set [S][rows][ldcomp] of BF16: dims (K, rows, S),
+// box (kb, box_rows, 1), swizzle matching a kb * 2-byte row.  Out-of-range
+// boxes (ragged M, N, K) read zeros.
+inline bool make_plane_map(CUtensorMap *map, const uint16_t *planes, int64_t K, int64_t rows, int S, int64_t ldcomp,
+                    int kb, int box_rows)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)K, (cuuint64_t)rows, (cuuint64_t)S};
+    cuuint64_t strides[2] = {(cuuint64_t)ldcomp * 2, (cuuint64_t)rows * ldcomp * 2};
+    cuuint32_t box[3] = {(cuuint32_t)kb, (cuuint32_t)box_rows, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    const CUtensorMapSwizzle swz = (kb == 64) ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<uint16_t *>(planes), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace emu
