@@ -209,7 +209,8 @@ class Case:
                                     self.C.data_ptr(), self.N, self.ws.data_ptr(), self.ws.numel(), st)
         else:
             r = emu.emu_prodsum_f64(self.M, self.N, self.K, self.Ap.data_ptr(), self.Bp.data_ptr(), self.ldk,
-                                    self.nprod, self.C.data_ptr(), self.N, self.ws.data_ptr(), self.ws.numel(), st)
+                                    self.v.data_ptr(), self.v.data_ptr() + 24, self.nprod, self.C.data_ptr(), self.N,
+                                    self.ws.data_ptr(), self.ws.numel(), st)
         assert r == 0, r
 
     def split_bytes(self):

@@ -11,8 +11,9 @@
  *   (Eq. (bf16rangefp64)).  Each operand is split into 6 BF16 slices by the
  *   fixed simplified Ozaki projection (Eq. (fp64split)); nprod = 6, 10, 15 or
  *   21 products (i + j < d, d = 3..6, Eq. (fp64productcounts)) are kept.  Each
- *   product is formed in FP32 per K-chunk of 256 and widened and accumulated
- *   in FP64 (Eq. (fp64reconstruction), Algorithm 2).
+ *   product is formed in FP32 per K-chunk of 256 (exact partials, summed
+ *   exactly) and widened and accumulated in FP64 (Eq. (fp64reconstruction),
+ *   Algorithm 2).
  *
  * Common conventions
  *   - Every pointer argument named as a matrix, plane set, workspace or v_out
@@ -115,10 +116,13 @@ emu_status emu_gemm_f32(int64_t M, int64_t N, int64_t K, const float *A, int64_t
                         size_t ws_bytes, emu_stream_t stream);
 
 /* FP64-mode emulated GEMM, Algorithm 2: C = A . B for FP64 inputs, nprod in
- * {6, 10, 15, 21}.  Per K-chunk of 256 each retained product's partial is
- * formed in FP32 on the tensor cores and added into an FP64 accumulator in
- * the oracle's order (chunk outer, diagonal order inner), so C equals the
- * oracle bit for bit. */
+ * {6, 10, 15, 21}.  Products are taken in Algorithm 2's diagonal order; for
+ * each, the FP32 component product fl32(A_i B_j) is formed on the tensor
+ * cores per K-chunk of 256 (every chunk partial is exact, Section 4.5), the
+ * partials are summed exactly, and the total is added once into the FP64
+ * result: C <- fl64(C + fl32(A_i B_j)).  C equals the oracle's product-outer
+ * order bit for bit.  C also serves as the FP64 accumulator while the kernel
+ * runs. */
 emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda,
                         const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,
                         void *ws, size_t ws_bytes, emu_stream_t stream);
@@ -130,12 +134,19 @@ emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
                            const uint16_t *Bcomps, int64_t ldcomp, float *C, int64_t ldc,
                            void *ws, size_t ws_bytes, emu_stream_t stream);
 
-/* Product-sum alone for FP64 mode, Eq. (fp64reconstruction): A planes
- * [6][M][ldcomp], B planes [6][N][ldcomp]; nprod in {6, 10, 15, 21}.
- * ws: at least emu_split_workspace_bytes(64). */
+/* Product-sum alone for FP64 mode, Eq. (fp64reconstruction), summed as in
+ * emu_gemm_f64: A planes [6][M][ldcomp], B planes [6][N][ldcomp]; nprod in
+ * {6, 10, 15, 21}.  vA, vB: the device arrays of level exponents v^(0..5)
+ * that emu_split_f64 wrote for A and for B (its v_out).  They give each
+ * product's unit, 2^(vA_i + vB_j - 16), which lets the kernel add a chunk
+ * partial with one FP32 addition while the running sum stays below 2^24
+ * units (provably exact); both may be NULL, and then every addition is done
+ * as an error-free TwoSum (same result, slower).  ws: at least
+ * emu_split_workspace_bytes(64). */
 emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acomps,
-                           const uint16_t *Bcomps, int64_t ldcomp, int nprod, double *C,
-                           int64_t ldc, void *ws, size_t ws_bytes, emu_stream_t stream);
+                           const uint16_t *Bcomps, int64_t ldcomp, const int32_t *vA,
+                           const int32_t *vB, int nprod, double *C, int64_t ldc, void *ws,
+                           size_t ws_bytes, emu_stream_t stream);
 
 /* FP64-mode emulated GEMM that allocates nothing and takes no workspace.
  * The paper has no counterpart: this entry point exists for callers that

@@ -30,6 +30,10 @@ FLAG_SLICE = 0x4
 ZERO_LEVEL = -(2 ** 31)
 KCHUNK = 256
 NPROD_TO_D = {6: 3, 10: 4, 15: 5, 21: 6}
+# FP64 summation orders of the exact chunk partials (see oracle.c)
+ORDER_CHUNK_OUTER = 0
+ORDER_PRODUCT_OUTER = 1
+ORDERS = {"chunk": ORDER_CHUNK_OUTER, "product": ORDER_PRODUCT_OUTER}
 
 
 def build(force: bool = False) -> str:
@@ -63,7 +67,7 @@ def _load():
         lib.oracle_products.argtypes = [i32, i32, vp]
         lib.oracle_products.restype = i32
         lib.oracle_prodsum_f32.argtypes = [i64, i64, i64, vp, vp, i64, i64, vp]
-        lib.oracle_prodsum_f64.argtypes = [i64, i64, i64, vp, vp, i32, i64, i64, vp, vp]
+        lib.oracle_prodsum_f64.argtypes = [i64, i64, i64, vp, vp, i32, i32, i64, i64, vp, vp]
         lib.oracle_ref_dd.argtypes = [i64, i64, i64, vp, i64, vp, i64, i64, i64, vp, vp]
         _lib = lib
     return _lib
@@ -127,8 +131,12 @@ def prodsum_f32(Ap: np.ndarray, Bp: np.ndarray, rows=None) -> np.ndarray:
     return C
 
 
-def prodsum_f64(Ap: np.ndarray, Bp: np.ndarray, nprod: int, rows=None, check_exact: bool = False):
-    """FP64-mode product-sum (Eq. (fp64reconstruction)); optionally counts inexact FP32 partials."""
+def prodsum_f64(Ap: np.ndarray, Bp: np.ndarray, nprod: int, rows=None, check_exact: bool = False,
+                order: str = "product"):
+    """FP64-mode product-sum (Eq. (fp64reconstruction)); order "product"
+    (Algorithm 2 as written, chunk partials summed exactly per product) or
+    "chunk" (chunk outer, every partial added in FP64).  Optionally counts
+    inexact FP32 partials."""
     Ap = np.ascontiguousarray(Ap, dtype=np.uint16)
     Bp = np.ascontiguousarray(Bp, dtype=np.uint16)
     _, M, K = Ap.shape
@@ -136,7 +144,7 @@ def prodsum_f64(Ap: np.ndarray, Bp: np.ndarray, nprod: int, rows=None, check_exa
     r0, r1 = (0, M) if rows is None else rows
     C = np.empty((r1 - r0, N), dtype=np.float64)
     bad = ctypes.c_int64(-1)
-    _load().oracle_prodsum_f64(M, N, K, Ap.ctypes.data, Bp.ctypes.data, int(nprod), r0, r1 - r0,
+    _load().oracle_prodsum_f64(M, N, K, Ap.ctypes.data, Bp.ctypes.data, int(nprod), ORDERS[order], r0, r1 - r0,
                                C.ctypes.data, ctypes.byref(bad) if check_exact else None)
     return (C, int(bad.value)) if check_exact else C
 
@@ -149,11 +157,11 @@ def gemm_f32(A: np.ndarray, B: np.ndarray, rows=None):
     return prodsum_f32(Ap, Bp), fa | fb
 
 
-def gemm_f64(A: np.ndarray, B: np.ndarray, nprod: int, rows=None):
+def gemm_f64(A: np.ndarray, B: np.ndarray, nprod: int, rows=None, order: str = "product"):
     """Algorithm 2 end to end (the split of A is global, so A is split whole)."""
     Ap, _, fa = split_f64(A)
     Bp, _, fb = split_f64(B)
-    return prodsum_f64(Ap, Bp, nprod, rows=rows), fa | fb
+    return prodsum_f64(Ap, Bp, nprod, rows=rows, order=order), fa | fb
 
 
 def ref_dd(A: np.ndarray, B: np.ndarray, rows=None):

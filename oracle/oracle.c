@@ -28,9 +28,14 @@
  *     K step in the operand-reuse order of Eq. (fp32reuseorder), one FP32
  *     accumulator per chunk, chunk results added into an FP32 output
  *     accumulator (Section 5.3, reconstruction of the FP32 path).
- *   - FP64 mode: chunk outer, products inner in diagonal order (l ascending,
- *     i ascending within a diagonal), each FP32 chunk partial widened and
- *     added in FP64 (Algorithm 2, Eq. (fp64reconstruction), Section 5.3).
+ *   - FP64 mode, two summation orders of the same exact FP32 chunk partials:
+ *     ORDER_CHUNK_OUTER: chunk outer, products inner in diagonal order (l
+ *       ascending, i ascending within a diagonal), each partial widened and
+ *       added in FP64 (the per-panel reconstruction of Section 5.3);
+ *     ORDER_PRODUCT_OUTER: products in diagonal order outer, as Algorithm 2
+ *       is written (C <- fl64(C + fl32(A_i B_j))): the FP32 component product
+ *       is formed per K-chunk and its chunk partials are summed exactly (they
+ *       are integers in one unit, see oracle_prodsum_f64), then added once.
  */
 #include <float.h>
 #include <math.h>
@@ -43,6 +48,8 @@
 #define ORACLE_FLAG_SLICE     0x4u /* a slice is not a normal BF16 value (or is non-finite) */
 
 #define ORACLE_ZERO_LEVEL INT32_MIN /* v^(r) of an all-zero residual */
+#define ORACLE_ORDER_CHUNK_OUTER 0
+#define ORACLE_ORDER_PRODUCT_OUTER 1
 #define ORACLE_KCHUNK 256           /* B_K of Section 5.1 */
 
 /* ------------------------------------------------------------------------ */
@@ -270,40 +277,52 @@ void oracle_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, con
 }
 
 /* ------------------------------------------------------------------------ */
-/* FP64-mode product-sum, Eq. (fp64reconstruction), Algorithm 2: for every   */
-/* K-chunk and every selected pair (i_q, j_q) in executed order, the chunk   */
-/* partial P = fl32(A_i B_j) is formed in FP32, widened exactly, and added   */
-/* into the FP64 accumulator.  If n_inexact is non-NULL each FP32 partial is */
-/* also formed in FP64 and the number of partials that differ is counted:    */
-/* Section 4.5 says BF16 products are exact in FP32; with slices on the grid */
-/* of Eq. (fp64split) every chunk partial is exact as well.                 */
+/* FP64-mode product-sum, Eq. (fp64reconstruction), Algorithm 2.  Every      */
+/* chunk partial P = fl32(sum_k A_i B_j) is formed in FP32 (k ascending).    */
+/* Slices lie on the grid of Eq. (fp64split): integers times 2^(v-8) of     */
+/* magnitude <= 256, so a BF16 product is <= 2^16 units and a 256-long chunk */
+/* <= 2^24 units: P is exact (Section 4.5 extended to the chunk).            */
+/*   order 0 (chunk outer): for chunk, for pair: C = fl64(C + (double)P).    */
+/*   order 1 (product outer): for pair: S = sum over chunks of (double)P --  */
+/*     exact in FP64, a sum of integers in one unit below 2^53 units -- then */
+/*     C = fl64(C + S).                                                      */
+/* If n_inexact is non-NULL each partial is also formed in FP64 and the     */
+/* number of partials that differ is counted.                               */
 /* ------------------------------------------------------------------------ */
 void oracle_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
-                        int nprod, int64_t r0, int64_t nr, double *C, int64_t *n_inexact)
+                        int nprod, int order, int64_t r0, int64_t nr, double *C, int64_t *n_inexact)
 {
     int pairs[42];
     const int np = oracle_products(64, nprod, pairs);
     if (np < 0) return;
     float *a = expand_a(Ap, 6, M, K, r0, nr);
     float *b = expand_bt(Bp, 6, K, N);
+    const int64_t nch = (K + ORACLE_KCHUNK - 1) / ORACLE_KCHUNK;
     int64_t bad = 0;
     #pragma omp parallel for collapse(2) schedule(dynamic, 16) reduction(+:bad)
     for (int64_t i = 0; i < nr; ++i) {
         for (int64_t n = 0; n < N; ++n) {
             double c64 = 0.0;
-            for (int64_t c0 = 0; c0 < K; c0 += ORACLE_KCHUNK) {
+            double s = 0.0;
+            for (int64_t t = 0; t < nch * np; ++t) {
+                const int64_t c = (order == ORACLE_ORDER_CHUNK_OUTER) ? t / np : t % nch;
+                const int q = (int)((order == ORACLE_ORDER_CHUNK_OUTER) ? t % np : t / nch);
+                const int64_t c0 = c * ORACLE_KCHUNK;
                 const int64_t c1 = (c0 + ORACLE_KCHUNK < K) ? c0 + ORACLE_KCHUNK : K;
-                for (int q = 0; q < np; ++q) {
-                    const float *ai = a + (pairs[2 * q] * nr + i) * K;
-                    const float *bj = b + (pairs[2 * q + 1] * N + n) * K;
-                    float p = 0.0f;
-                    for (int64_t k = c0; k < c1; ++k) p = p + ai[k] * bj[k];
-                    if (n_inexact) {
-                        double pd = 0.0;
-                        for (int64_t k = c0; k < c1; ++k) pd = pd + (double)ai[k] * (double)bj[k];
-                        if ((double)p != pd) ++bad;
-                    }
+                const float *ai = a + (pairs[2 * q] * nr + i) * K;
+                const float *bj = b + (pairs[2 * q + 1] * N + n) * K;
+                float p = 0.0f;
+                for (int64_t k = c0; k < c1; ++k) p = p + ai[k] * bj[k];
+                if (n_inexact) {
+                    double pd = 0.0;
+                    for (int64_t k = c0; k < c1; ++k) pd = pd + (double)ai[k] * (double)bj[k];
+                    if ((double)p != pd) ++bad;
+                }
+                if (order == ORACLE_ORDER_CHUNK_OUTER) {
                     c64 = c64 + (double)p;
+                } else {
+                    s = s + (double)p;                       /* exact */
+                    if (c == nch - 1) { c64 = c64 + s; s = 0.0; }
                 }
             }
             C[i * N + n] = c64;

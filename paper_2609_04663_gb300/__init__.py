@@ -34,7 +34,7 @@ _SIGS = {
     "emu_gemm_f32": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "p", "size", "p"]),
     "emu_gemm_f64": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "size", "p"]),
     "emu_prodsum_f32": ("i", ["l", "l", "l", "p", "p", "l", "p", "l", "p", "size", "p"]),
-    "emu_prodsum_f64": ("i", ["l", "l", "l", "p", "p", "l", "i", "p", "l", "p", "size", "p"]),
+    "emu_prodsum_f64": ("i", ["l", "l", "l", "p", "p", "l", "p", "p", "i", "p", "l", "p", "size", "p"]),
     "emu_gemm_f64_noalloc": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "p"]),
     "emu_read_flags": ("i", ["p", "p", "p"]),
     "emu_selftest_timeout": ("i", ["p", "size", "u32", "p"]),
@@ -187,11 +187,14 @@ def prodsum_f32(Ap, Bp, M: int, N: int, K: int, C=None, ws=None, stream=None):
     return C, ws
 
 
-def prodsum_f64(Ap, Bp, M: int, N: int, K: int, nprod: int, C=None, ws=None, stream=None):
-    """FP64-mode product-sum alone from planes Ap [6, M, ldcomp], Bp [6, N, ldcomp]."""
+def prodsum_f64(Ap, Bp, M: int, N: int, K: int, nprod: int, vA=None, vB=None, C=None, ws=None, stream=None):
+    """FP64-mode product-sum alone from planes Ap [6, M, ldcomp], Bp [6, N, ldcomp];
+    vA, vB: the level exponents emu_split_f64 returned for A and B (or None)."""
     torch = _torch()
     C = C if C is not None else torch.empty((M, N), dtype=torch.float64, device=Ap.device)
     ws = ws if ws is not None else workspace(emu_split_workspace_bytes(64), Ap.device)
-    _check(emu_prodsum_f64(M, N, K, Ap.data_ptr(), Bp.data_ptr(), Ap.shape[2], int(nprod), C.data_ptr(),
-                           C.stride(0), ws.data_ptr(), ws.numel(), _stream(stream)), "emu_prodsum_f64")
+    _check(emu_prodsum_f64(M, N, K, Ap.data_ptr(), Bp.data_ptr(), Ap.shape[2],
+                           vA.data_ptr() if vA is not None else None, vB.data_ptr() if vB is not None else None,
+                           int(nprod), C.data_ptr(), C.stride(0), ws.data_ptr(), ws.numel(), _stream(stream)),
+           "emu_prodsum_f64")
     return C, ws

@@ -23,6 +23,7 @@ struct WsHeader {
     int32_t v[2][6];                      // final level exponents
     int32_t fix_from[2];                  // first level the fix passes redo (6 = none)
     uint32_t slice_bad[2];                // spec pass: bit r set = slice violation at level r
+    int32_t vout[2][6];                   // final level exponents as published by the split
 };
 constexpr size_t kWsHeaderBytes = 512;
 static_assert(sizeof(WsHeader) <= kWsHeaderBytes, "workspace header too large");

@@ -11,8 +11,8 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
 cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st);
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
-                               int64_t ldcomp, int nprod, double *C, int64_t ldc, uint32_t *flags,
-                               cudaStream_t st);
+                               int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
+                               int64_t ldc, uint32_t *flags, cudaStream_t st);
 
 // Watchdog self-test: one bounded wait on a barrier that nothing completes.
 namespace {
@@ -166,9 +166,10 @@ emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_
     const int64_t ldk = gemm_ldk(K);
     uint16_t *Ap = reinterpret_cast<uint16_t *>(static_cast<char *>(ws) + kWsHeaderBytes);
     uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(6 * M * ldk * 2, 256));
-    e = launch_split_f64(A, M, K, lda, false, Ap, ldk, nullptr, h, 0, st);
-    if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, nullptr, h, 1, st);
-    if (e == cudaSuccess) e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, nprod, C, ldc, &h->flags, st);
+    e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st);
+    if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st);
+    if (e == cudaSuccess)
+        e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, C, ldc, &h->flags, st);
     return cuda_status(e);
 }
 
@@ -191,8 +192,8 @@ emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
 }
 
 emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acomps, const uint16_t *Bcomps,
-                           int64_t ldcomp, int nprod, double *C, int64_t ldc, void *ws, size_t ws_bytes,
-                           emu_stream_t stream)
+                           int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
+                           int64_t ldc, void *ws, size_t ws_bytes, emu_stream_t stream)
 {
     if (M < 0 || N < 0 || K < 0 || ldc < (N > 0 ? N : 1) || !ws) return EMU_ERR_INVALID_ARG;
     if (nprod != 6 && nprod != 10 && nprod != 15 && nprod != 21) return EMU_ERR_INVALID_ARG;
@@ -207,7 +208,8 @@ emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
     if (K == 0) return zero_c(C, M, N, ldc, st);
     emu_status s = check_planes(Acomps, Bcomps, ldcomp, K);
     if (s != EMU_OK) return s;
-    return cuda_status(launch_prodsum_f64(M, N, K, Acomps, Bcomps, ldcomp, nprod, C, ldc, &h->flags, st));
+    if ((vA == nullptr) != (vB == nullptr)) return EMU_ERR_INVALID_ARG;
+    return cuda_status(launch_prodsum_f64(M, N, K, Acomps, Bcomps, ldcomp, vA, vB, nprod, C, ldc, &h->flags, st));
 }
 
 emu_status emu_read_flags(const void *ws, uint32_t *host_flags, emu_stream_t stream)

@@ -23,8 +23,8 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
                              uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
                              cudaStream_t st);
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
-                               int64_t ldcomp, int nprod, double *C, int64_t ldc, uint32_t *flags,
-                               cudaStream_t st);
+                               int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
+                               int64_t ldc, uint32_t *flags, cudaStream_t st);
 }  // namespace emu
 
 using namespace emu;
@@ -88,9 +88,10 @@ extern "C" emu_status emu_gemm_f64_noalloc(int64_t M, int64_t N, int64_t K, cons
         } else {
             uint16_t *Ap = reinterpret_cast<uint16_t *>(scratch + kWsHeaderBytes);
             uint16_t *Bp = reinterpret_cast<uint16_t *>(scratch + kWsHeaderBytes + a_bytes);
-            e = launch_split_f64(A, M, K, lda, false, Ap, ldk, nullptr, h, 0, st);
-            if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, nullptr, h, 1, st);
-            if (e == cudaSuccess) e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, nprod, C, ldc, &h->flags, st);
+            e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st);
+            if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st);
+            if (e == cudaSuccess)
+                e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, C, ldc, &h->flags, st);
         }
     }
     if (e == cudaSuccess && flags_out)

@@ -1,4 +1,27 @@
 // FP64-mode tensor-core product-sum, Eq. (fp64reconstruction) / Algorithm 2.
+//
+// Products are taken in Algorithm 2's diagonal order (outer loop); for each
+// product the K dimension is walked in chunks of 256 (B_K of Section 5.1).
+// Every chunk partial fl32(A_i B_j) is formed on the tensor cores in its own
+// TMEM buffer (two rotating 128-column buffers).  The partials are exact:
+// slice entries are integers times 2^(v-8) of magnitude <= 256, so a chunk
+// partial is an integer of at most 2^24 units.  Sixteen drain warps add the
+// partials of one product exactly in FP32: the running sum hi stays in
+// registers, and while it stays below 2^24 units (known from the split's level
+// exponents) a plain FP32 addition is exact.  Past that bound the error of
+// each addition is recovered with Knuth's TwoSum and summed into a low part
+// kept in the output buffer C, which is free scratch until the last product
+// (uniform data never gets there).
+// FP32 adds only, so GB300's slow FP64 pipe is not touched per chunk.  When
+// the product is complete, hi + lo is widened (exact; the common hi-only case
+// by integer bit operations) and added once into the FP64 accumulator in the
+// upper 256 TMEM columns: C <- fl64(C + fl32(A_i B_j)), Algorithm 2's step.
+// The result is bit-identical to the oracle in its product-outer order.
+//
+// Warp roles: warp 0 lane 0 issues TMA loads, warp 1 owns TMEM and lane 0
+// issues the MMAs, warps 4-19 drain (setmaxnreg moves registers from the
+// control warpgroup to the four drain warpgroups).  Every wait is bounded and reports
+// EMU_FLAG_TIMEOUT instead of hanging.
 #include "gemm_common.cuh"
 
 namespace emu {
@@ -11,22 +34,95 @@ __constant__ int8_t kDiag[21][2] = {{0, 0}, {0, 1}, {1, 0}, {0, 2}, {1, 1}, {2, 
                                     {1, 2}, {2, 1}, {3, 0}, {0, 4}, {1, 3}, {2, 2}, {3, 1},
                                     {4, 0}, {0, 5}, {1, 4}, {2, 3}, {3, 2}, {4, 1}, {5, 0}};
 
-// ===================================================================== FP64
 struct F64Cfg {
-    static constexpr int BN = 128, KB = 64, STAGES = 6, NBUF = 4;
-    static constexpr int A_TILE = kBM * KB * 2, B_TILE = BN * KB * 2;
+    // A stage holds SUB K-blocks of 64 (one 128-byte swizzle row each) of the
+    // A slice and of the B slice: 64 KB, eight MMAs, so the single-thread
+    // producer and MMA loops pay their per-stage overhead once per 128 of K.
+    static constexpr int BN = 128, KB = 64, SUB = 2, STAGES = 3, NBUF = 2;
+    static constexpr int KSPAN = KB * SUB;                          // K per stage
+    static constexpr int A_SUB = kBM * KB * 2, B_SUB = BN * KB * 2; // one 64-wide K-block tile
+    static constexpr int A_TILE = A_SUB * SUB, B_TILE = B_SUB * SUB;
     static constexpr int STAGE = A_TILE + B_TILE;
-    static constexpr uint32_t SWZ = 2u, SBO = 1024u;
+    static constexpr uint32_t SWZ = 2u, SBO = 1024u;              // 128-byte swizzle
     static constexpr int BAR_OFF = STAGES * STAGE;
     static constexpr int SMEM = BAR_OFF + 256 + 1024;
-    static constexpr int DRAIN_WARPS = 8, THREADS = 32 * (2 + DRAIN_WARPS);
-    static constexpr int COLS_PER_WARP = BN / (DRAIN_WARPS / 4);   // 64
+    // warpgroup 0: TMA producer (warp 0), MMA issuer + TMEM owner (warp 1),
+    // two idle warps; warpgroups 1-4: sixteen drain warps, four per TMEM lane
+    // quarter, 32 columns each.
+    static constexpr int DRAIN_WARPS = 16, THREADS = 640, FIRST_DRAIN = 4;
+    static constexpr int COLS = BN / (DRAIN_WARPS / 4);            // 32 columns per drain thread
+    // Register split: the launch reserves 640 x 96 (five warps per SMSP);
+    // warpgroup 0 drops to 32, the drain warpgroups rise to 112:
+    // 128 x 32 + 512 x 112 = 61440 = 640 x 96.
+    static constexpr int REG_CTRL = 32, REG_DRAIN = 112, REG_LAUNCH = 96;
+    static constexpr uint32_t ACC_COL = NBUF * BN;                 // FP64 accumulator: 2 words per column
 };
+static_assert(F64Cfg::ACC_COL + 2 * F64Cfg::BN == 512, "TMEM budget: 2 partial buffers + FP64 accumulator");
+static_assert(128 * F64Cfg::REG_CTRL + 512 * F64Cfg::REG_DRAIN <= F64Cfg::THREADS * F64Cfg::REG_LAUNCH,
+              "setmaxnreg split exceeds the registers reserved at launch");
+
+template <uint32_t R> __device__ __forceinline__ void regs_dec() { asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R)); }
+template <uint32_t R> __device__ __forceinline__ void regs_inc() { asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(R)); }
+
+// Exact FP32 -> FP64 widening of a normal or zero value by bit operations
+// (rebias the exponent, shift the significand); other values take the
+// conversion instruction.
+__device__ __forceinline__ double widen_exact(float x)
+{
+    const uint32_t u = __float_as_uint(x);
+    const uint32_t ex = (u >> 23) & 0xFFu;
+    if ((u & 0x7FFFFFFFu) == 0u) return __hiloint2double((int)(u & 0x80000000u), 0);
+    if (ex == 0u || ex == 0xFFu) return (double)x;
+    return __hiloint2double((int)((u & 0x80000000u) | ((ex + 896u) << 20) | ((u & 0x7FFFFFu) >> 3)), (int)(u << 29));
+}
+
+
+// Largest running-sum magnitude below which adding a chunk partial of product
+// (i, j) in FP32 is provably exact: every partial is an integer multiple of the
+// unit u = 2^(vA_i + vB_j - 16), so any sum of magnitude below 2^24 u is
+// representable, and rounding is monotone, so a rounded sum below 2^24 u was
+// exact.  0 (always take the error-free path) when the levels are unknown or
+// the bound is not a normal float; +inf for a product of an all-zero slice.
+__device__ __forceinline__ float exact_bound(const int32_t *vA, const int32_t *vB, int i, int j)
+{
+    if (!vA) return 0.0f;
+    const int a = vA[i], b = vB[j];
+    if (a == kZeroLevel || b == kZeroLevel) return __int_as_float(0x7F800000);
+    const int e = a + b + 8;                          // 2^24 * 2^(a + b - 16)
+    if (e < -126 || e > 127) return 0.0f;
+    return __int_as_float((e + 127) << 23);
+}
+
+// 16 consecutive 32-bit TMEM columns of this thread's lane: load / store.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16])
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+        ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+          "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
 
 template <int NPROD>
 __global__ void __launch_bounds__(F64Cfg::THREADS, 1)
 prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   int M, int N, int K, double *__restrict__ C, int64_t ldc, uint32_t *flags)
+                   int M, int N, int K, const int32_t *__restrict__ vA, const int32_t *__restrict__ vB,
+                   double *__restrict__ C, int64_t ldc, uint32_t *flags)
 {
     using Cfg = F64Cfg;
     extern __shared__ uint8_t smem_raw[];
@@ -45,7 +141,7 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     tile_coords(blockIdx.x, tiles_m, tiles_n, tm, tn);
     const int m0 = tm * kBM, n0 = tn * Cfg::BN;
     const int nch = (K + kKChunk - 1) / kKChunk;
-    const int nt = nch * NPROD;                   // (chunk, pair) partials of this tile
+    const int nt = NPROD * nch;                   // partials of this tile, product-major
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < Cfg::STAGES; ++s) { mbar_init(full0 + 8u * s, 1); mbar_init(empty0 + 8u * s, 1); }
@@ -61,92 +157,159 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 0 && lane == 0) {
-        // ---------------- TMA producer: for chunk, for pair, for K-block
-        long L = 0;
+    if (warp < Cfg::FIRST_DRAIN) {
+      regs_dec<Cfg::REG_CTRL>();
+      if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer: for product, for chunk, for K-span of the chunk
+        int L = 0, s = 0;
+        uint32_t ph = 0;
         bool ok = true;
-        for (int t = 0; t < nt && ok; ++t) {
-            const int c = t / NPROD, q = t % NPROD;
-            const int kbn = min(kKChunk / Cfg::KB, (K - c * kKChunk + Cfg::KB - 1) / Cfg::KB);
-            for (int kb = 0; kb < kbn; ++kb, ++L) {
-                const int s = (int)(L % Cfg::STAGES);
-                if (!(ok = mbar_wait(empty0 + 8u * s, (uint32_t)(((L / Cfg::STAGES) & 1) ^ 1), flags))) break;
-                const uint32_t st = base + (uint32_t)(s * Cfg::STAGE), fb = full0 + 8u * s;
-                const int k0 = c * kKChunk + kb * Cfg::KB;
-                mbar_arrive_expect_tx(fb, Cfg::STAGE);
-                tma_load_3d(st, &tmA, fb, k0, m0, kDiag[q][0]);
-                tma_load_3d(st + Cfg::A_TILE, &tmB, fb, k0, n0, kDiag[q][1]);
+        for (int q = 0; q < NPROD && ok; ++q) {
+            const int ia = kDiag[q][0], jb = kDiag[q][1];
+            for (int c = 0; c < nch && ok; ++c) {
+                const int kspans = min(kKChunk / Cfg::KSPAN, (K - c * kKChunk + Cfg::KSPAN - 1) / Cfg::KSPAN);
+                for (int u = 0; u < kspans; ++u, ++L) {
+                    if (!(ok = mbar_wait(empty0 + 8u * s, ph ^ 1u, flags))) break;
+                    const uint32_t st = base + (uint32_t)(s * Cfg::STAGE), fb = full0 + 8u * s;
+                    const int k0 = c * kKChunk + u * Cfg::KSPAN;
+                    mbar_arrive_expect_tx(fb, Cfg::STAGE);
+#pragma unroll
+                    for (int h = 0; h < Cfg::SUB; ++h) {
+                        tma_load_3d(st + h * Cfg::A_SUB, &tmA, fb, k0 + h * Cfg::KB, m0, ia);
+                        tma_load_3d(st + Cfg::A_TILE + h * Cfg::B_SUB, &tmB, fb, k0 + h * Cfg::KB, n0, jb);
+                    }
+                    if (++s == Cfg::STAGES) { s = 0; ph ^= 1u; }
+                }
             }
         }
         if (!ok) drain_inflight(full0, Cfg::STAGES, L, flags);
-    } else if (warp == 1 && lane == 0) {
-        // ---------------- MMA issuer: one partial per (chunk, pair) into buffer t % NBUF
+      } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer: one chunk partial into buffer t % NBUF
         constexpr uint32_t idesc = make_idesc_bf16(kBM, Cfg::BN);
-        long L = 0;
+        int s = 0, b = 0;
+        uint32_t ph = 0, tph = 0;
         bool ok = true;
         for (int t = 0; t < nt && ok; ++t) {
-            const int c = t / NPROD, b = t % Cfg::NBUF;
-            const int kbn = min(kKChunk / Cfg::KB, (K - c * kKChunk + Cfg::KB - 1) / Cfg::KB);
-            if (!(ok = mbar_wait(tempty0 + 8u * b, (uint32_t)(((t / Cfg::NBUF) & 1) ^ 1), flags))) break;
+            const int c = t % nch;
+            const int kspans = min(kKChunk / Cfg::KSPAN, (K - c * kKChunk + Cfg::KSPAN - 1) / Cfg::KSPAN);
+            if (!(ok = mbar_wait(tempty0 + 8u * b, tph ^ 1u, flags))) break;
             tc_fence_after();
             const uint32_t d = tmem + (uint32_t)(b * Cfg::BN);
-            for (int kb = 0; kb < kbn; ++kb, ++L) {
-                const int s = (int)(L % Cfg::STAGES);
-                if (!(ok = mbar_wait(full0 + 8u * s, (uint32_t)((L / Cfg::STAGES) & 1), flags))) break;
+            for (int u = 0; u < kspans; ++u) {
+                if (!(ok = mbar_wait(full0 + 8u * s, ph, flags))) break;
                 tc_fence_after();
                 const uint32_t st = base + (uint32_t)(s * Cfg::STAGE);
 #pragma unroll
-                for (int kk = 0; kk < Cfg::KB / 16; ++kk) {
-                    const uint64_t ad = make_sdesc(st + kk * 32, Cfg::SBO, Cfg::SWZ);
-                    const uint64_t bd = make_sdesc(st + Cfg::A_TILE + kk * 32, Cfg::SBO, Cfg::SWZ);
-                    mma_bf16(d, ad, bd, idesc, (kb | kk) != 0);
+                for (int h = 0; h < Cfg::SUB; ++h) {
+#pragma unroll
+                    for (int kk = 0; kk < Cfg::KB / 16; ++kk) {
+                        const uint64_t ad = make_sdesc(st + h * Cfg::A_SUB + kk * 32, Cfg::SBO, Cfg::SWZ);
+                        const uint64_t bd = make_sdesc(st + Cfg::A_TILE + h * Cfg::B_SUB + kk * 32, Cfg::SBO, Cfg::SWZ);
+                        mma_bf16(d, ad, bd, idesc, (u | h | kk) != 0);
+                    }
                 }
                 mma_commit(empty0 + 8u * s);
+                if (++s == Cfg::STAGES) { s = 0; ph ^= 1u; }
             }
             if (ok) mma_commit(tfull0 + 8u * b);
+            if (++b == Cfg::NBUF) { b = 0; tph ^= 1u; }
         }
         mma_commit(done_bar);
         (void)mbar_wait(done_bar, 0, flags);
-    } else if (warp >= 2) {
-        // ---------------- drain: widen each exact FP32 partial, add in FP64
-        const int quarter = warp & 3;                       // TMEM lanes 32*quarter ..
-        const int colh = ((warp - 2) >> 2) * Cfg::COLS_PER_WARP;
-        const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)colh;
-        double acc[Cfg::COLS_PER_WARP];
-#pragma unroll
-        for (int j = 0; j < Cfg::COLS_PER_WARP; ++j) acc[j] = 0.0;
-        bool ok = true;
-        for (int t = 0; t < nt; ++t) {
-            const int b = t % Cfg::NBUF;
-            ok = mbar_wait(tfull0 + 8u * b, (uint32_t)((t / Cfg::NBUF) & 1), flags);
-            __syncwarp();
-            if (!ok) break;
-            tc_fence_after();
-#pragma unroll
-            for (int h = 0; h < Cfg::COLS_PER_WARP; h += 32) {
-                uint32_t v[32];
-                tmem_ld32(lane_base + (uint32_t)(b * Cfg::BN + h), v);
-                tmem_ld_wait();
-#pragma unroll
-                for (int j = 0; j < 32; ++j) acc[h + j] = __dadd_rn(acc[h + j], (double)__uint_as_float(v[j]));
-            }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(tempty0 + 8u * b);
-        }
+      }
+    } else {
+        regs_inc<Cfg::REG_DRAIN>();
+        // ---------------- drain: exact per-product sum of the partials, one FP64 add per product
+        const int quarter = warp & 3;                                    // TMEM lanes 32*quarter ..
+        const int colh = ((warp - Cfg::FIRST_DRAIN) >> 2) * Cfg::COLS;   // this warp's 32 columns
+        const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
+        const uint32_t acc_base = lane_base + Cfg::ACC_COL + 2u * (uint32_t)colh;
         const int row = m0 + quarter * 32 + lane;
-        if (ok && row < M) {
-            double *crow = C + (int64_t)row * ldc + n0 + colh;
-            const int lim = N - (n0 + colh);
-            if (lim >= Cfg::COLS_PER_WARP && ((ldc & 1) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15u) == 0)) {
+        const bool row_ok = row < M;
+        const bool vec = ((ldc & 1) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15u) == 0);
+        double *crow = C + (int64_t)row * ldc + n0 + colh;
+        const int lim = N - (n0 + colh);                  // valid columns of this warp's slice
+        float hi[Cfg::COLS];
+        bool ok = true;
+        for (int q = 0; q < NPROD && ok; ++q) {
 #pragma unroll
-                for (int j = 0; j < Cfg::COLS_PER_WARP; j += 2)
-                    *reinterpret_cast<double2 *>(crow + j) = make_double2(acc[j], acc[j + 1]);
-            } else {
+            for (int j = 0; j < Cfg::COLS; ++j) hi[j] = 0.0f;
+            uint32_t dirty = 0;                           // 16-column groups whose low part lives in C
+            const float bound = exact_bound(vA, vB, kDiag[q][0], kDiag[q][1]);
+            for (int c = 0; c < nch; ++c) {
+                const int t = q * nch + c, b = t % Cfg::NBUF;
+                ok = mbar_wait(tfull0 + 8u * b, (uint32_t)((t / Cfg::NBUF) & 1), flags);
+                __syncwarp();
+                if (!ok) break;
+                tc_fence_after();
+                uint32_t v[Cfg::COLS];
 #pragma unroll
-                for (int j = 0; j < Cfg::COLS_PER_WARP; ++j)
-                    if (j < lim) crow[j] = acc[j];
+                for (int h = 0; h < Cfg::COLS; h += 16)
+                    tmem_ld16(lane_base + (uint32_t)(b * Cfg::BN + colh + h), *reinterpret_cast<uint32_t(*)[16]>(v + h));
+                tmem_ld_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(tempty0 + 8u * b);    // buffer free: values are in registers
+#pragma unroll
+                for (int h = 0; h < Cfg::COLS; h += 16) {
+                    float sum[16];
+                    bool big = false;
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        sum[j] = __fadd_rn(hi[h + j], __uint_as_float(v[h + j]));
+                        big |= !(fabsf(sum[j]) < bound);
+                    }
+                    if (__any_sync(0xFFFFFFFFu, big)) {       // rare: exact TwoSum errors into the low part
+                        const bool was = (dirty >> (h / 16)) & 1u;
+                        dirty |= 1u << (h / 16);
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            const float p = __uint_as_float(v[h + j]);
+                            const float bb = __fsub_rn(sum[j], hi[h + j]);
+                            const float e = __fadd_rn(__fsub_rn(hi[h + j], __fsub_rn(sum[j], bb)), __fsub_rn(p, bb));
+                            if (row_ok && h + j < lim) crow[h + j] = __dadd_rn(was ? crow[h + j] : 0.0, (double)e);
+                        }
+                    }
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) hi[h + j] = sum[j];
+                }
             }
+            if (!ok) break;
+            // fold: C <- fl64(C + (hi + lo)); hi + lo is exact in FP64
+            const bool last = (q == NPROD - 1);
+#pragma unroll
+            for (int g = 0; g < Cfg::COLS; g += 8) {
+                uint32_t w[16];
+                if (q > 0) {
+                    tmem_ld16(acc_base + 2u * g, w);
+                    tmem_ld_wait();
+                }
+                const bool dg = (dirty >> (g / 16)) & 1u;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    double sq = widen_exact(hi[g + j]);
+                    if (dg && row_ok && g + j < lim) sq = __dadd_rn(sq, crow[g + j]);   // exact
+                    const double cprev = (q > 0) ? __hiloint2double((int)w[2 * j + 1], (int)w[2 * j]) : 0.0;
+                    const double out = __dadd_rn(cprev, sq);
+                    w[2 * j] = (uint32_t)__double2loint(out);
+                    w[2 * j + 1] = (uint32_t)__double2hiint(out);
+                }
+                if (!last) {
+                    tmem_st16(acc_base + 2u * g, w);
+                } else if (row_ok) {
+                    if (vec && lim >= g + 8) {
+#pragma unroll
+                        for (int j = 0; j < 8; j += 2)
+                            *reinterpret_cast<int4 *>(crow + g + j) =
+                                make_int4((int)w[2 * j], (int)w[2 * j + 1], (int)w[2 * j + 2], (int)w[2 * j + 3]);
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 8; ++j)
+                            if (g + j < lim) crow[g + j] = __hiloint2double((int)w[2 * j + 1], (int)w[2 * j]);
+                    }
+                }
+            }
+            if (!last) tmem_st_wait();
         }
     }
     tc_fence_before();
@@ -160,7 +323,7 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
 
 template <int NPROD>
 cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
-                    double *C, int64_t ldc, uint32_t *flags, cudaStream_t st)
+                    const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, uint32_t *flags, cudaStream_t st)
 {
     using Cfg = F64Cfg;
     CUtensorMap ta, tb;
@@ -170,20 +333,21 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
     const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + Cfg::BN - 1) / Cfg::BN);
-    kern<<<(unsigned)tiles, Cfg::THREADS, Cfg::SMEM, st>>>(ta, tb, (int)M, (int)N, (int)K, C, ldc, flags);
+    kern<<<(unsigned)tiles, Cfg::THREADS, Cfg::SMEM, st>>>(ta, tb, (int)M, (int)N, (int)K, vA, vB, C, ldc, flags);
     return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
-                               int64_t ldcomp, int nprod, double *C, int64_t ldc, uint32_t *flags, cudaStream_t st)
+                               int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
+                               int64_t ldc, uint32_t *flags, cudaStream_t st)
 {
     switch (nprod) {
-    case 6: return run_f64<6>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st);
-    case 10: return run_f64<10>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st);
-    case 15: return run_f64<15>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st);
-    case 21: return run_f64<21>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st);
+    case 6: return run_f64<6>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st);
+    case 10: return run_f64<10>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st);
+    case 15: return run_f64<15>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st);
+    case 21: return run_f64<21>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st);
     default: return cudaErrorInvalidValue;
     }
 }

@@ -117,6 +117,58 @@ __device__ __forceinline__ uint16_t f64_level(double &R, int v, bool &bad)
     return s;
 }
 
+// The same level computed with integer operations only (GB300 runs FP64 at a
+// small fraction of its integer rate).  It restates the projection exactly:
+// for |R| <= 2^v, fl64(R + 2^(v+45)) lies in the binade above 2^(v+45) when
+// R >= 0 (spacing 2^(v-7)) and in the binade below it when R < 0 (spacing
+// 2^(v-8)), and the subtraction of 2^(v+45) is exact; so Z is R rounded to
+// nearest, ties to even, on the grid G = 2^(v-7) or 2^(v-8): Z = sign * n * G
+// with n <= 256.  R - Z is exact and is renormalised from the integer
+// difference.  Values it cannot take this way (non-finite input, R not below
+// 2^v, or Z outside the normal BF16 range) go through f64_level.
+__device__ __forceinline__ uint16_t f64_level_int(double &R, int v, bool &bad)
+{
+    if (v == kZeroLevel) return 0;
+    const uint64_t b = (uint64_t)__double_as_longlong(R);
+    const uint64_t a = b & 0x7FFFFFFFFFFFFFFFull;
+    if (a == 0) return 0;                                      // Z = +0, R unchanged
+    const uint32_t sgn = (uint32_t)(b >> 63);
+    int E = (int)(a >> 52);
+    if (E == 0x7FF) return f64_level(R, v, bad);
+    uint64_t M = a & 0x000FFFFFFFFFFFFFull;
+    if (E == 0) E = 1; else M |= 1ull << 52;                  // |R| = M * 2^(E - 1075)
+    const int G = v - (sgn ? 8 : 7);                           // grid exponent
+    const int sh = G - (E - 1075);
+    if (sh <= 0 || sh > 60) {
+        if (sh > 60) return 0;                                 // |R| < G / 2: Z = +0
+        return f64_level(R, v, bad);
+    }
+    uint64_t n = M >> sh;
+    const uint64_t rem = M & ((1ull << sh) - 1ull), half = 1ull << (sh - 1);
+    if (rem > half || (rem == half && (n & 1ull))) ++n;
+    if (n == 0) return 0;
+    if (n > 256) return f64_level(R, v, bad);                 // |R| > 2^v: not this level's grid
+    const int p = 31 - __clz((unsigned)n);                     // leading bit of n, 0..8
+    const int ez = G + p;                                      // exponent of Z's leading bit
+    if (ez < -126 || ez > 127) return f64_level(R, v, bad);
+    // residual R - Z = sign * (M - n * 2^sh) * 2^(E - 1075), exact
+    const int64_t d = (int64_t)M - (int64_t)(n << sh);
+    if (d == 0) {
+        R = 0.0;
+    } else {
+        const uint64_t ad = (uint64_t)(d < 0 ? -d : d);
+        const uint64_t rs = (uint64_t)(sgn ^ (d < 0 ? 1u : 0u)) << 63;
+        const int lz = __clzll((long long)ad) - 11;            // bring the leading bit to bit 52
+        int er = E - lz;
+        uint64_t rb;
+        if (er >= 1) rb = rs | ((uint64_t)er << 52) | ((ad << lz) & 0x000FFFFFFFFFFFFFull);
+        else rb = rs | ((ad << lz) >> (1 - er));              // subnormal result, still exact
+        R = __longlong_as_double((long long)rb);
+    }
+    const uint32_t mant = (p <= 7 ? ((uint32_t)n << (7 - p)) : ((uint32_t)n >> 1)) & 0x7Fu;
+    return (uint16_t)((sgn << 15) | ((uint32_t)(ez + 127) << 7) | mant);
+}
+
 // Final v^(0..5) of operand `slot` once verification and fix passes ran
 // (levels up to fix_from come from the verifier, later ones from the fix
 // maxima).  Levels past an all-zero residual are kZeroLevel.
@@ -135,24 +187,27 @@ __device__ __forceinline__ void final_levels(const WsHeader *ws, int slot, int u
     }
 }
 
-__device__ __forceinline__ double warp_max(double x)
+__device__ __forceinline__ unsigned long long warp_max(unsigned long long x)
 {
-    for (int o = 16; o; o >>= 1) x = fmax(x, __shfl_xor_sync(0xFFFFFFFFu, x, o));
+    for (int o = 16; o; o >>= 1) {
+        const unsigned long long y = __shfl_xor_sync(0xFFFFFFFFu, x, o);
+        x = y > x ? y : x;
+    }
     return x;
 }
 
-// Block-wide max of one value per thread, then one atomicMax on the bit
-// pattern (non-negative doubles order like their bit patterns).
-__device__ __forceinline__ void block_max_to(double x, unsigned long long *dst, double *red)
+// Block-wide max of one value per thread, then one atomicMax: the values are
+// bit patterns of non-negative doubles, which order like the doubles.
+__device__ __forceinline__ void block_max_to(unsigned long long x, unsigned long long *dst, unsigned long long *red)
 {
     x = warp_max(x);
     const int w = threadIdx.x >> 5;
     if (lane_id() == 0) red[w] = x;
     __syncthreads();
     if (threadIdx.x == 0) {
-        double m = 0.0;
-        for (int i = 0; i < kThreads / 32; ++i) m = fmax(m, red[i]);
-        if (m > 0.0) atomicMax(dst, (unsigned long long)__double_as_longlong(m));
+        unsigned long long m = 0;
+        for (int i = 0; i < kThreads / 32; ++i) m = red[i] > m ? red[i] : m;
+        if (m) atomicMax(dst, m);
     }
     __syncthreads();
 }
@@ -171,7 +226,7 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
     auto sm = [&](int r, int row, int col) -> uint16_t & {
         return smdyn[((size_t)r * kTile + row) * kSRow + col];
     };
-    __shared__ double red[kThreads / 32];
+    __shared__ unsigned long long red[kThreads / 32];
 
     int v[6] = {0, 0, 0, 0, 0, 0};
     if constexpr (MODE == 1) {
@@ -183,7 +238,7 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
         final_levels(ws, slot, 6, v);
     }
 
-    double mx[5] = {0.0, 0.0, 0.0, 0.0, 0.0};
+    unsigned long long mx[5] = {0, 0, 0, 0, 0};         // max |A^(r)| as bit patterns
     uint32_t badmask = 0, flagbits = 0;
     const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;   // 16 x 16 threads
@@ -231,10 +286,14 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
 #pragma unroll
                     for (int r = 0; r < 6; ++r) {
                         if constexpr (MODE == 1) {
-                            if (r > 0) mx[r - 1] = fmax(mx[r - 1], fabs(R));
+                            if (r > 0) {
+                                const unsigned long long ab =
+                                    (unsigned long long)__double_as_longlong(R) & 0x7FFFFFFFFFFFFFFFull;
+                                mx[r - 1] = ab > mx[r - 1] ? ab : mx[r - 1];
+                            }
                         }
                         bool bad = false;
-                        s[r] = f64_level(R, v[r], bad);
+                        s[r] = f64_level_int(R, v[r], bad);
                         if (bad) badmask |= 1u << r;
                     }
                 }
@@ -288,15 +347,17 @@ __global__ void __launch_bounds__(kThreads)
 f64_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, WsHeader *ws,
                int slot)
 {
-    __shared__ double red[kThreads / 32];
+    __shared__ unsigned long long red[kThreads / 32];
     int v[6] = {0, 0, 0, 0, 0, 0};
     if constexpr (LEVEL > 0) {
         if (ws->fix_from[slot] >= LEVEL) return;
         final_levels(ws, slot, LEVEL, v);
         if (v[LEVEL - 1] == kZeroLevel) return;   // residual already zero
     }
-    const double lo = 0x1p-126, hi = 0x1.fcp127;  // (2 - 2^-7) * 2^127
-    double m = 0.0;
+    // bit patterns of |x|: 2^-126 and (2 - 2^-7) * 2^127, and the exponent mask
+    constexpr unsigned long long kLo = 0x3810000000000000ull, kHi = 0x47EFE00000000000ull;
+    constexpr unsigned long long kInf = 0x7FF0000000000000ull;
+    unsigned long long m = 0;
     uint32_t flagbits = 0;
     const int64_t segs = (cols + 4 * kThreads - 1) / (4 * kThreads);
     for (int64_t it = blockIdx.x; it < rows * segs; it += gridDim.x) {
@@ -314,16 +375,18 @@ f64_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             double R = x[e];
-            if constexpr (LEVEL == 0) {
-                const double a = fabs(R);
-                if (!isfinite(R)) flagbits |= EMU_FLAG_NONFINITE;
-                else if (R != 0.0 && (a < lo || a > hi)) flagbits |= EMU_FLAG_RANGE;
-                if (!isnan(R)) m = fmax(m, a);
-            } else {
+            if constexpr (LEVEL > 0) {
                 bool bad = false;
 #pragma unroll
-                for (int r = 0; r < LEVEL; ++r) (void)f64_level(R, v[r], bad);
-                m = fmax(m, fabs(R));
+                for (int r = 0; r < LEVEL; ++r) (void)f64_level_int(R, v[r], bad);
+            }
+            const unsigned long long ab = (unsigned long long)__double_as_longlong(R) & 0x7FFFFFFFFFFFFFFFull;
+            if constexpr (LEVEL == 0) {
+                if (ab >= kInf) flagbits |= EMU_FLAG_NONFINITE;
+                else if (ab != 0 && (ab < kLo || ab > kHi)) flagbits |= EMU_FLAG_RANGE;
+                if (ab <= kInf) m = ab > m ? ab : m;                  // NaN never wins
+            } else {
+                m = ab > m ? ab : m;
             }
         }
     }

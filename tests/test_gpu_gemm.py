@@ -134,12 +134,30 @@ def test_prodsum_f64_from_gpu_planes(dev):
     M, N, K = 150, 170, 400
     A, B = synth.gemm_inputs("f64", M, N, K, 8)
     ldk = emu.gemm_ldk(K)
-    Ap, _, ws = emu.split_f64(to_dev(A, dev), ldcomp=ldk)
-    Bp, _, _ = emu.split_f64(to_dev(B, dev), transpose=True, ldcomp=ldk, ws=ws)
+    Ap, vA, ws = emu.split_f64(to_dev(A, dev), ldcomp=ldk)
+    Bp, vB, _ = emu.split_f64(to_dev(B, dev), transpose=True, ldcomp=ldk, ws=ws)
     for nprod in (6, 21):
-        C, _ = emu.prodsum_f64(Ap, Bp, M, N, K, nprod)
         Co = oracle.prodsum_f64(oracle.split_f64(A)[0], oracle.split_f64(B)[0], nprod)
+        C, _ = emu.prodsum_f64(Ap, Bp, M, N, K, nprod, vA=vA, vB=vB)       # bounded plain adds
         assert np.array_equal(C.cpu().numpy(), Co)
+        C, _ = emu.prodsum_f64(Ap, Bp, M, N, K, nprod)                     # every add error-free
+        assert np.array_equal(C.cpu().numpy(), Co)
+
+
+def test_prodsum_f64_error_free_path_at_the_2pow24_edge(dev):
+    """Without level exponents every partial goes through TwoSum; with them the
+    running sums pass 2^24 units after two chunks and take the same path."""
+    K = 768
+    A = np.full((130, K), -255 / 256)
+    B = np.full((K, 140), -255 / 256)
+    B[0, :] = -254 / 256
+    ldk = emu.gemm_ldk(K)
+    Ap, vA, ws = emu.split_f64(to_dev(A, dev), ldcomp=ldk)
+    Bp, vB, _ = emu.split_f64(to_dev(B, dev), transpose=True, ldcomp=ldk, ws=ws)
+    want = (65025 * 767 + 255 * 254) * 2.0**-16
+    for va, vb in ((vA, vB), (None, None)):
+        C, _ = emu.prodsum_f64(Ap, Bp, 130, 140, K, 6, vA=va, vB=vb)
+        assert np.all(C.cpu().numpy() == want)
 
 
 # ------------------------------------------------------------ edges, errors
@@ -169,10 +187,13 @@ def test_error_codes(dev):
                             ws.data_ptr(), ws.numel() - 1, s) == 3
     planes = torch.zeros((6, 64, 72), dtype=torch.int16, device=dev)
     # plane rows not a multiple of 16 bytes -> MISALIGNED; base off by 2 bytes -> MISALIGNED
-    assert emu.emu_prodsum_f64(64, 64, 64, planes.data_ptr(), planes.data_ptr(), 66, 6, C.data_ptr(), 64,
-                               ws.data_ptr(), ws.numel(), s) == 2
-    assert emu.emu_prodsum_f64(64, 64, 64, planes.data_ptr() + 2, planes.data_ptr(), 72, 6, C.data_ptr(), 64,
-                               ws.data_ptr(), ws.numel(), s) == 2
+    assert emu.emu_prodsum_f64(64, 64, 64, planes.data_ptr(), planes.data_ptr(), 66, None, None, 6, C.data_ptr(),
+                               64, ws.data_ptr(), ws.numel(), s) == 2
+    assert emu.emu_prodsum_f64(64, 64, 64, planes.data_ptr() + 2, planes.data_ptr(), 72, None, None, 6,
+                               C.data_ptr(), 64, ws.data_ptr(), ws.numel(), s) == 2
+    v = torch.zeros(6, dtype=torch.int32, device=dev)
+    assert emu.emu_prodsum_f64(64, 64, 64, planes.data_ptr(), planes.data_ptr(), 72, v.data_ptr(), None, 6,
+                               C.data_ptr(), 64, ws.data_ptr(), ws.numel(), s) == 1    # vA without vB
 
 
 def test_watchdog_timeout_reports_and_context_survives(dev):

@@ -279,16 +279,18 @@ def _exact_slice_sum(Ap, Bp, pairs):
     return out, absout
 
 
+@pytest.mark.parametrize("order", ["chunk", "product"])
 @pytest.mark.parametrize("K", [8, 300])
-def test_brute_force_fp64_against_exact_retained_sum(K):
+def test_brute_force_fp64_against_exact_retained_sum(K, order):
     """8x8xK brute force: the oracle's FP64 product-sum equals the exact sum of
-    the retained products up to the FP64 rounding of its additions."""
+    the retained products up to the FP64 rounding of its additions (in either
+    summation order of the exact chunk partials)."""
     A, B = synth.gemm_inputs("f64", 8, 8, K, 17)
     Ap, _, _ = oracle.split_f64(A)
     Bp, _, _ = oracle.split_f64(B)
     nch = -(-K // oracle.KCHUNK)
     for nprod in (6, 21):
-        C = oracle.prodsum_f64(Ap, Bp, nprod)
+        C = oracle.prodsum_f64(Ap, Bp, nprod, order=order)
         S, absS = _exact_slice_sum(Ap, Bp, oracle.products(64, nprod))
         nadd = nch * nprod
         for m in range(8):
@@ -324,20 +326,22 @@ def test_fp32_bf16_exact_integers_give_exact_product():
         assert np.array_equal(C.astype(np.int64), A.astype(np.int64) @ B.astype(np.int64))
 
 
+@pytest.mark.parametrize("order", ["chunk", "product"])
 @pytest.mark.parametrize("nprod", [6, 10, 15, 21])
-def test_fp64_two_slice_integers_give_exact_product(nprod):
+def test_fp64_two_slice_integers_give_exact_product(nprod, order):
     """Integers |x| <= 2^15 need two slices; with d >= 3 all of A0B0, A0B1,
     A1B0, A1B1 are retained, so the result is the exact product."""
     rng = np.random.default_rng(5)
     A = rng.integers(-2**15, 2**15 + 1, size=(16, 520)).astype(np.float64)
     B = rng.integers(-2**15, 2**15 + 1, size=(520, 12)).astype(np.float64)
-    C, flags = oracle.gemm_f64(A, B, nprod)
+    C, flags = oracle.gemm_f64(A, B, nprod, order=order)
     assert flags == 0
     assert np.array_equal(C, (A.astype(np.int64) @ B.astype(np.int64)).astype(np.float64))
 
 
+@pytest.mark.parametrize("order", ["chunk", "product"])
 @pytest.mark.parametrize("nprod", [6, 10, 15])
-def test_fp64_omitted_products_term(nprod):
+def test_fp64_omitted_products_term(nprod, order):
     """Integers up to 2^23 need three slices, all integer-valued.  Every sum is
     then exact, so C_hat = A.B - E_omit exactly, with E_omit of Eq. (omit)."""
     rng = np.random.default_rng(6)
@@ -350,7 +354,7 @@ def test_fp64_omitted_products_term(nprod):
     assert all(np.array_equal(x.astype(np.float64), oracle.bf16_to_f32(Ap[s])) for s, x in enumerate(a))
     retained = set(oracle.products(64, nprod))
     omit = sum(a[i] @ b[j] for i in range(6) for j in range(6) if (i, j) not in retained)
-    C = oracle.prodsum_f64(Ap, Bp, nprod)
+    C = oracle.prodsum_f64(Ap, Bp, nprod, order=order)
     exact = A.astype(np.int64) @ B.astype(np.int64)
     assert np.array_equal(C.astype(np.int64), exact - omit)
     assert np.array_equal(C, (exact - omit).astype(np.float64))
@@ -442,3 +446,24 @@ def test_fp64_partials_exact_at_the_2pow24_edge():
     assert bad == 0
     assert C[0, 0] == (65025 * 511 + 255 * 254) * 2.0**-16
     assert (65025 * 255 + 255 * 254) > 2**23          # chunk 0 needs all 24 bits
+
+
+def test_fp64_orders_agree_within_fp64_rounding():
+    """The two summation orders add the same exact chunk partials; they may
+    differ only by the FP64 rounding of the additions, and the product-outer
+    order rounds less often (one addition per product instead of one per
+    chunk and product)."""
+    A, B = synth.gemm_inputs("f64_scaled", 40, 36, 1500, 7, phi=2.0)
+    Ap, _, _ = oracle.split_f64(A)
+    Bp, _, _ = oracle.split_f64(B)
+    hi, lo = oracle.ref_dd(A, B)
+    nch = -(-1500 // oracle.KCHUNK)
+    for nprod in (6, 21):
+        Cc = oracle.prodsum_f64(Ap, Bp, nprod, order="chunk")
+        Cp = oracle.prodsum_f64(Ap, Bp, nprod, order="product")
+        a = [oracle.bf16_to_f32(Ap[s]).astype(np.float64) for s in range(6)]
+        b = [oracle.bf16_to_f32(Bp[s]).astype(np.float64) for s in range(6)]
+        absP = sum(np.abs(a[i]) @ np.abs(b[j]) for i, j in oracle.products(64, nprod))
+        assert np.all(np.abs(Cc - Cp) <= 2 * nprod * nch * 2.0**-53 * absP)
+        ec, ep = oracle.errors(Cc, hi, lo), oracle.errors(Cp, hi, lo)
+        assert ep["e_F"] <= 1.01 * ec["e_F"] + 1e-300
