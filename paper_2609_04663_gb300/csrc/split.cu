@@ -169,6 +169,79 @@ __device__ __forceinline__ uint16_t f64_level_int(double &R, int v, bool &bad)
     return (uint16_t)((sgn << 15) | ((uint32_t)(ez + 127) << 7) | mant);
 }
 
+// The six speculative levels v^(r) = v0 - 8r of one entry in fixed point.
+// x is converted once to a signed integer X in units of 2^F, F = v0 - 50 (two
+// bits below the finest grid 2^(v0 - 48)), truncating with a sticky ("jam")
+// bit in the last place when x has bits below 2^F.  Every grid and every
+// half-grid is an even multiple of 2^F, and a jammed value is odd and within
+// one unit of the true one, so all round-to-nearest-even decisions and all
+// comparisons with powers of two >= 2^(F+1) are those of the exact value;
+// exact values stay exact.  Level r rounds X to nearest, ties to even, on the
+// grid 2^(43 - 8r) (X >= 0) or 2^(42 - 8r) (X < 0) units -- the sign-dependent
+// grid of the add-subtract projection -- and subtracts it.  |X| before level
+// r goes to mx[r - 1] (in units of 2^F).  Levels 0-2 need 64-bit words; from
+// level 3 on |X| < 2^27 and 32-bit words suffice.
+__device__ __forceinline__ void spec_levels(double x, int v0, uint16_t (&s)[6], uint32_t &badmask,
+                                            unsigned long long (&mx)[5])
+{
+    const uint64_t b = (uint64_t)__double_as_longlong(x);
+    const uint32_t xs = (uint32_t)(b >> 63);
+    const int E = (int)((b >> 52) & 0x7FFu);
+    uint64_t M = b & 0x000FFFFFFFFFFFFFull;
+    int Ee = E;
+    if (E == 0) Ee = 1; else M |= 1ull << 52;
+    const int F = v0 - 50;
+    const int sh0 = (Ee - 1075) - F;                   // left shift into units of 2^F
+    uint64_t mag;
+    if (E == 0x7FF) badmask |= 1u;                     // a non-finite slice 0 (NONFINITE comes from the max pass)
+    if (E == 0x7FF || M == 0) mag = 0;
+    else if (sh0 >= 0) mag = sh0 < 12 ? (M << sh0) : (1ull << 62);   // (|x| > 2^v0 cannot occur)
+    else if (sh0 > -64) mag = (M >> (-sh0)) | ((M << (64 + sh0)) != 0 ? 1ull : 0ull);
+    else mag = 1;
+    int64_t X = xs ? -(int64_t)mag : (int64_t)mag;
+    // levels 0..2 in 64-bit
+#pragma unroll
+    for (int r = 0; r < 3; ++r) {
+        const uint32_t sg = X < 0 ? 1u : 0u;
+        const uint64_t a = (uint64_t)(sg ? -X : X);
+        if (r > 0) mx[r - 1] = a > mx[r - 1] ? a : mx[r - 1];
+        const int g = 43 - 8 * r - (int)sg;            // grid in units of 2^F
+        const uint64_t n = (a + (1ull << (g - 1)) - 1ull + ((a >> g) & 1ull)) >> g;
+        const int64_t zm = (int64_t)(n << g);
+        X = sg ? (zm - (int64_t)a) : ((int64_t)a - zm);
+        uint16_t out = 0;
+        if (n) {
+            const int p = 31 - __clz((unsigned)n);
+            const int ez = F + g + p;                  // exponent of Z's leading bit
+            if (ez < -126 || ez > 127) badmask |= 1u << r;
+            const uint32_t mant = (p <= 7 ? ((uint32_t)n << (7 - p)) : ((uint32_t)n >> 1)) & 0x7Fu;
+            out = (uint16_t)((sg << 15) | ((uint32_t)(ez + 127) << 7) | mant);
+        }
+        s[r] = out;
+    }
+    // levels 3..5 in 32-bit: |X| <= 2^26 + 1 here
+    int32_t Y = (int32_t)X;
+#pragma unroll
+    for (int r = 3; r < 6; ++r) {
+        const uint32_t sg = Y < 0 ? 1u : 0u;
+        const uint32_t a = (uint32_t)(sg ? -Y : Y);
+        mx[r - 1] = a > mx[r - 1] ? a : mx[r - 1];
+        const int g = 43 - 8 * r - (int)sg;
+        const uint32_t n = (a + (1u << (g - 1)) - 1u + ((a >> g) & 1u)) >> g;
+        const int32_t zm = (int32_t)(n << g);
+        Y = sg ? (zm - (int32_t)a) : ((int32_t)a - zm);
+        uint16_t out = 0;
+        if (n) {
+            const int p = 31 - __clz(n);
+            const int ez = F + g + p;
+            if (ez < -126 || ez > 127) badmask |= 1u << r;
+            const uint32_t mant = (p <= 7 ? (n << (7 - p)) : (n >> 1)) & 0x7Fu;
+            out = (uint16_t)((sg << 15) | ((uint32_t)(ez + 127) << 7) | mant);
+        }
+        s[r] = out;
+    }
+}
+
 // Final v^(0..5) of operand `slot` once verification and fix passes ran
 // (levels up to fix_from come from the verifier, later ones from the fix
 // maxima).  Levels past an all-zero residual are kZeroLevel.
@@ -281,17 +354,17 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
                         if ((b & 0x7F80u) == 0x7F80u) flagbits |= EMU_FLAG_SLICE;
                         a = __fsub_rn(a, bf16_as_float(b));
                     }
+                } else if constexpr (MODE == 1) {
+                    if (v[0] == kZeroLevel) {
+#pragma unroll
+                        for (int r = 0; r < 6; ++r) s[r] = 0;
+                    } else {
+                        spec_levels(x[e], v[0], s, badmask, mx);
+                    }
                 } else {
                     double R = x[e];
 #pragma unroll
                     for (int r = 0; r < 6; ++r) {
-                        if constexpr (MODE == 1) {
-                            if (r > 0) {
-                                const unsigned long long ab =
-                                    (unsigned long long)__double_as_longlong(R) & 0x7FFFFFFFFFFFFFFFull;
-                                mx[r - 1] = ab > mx[r - 1] ? ab : mx[r - 1];
-                            }
-                        }
                         bool bad = false;
                         s[r] = f64_level_int(R, v[r], bad);
                         if (bad) badmask |= 1u << r;
@@ -333,8 +406,13 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
         if (badmask && lane_id() == 0) atomicOr(&ws->slice_bad[slot], MODE == 1 ? badmask : badmask << 8);
     }
     if constexpr (MODE == 1) {
+        // mx holds |A^(r)| in units of 2^(v0 - 50), below 2^53: exact as doubles
+        const int F = (v[0] == kZeroLevel) ? 0 : v[0] - 50;
 #pragma unroll
-        for (int r = 0; r < 5; ++r) block_max_to(mx[r], &ws->maxbits[slot][r + 1], red);
+        for (int r = 0; r < 5; ++r) {
+            const double m = (double)mx[r] * pow2_d(F);
+            block_max_to((unsigned long long)__double_as_longlong(m), &ws->maxbits[slot][r + 1], red);
+        }
     }
 }
 
