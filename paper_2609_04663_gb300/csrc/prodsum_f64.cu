@@ -5,23 +5,31 @@
 // Every chunk partial fl32(A_i B_j) is formed on the tensor cores in its own
 // TMEM buffer (two rotating 128-column buffers).  The partials are exact:
 // slice entries are integers times 2^(v-8) of magnitude <= 256, so a chunk
-// partial is an integer of at most 2^24 units.  Sixteen drain warps add the
-// partials of one product exactly in FP32: the running sum hi stays in
-// registers, and while it stays below 2^24 units (known from the split's level
-// exponents) a plain FP32 addition is exact.  Past that bound the error of
-// each addition is recovered with Knuth's TwoSum and summed into a low part
-// kept in the output buffer C, which is free scratch until the last product
-// (uniform data never gets there).
-// FP32 adds only, so GB300's slow FP64 pipe is not touched per chunk.  When
-// the product is complete, hi + lo is widened (exact; the common hi-only case
-// by integer bit operations) and added once into the FP64 accumulator in the
-// upper 256 TMEM columns: C <- fl64(C + fl32(A_i B_j)), Algorithm 2's step.
-// The result is bit-identical to the oracle in its product-outer order.
+// partial is an integer of at most 2^24 units u = 2^(vA_i + vB_j - 16).
+//
+// Sixteen drain warps sum the partials of one product exactly in FP32
+// registers: while the running sum hi stays below 2^24 u (known from the
+// split's level exponents) a plain FP32 addition is exact.  Past that bound
+// the error of each addition is recovered with Knuth's TwoSum and summed into
+// a low part lo, an FP32 word kept in the output buffer C (free scratch until
+// the last product; even products use one half of each C word, odd products
+// the other); (hi, lo) is renormalised by another TwoSum whenever lo reaches
+// 2^23 u, so the additions into lo are exact for any K.
+//
+// A finished product's sums go through a 64 KB shared-memory hand-off to four
+// fold warps, which add hi + lo (exact in FP64) once into the FP64
+// accumulator in the upper 256 TMEM columns: C <- fl64(C + fl32(A_i B_j)),
+// Algorithm 2's step.  GB300's FP64 pipe does two adds per clock per SM, so
+// a product's 128 x 128 FP64 adds take as long as several chunk partials; with
+// the fold in its own warps the drain warps go straight on to the next
+// product and the tensor cores keep running.  The result is bit-identical to
+// the oracle in its product-outer order.
 //
 // Warp roles: warp 0 lane 0 issues TMA loads, warp 1 owns TMEM and lane 0
-// issues the MMAs, warps 4-19 drain (setmaxnreg moves registers from the
-// control warpgroup to the four drain warpgroups).  Every wait is bounded and reports
-// EMU_FLAG_TIMEOUT instead of hanging.
+// issues the MMAs, warps 4-19 drain (four per TMEM lane quarter, 32 columns
+// each), warps 20-23 fold (one per lane quarter, 128 columns each).
+// setmaxnreg moves registers between the warpgroups.  Every wait is bounded
+// and reports EMU_FLAG_TIMEOUT instead of hanging.
 #include "gemm_common.cuh"
 
 namespace emu {
@@ -36,29 +44,38 @@ __constant__ int8_t kDiag[21][2] = {{0, 0}, {0, 1}, {1, 0}, {0, 2}, {1, 1}, {2, 
 
 struct F64Cfg {
     // A stage holds SUB K-blocks of 64 (one 128-byte swizzle row each) of the
-    // A slice and of the B slice: 64 KB, eight MMAs, so the single-thread
-    // producer and MMA loops pay their per-stage overhead once per 128 of K.
-    static constexpr int BN = 128, KB = 64, SUB = 2, STAGES = 3, NBUF = 2;
+    // A slice and of the B slice.
+    static constexpr int BN = 128, KB = 64, SUB = 2, STAGES = 2, NBUF = 2;
     static constexpr int KSPAN = KB * SUB;                          // K per stage
     static constexpr int A_SUB = kBM * KB * 2, B_SUB = BN * KB * 2; // one 64-wide K-block tile
     static constexpr int A_TILE = A_SUB * SUB, B_TILE = B_SUB * SUB;
     static constexpr int STAGE = A_TILE + B_TILE;
     static constexpr uint32_t SWZ = 2u, SBO = 1024u;              // 128-byte swizzle
-    static constexpr int BAR_OFF = STAGES * STAGE;
+    // hand-off of a product's sums: [128 rows][128 columns] FP32, 16-byte
+    // chunks of a row XOR-swizzled by (row & 7); then one low-part mask byte
+    // per (row, drain column quarter)
+    static constexpr int HAND_OFF = STAGES * STAGE;
+    static constexpr int MASK_OFF = HAND_OFF + kBM * BN * 4;
+    static constexpr int BAR_OFF = MASK_OFF + kBM * 4;
+    // barriers: full/empty per stage, tfull/tempty per buffer, hand-off
+    // full/empty, done; then the TMEM address slot
+    static constexpr int NBARS = 2 * STAGES + 2 * NBUF + 2 + 1;
     static constexpr int SMEM = BAR_OFF + 256 + 1024;
     // warpgroup 0: TMA producer (warp 0), MMA issuer + TMEM owner (warp 1),
-    // two idle warps; warpgroups 1-4: sixteen drain warps, four per TMEM lane
-    // quarter, 32 columns each.
-    static constexpr int DRAIN_WARPS = 16, THREADS = 640, FIRST_DRAIN = 4;
+    // two idle warps; warpgroups 1-4: sixteen drain warps; warpgroup 5: fold
+    static constexpr int FIRST_DRAIN = 4, DRAIN_WARPS = 16, FIRST_FOLD = 20, THREADS = 24 * 32;
     static constexpr int COLS = BN / (DRAIN_WARPS / 4);            // 32 columns per drain thread
-    // Register split: the launch reserves 640 x 96 (five warps per SMSP);
-    // warpgroup 0 drops to 32, the drain warpgroups rise to 112:
-    // 128 x 32 + 512 x 112 = 61440 = 640 x 96.
-    static constexpr int REG_CTRL = 32, REG_DRAIN = 112, REG_LAUNCH = 96;
+    // Register split: the launch reserves 768 x 80 (six warps per SMSP);
+    // 128 x 32 (control) + 512 x 96 (drain) + 128 x 64 (fold) = 61440 = 768 x 80.
+    static constexpr int REG_CTRL = 32, REG_DRAIN = 96, REG_FOLD = 64, REG_LAUNCH = 80;
     static constexpr uint32_t ACC_COL = NBUF * BN;                 // FP64 accumulator: 2 words per column
 };
 static_assert(F64Cfg::ACC_COL + 2 * F64Cfg::BN == 512, "TMEM budget: 2 partial buffers + FP64 accumulator");
-static_assert(128 * F64Cfg::REG_CTRL + 512 * F64Cfg::REG_DRAIN <= F64Cfg::THREADS * F64Cfg::REG_LAUNCH,
+static_assert(kKChunk % F64Cfg::KSPAN == 0, "a K-chunk is a whole number of stages");
+static_assert(8 * F64Cfg::NBARS + 8 <= 256, "barrier area");
+static_assert(F64Cfg::SMEM <= 232448, "shared memory per CTA");
+static_assert(128 * F64Cfg::REG_CTRL + 512 * F64Cfg::REG_DRAIN + 128 * F64Cfg::REG_FOLD <=
+                  F64Cfg::THREADS * F64Cfg::REG_LAUNCH,
               "setmaxnreg split exceeds the registers reserved at launch");
 
 template <uint32_t R> __device__ __forceinline__ void regs_dec() { asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R)); }
@@ -81,8 +98,9 @@ __device__ __forceinline__ double widen_exact(float x)
 // (i, j) in FP32 is provably exact: every partial is an integer multiple of the
 // unit u = 2^(vA_i + vB_j - 16), so any sum of magnitude below 2^24 u is
 // representable, and rounding is monotone, so a rounded sum below 2^24 u was
-// exact.  0 (always take the error-free path) when the levels are unknown or
-// the bound is not a normal float; +inf for a product of an all-zero slice.
+// exact.  0 (always take the error-free path, renormalising every time) when
+// the levels are unknown or the bound is not a normal float; +inf for a
+// product of an all-zero slice.
 __device__ __forceinline__ float exact_bound(const int32_t *vA, const int32_t *vB, int i, int j)
 {
     if (!vA) return 0.0f;
@@ -115,8 +133,58 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16
         : "memory");
 }
 
+__device__ __forceinline__ uint32_t tmem_ld1(uint32_t taddr)
+{
+    uint32_t r;
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(r) : "r"(taddr) : "memory");
+    return r;
+}
+
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&r)[8])
+{
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                 : "r"(taddr)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8])
+{
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};"
+                 ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+                 : "memory");
+}
+
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
+
+// Error-free sum of two FP32 values (Knuth's TwoSum): s = fl(a + b), a + b = s + e.
+__device__ __forceinline__ float two_sum(float a, float b, float &e)
+{
+    const float s = __fadd_rn(a, b);
+    const float bb = __fsub_rn(s, a);
+    e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+    return s;
+}
+
+__device__ __forceinline__ void sts_v4(uint32_t addr, float a, float b, float c, float d)
+{
+    asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d) : "memory");
+}
+
+__device__ __forceinline__ float4 lds_v4(uint32_t addr)
+{
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr) : "memory");
+    return v;
+}
+
+// Shared-memory address of 16-byte chunk `c` (columns 4c .. 4c+3) of row r
+// of the hand-off area.
+__device__ __forceinline__ uint32_t hand_addr(uint32_t hand, int r, int c)
+{
+    return hand + (uint32_t)(r * 512 + ((c ^ (r & 7)) << 4));
+}
 
 template <int NPROD>
 __global__ void __launch_bounds__(F64Cfg::THREADS, 1)
@@ -131,9 +199,9 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     uint8_t *base_ptr = smem_raw + (base - raw);
     const uint32_t full0 = base + Cfg::BAR_OFF, empty0 = full0 + 8u * Cfg::STAGES;
     const uint32_t tfull0 = empty0 + 8u * Cfg::STAGES, tempty0 = tfull0 + 8u * Cfg::NBUF;
-    const uint32_t done_bar = tempty0 + 8u * Cfg::NBUF;
-    volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(
-        base_ptr + Cfg::BAR_OFF + 16 * Cfg::STAGES + 16 * Cfg::NBUF + 8);
+    const uint32_t hfull = tempty0 + 8u * Cfg::NBUF, hempty = hfull + 8u, done_bar = hempty + 8u;
+    const uint32_t hand = base + Cfg::HAND_OFF, hmask = base + Cfg::MASK_OFF;
+    volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(base_ptr + Cfg::BAR_OFF + 8 * Cfg::NBARS);
 
     const int warp = threadIdx.x >> 5, lane = lane_id();
     const int tiles_m = (M + kBM - 1) / kBM, tiles_n = (N + Cfg::BN - 1) / Cfg::BN;
@@ -141,11 +209,12 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     tile_coords(blockIdx.x, tiles_m, tiles_n, tm, tn);
     const int m0 = tm * kBM, n0 = tn * Cfg::BN;
     const int nch = (K + kKChunk - 1) / kKChunk;
-    const int nt = NPROD * nch;                   // partials of this tile, product-major
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < Cfg::STAGES; ++s) { mbar_init(full0 + 8u * s, 1); mbar_init(empty0 + 8u * s, 1); }
         for (int b = 0; b < Cfg::NBUF; ++b) { mbar_init(tfull0 + 8u * b, 1); mbar_init(tempty0 + 8u * b, Cfg::DRAIN_WARPS); }
+        mbar_init(hfull, Cfg::DRAIN_WARPS);
+        mbar_init(hempty, 4);
         mbar_init(done_bar, 1);
         fence_mbar_init();
         tma_prefetch_desc(&tmA);
@@ -189,7 +258,7 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
         int s = 0, b = 0;
         uint32_t ph = 0, tph = 0;
         bool ok = true;
-        for (int t = 0; t < nt && ok; ++t) {
+        for (int t = 0; t < NPROD * nch && ok; ++t) {
             const int c = t % nch;
             const int kspans = min(kKChunk / Cfg::KSPAN, (K - c * kKChunk + Cfg::KSPAN - 1) / Cfg::KSPAN);
             if (!(ok = mbar_wait(tempty0 + 8u * b, tph ^ 1u, flags))) break;
@@ -217,18 +286,16 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
         mma_commit(done_bar);
         (void)mbar_wait(done_bar, 0, flags);
       }
-    } else {
+    } else if (warp < Cfg::FIRST_FOLD) {
         regs_inc<Cfg::REG_DRAIN>();
-        // ---------------- drain: exact per-product sum of the partials, one FP64 add per product
+        // ---------------- drain: exact per-product sum of the partials
         const int quarter = warp & 3;                                    // TMEM lanes 32*quarter ..
-        const int colh = ((warp - Cfg::FIRST_DRAIN) >> 2) * Cfg::COLS;   // this warp's 32 columns
-        const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
-        const uint32_t acc_base = lane_base + Cfg::ACC_COL + 2u * (uint32_t)colh;
-        const int row = m0 + quarter * 32 + lane;
-        const bool row_ok = row < M;
-        const bool vec = ((ldc & 1) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15u) == 0);
-        double *crow = C + (int64_t)row * ldc + n0 + colh;
-        const int lim = N - (n0 + colh);                  // valid columns of this warp's slice
+        const int cq = (warp - Cfg::FIRST_DRAIN) >> 2;                   // column quarter
+        const int r = quarter * 32 + lane;                               // tile row of this thread
+        const uint32_t tcol = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(cq * Cfg::COLS);
+        const int row = m0 + r;
+        double *crow = C + (int64_t)row * ldc + n0 + cq * Cfg::COLS;
+        const int lim = row < M ? N - (n0 + cq * Cfg::COLS) : 0;        // valid columns of this thread
         float hi[Cfg::COLS];
         bool ok = true;
         for (int q = 0; q < NPROD && ok; ++q) {
@@ -242,74 +309,122 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                 __syncwarp();
                 if (!ok) break;
                 tc_fence_after();
-                uint32_t v[Cfg::COLS];
-#pragma unroll
-                for (int h = 0; h < Cfg::COLS; h += 16)
-                    tmem_ld16(lane_base + (uint32_t)(b * Cfg::BN + colh + h), *reinterpret_cast<uint32_t(*)[16]>(v + h));
-                tmem_ld_wait();
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(tempty0 + 8u * b);    // buffer free: values are in registers
 #pragma unroll
                 for (int h = 0; h < Cfg::COLS; h += 16) {
-                    float sum[16];
+                    const uint32_t taddr = tcol + (uint32_t)(b * Cfg::BN + h);
+                    uint32_t v[16];                           // the partials, then the sums
+                    tmem_ld16(taddr, v);
+                    tmem_ld_wait();
                     bool big = false;
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
-                        sum[j] = __fadd_rn(hi[h + j], __uint_as_float(v[h + j]));
-                        big |= !(fabsf(sum[j]) < bound);
+                        const float sm = __fadd_rn(hi[h + j], __uint_as_float(v[j]));
+                        big |= !(fabsf(sm) < bound);
+                        v[j] = __float_as_uint(sm);
                     }
-                    if (__any_sync(0xFFFFFFFFu, big)) {       // rare: exact TwoSum errors into the low part
+                    if (!__any_sync(0xFFFFFFFFu, big)) {
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) hi[h + j] = __uint_as_float(v[j]);
+                    } else {
+                        // rare: redo the 16 additions as TwoSums, the errors summed
+                        // exactly into the low part; the partials are read again from
+                        // TMEM (the buffer is not yet released)
                         const bool was = (dirty >> (h / 16)) & 1u;
                         dirty |= 1u << (h / 16);
+                        const float renorm = 0.5f * bound;        // lo is kept below 2^23 u
+                        float *lrow = reinterpret_cast<float *>(crow) + (q & 1);
 #pragma unroll
-                        for (int j = 0; j < 16; ++j) {
-                            const float p = __uint_as_float(v[h + j]);
-                            const float bb = __fsub_rn(sum[j], hi[h + j]);
-                            const float e = __fadd_rn(__fsub_rn(hi[h + j], __fsub_rn(sum[j], bb)), __fsub_rn(p, bb));
-                            if (row_ok && h + j < lim) crow[h + j] = __dadd_rn(was ? crow[h + j] : 0.0, (double)e);
+                        for (int jj = 0; jj < 16; ++jj) {
+                            const int j = h + jj;
+                            const float p = __uint_as_float(tmem_ld1(taddr + (uint32_t)jj));
+                            tmem_ld_wait();
+                            float e, lo;
+                            const float sm = two_sum(hi[j], p, e);
+                            const bool mine = j < lim;
+                            lo = __fadd_rn((was && mine) ? lrow[2 * j] : 0.0f, e);
+                            hi[j] = (fabsf(lo) < renorm) ? sm : two_sum(sm, lo, lo);   // renormalise (hi, lo)
+                            if (mine) lrow[2 * j] = lo;
                         }
                     }
-#pragma unroll
-                    for (int j = 0; j < 16; ++j) hi[h + j] = sum[j];
+                    if (h + 16 == Cfg::COLS) {                   // buffer free: all values are in registers
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(tempty0 + 8u * b);
+                    }
                 }
             }
             if (!ok) break;
-            // fold: C <- fl64(C + (hi + lo)); hi + lo is exact in FP64
+            // hand the sums over once the fold warps have taken the previous product's
+            if (q > 0) {
+                ok = mbar_wait(hempty, (uint32_t)((q - 1) & 1), flags);
+                __syncwarp();
+                if (!ok) break;
+            }
+#pragma unroll
+            for (int k = 0; k < Cfg::COLS / 4; ++k)
+                sts_v4(hand_addr(hand, r, cq * (Cfg::COLS / 4) + k), hi[4 * k], hi[4 * k + 1], hi[4 * k + 2], hi[4 * k + 3]);
+            asm volatile("st.shared.u8 [%0], %1;" ::"r"(hmask + (uint32_t)(r * 4 + cq)), "r"(dirty) : "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(hfull);
+        }
+    } else {
+        regs_dec<Cfg::REG_FOLD>();
+        // ---------------- fold: C <- fl64(C + (hi + lo)) per product, in product order
+        const int quarter = warp & 3;
+        const int r = quarter * 32 + lane;
+        const uint32_t tacc = tmem + ((uint32_t)(quarter * 32) << 16) + Cfg::ACC_COL;
+        const int row = m0 + r;
+        double *crow = C + (int64_t)row * ldc + n0;
+        const int lim = row < M ? N - n0 : 0;
+        const bool vec = ((ldc & 1) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15u) == 0);
+        for (int q = 0; q < NPROD; ++q) {
+            const bool ok = mbar_wait(hfull, (uint32_t)(q & 1), flags);
+            __syncwarp();
+            if (!ok) break;
             const bool last = (q == NPROD - 1);
+            const float *lrow = reinterpret_cast<const float *>(crow) + (q & 1);
+#pragma unroll 1
+            for (int cq = 0; cq < 4; ++cq) {
+                uint32_t mask;
+                asm volatile("ld.shared.u8 %0, [%1];" : "=r"(mask) : "r"(hmask + (uint32_t)(r * 4 + cq)) : "memory");
 #pragma unroll
-            for (int g = 0; g < Cfg::COLS; g += 8) {
-                uint32_t w[16];
-                if (q > 0) {
-                    tmem_ld16(acc_base + 2u * g, w);
-                    tmem_ld_wait();
-                }
-                const bool dg = (dirty >> (g / 16)) & 1u;
+                for (int k = 0; k < 8; k += 2) {
+                    const int col = cq * 32 + 4 * k;                 // 8 columns: chunks k, k + 1
+                    const float4 h0 = lds_v4(hand_addr(hand, r, cq * 8 + k));
+                    const float4 h1 = lds_v4(hand_addr(hand, r, cq * 8 + k + 1));
+                    const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+                    uint32_t w[16];
+                    if (q > 0) {
+                        tmem_ld16(tacc + 2u * (uint32_t)col, w);
+                        tmem_ld_wait();
+                    }
+                    const bool dg = (mask >> (k / 4)) & 1u;      // 16-column group of these 8 columns
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    double sq = widen_exact(hi[g + j]);
-                    if (dg && row_ok && g + j < lim) sq = __dadd_rn(sq, crow[g + j]);   // exact
-                    const double cprev = (q > 0) ? __hiloint2double((int)w[2 * j + 1], (int)w[2 * j]) : 0.0;
-                    const double out = __dadd_rn(cprev, sq);
-                    w[2 * j] = (uint32_t)__double2loint(out);
-                    w[2 * j + 1] = (uint32_t)__double2hiint(out);
-                }
-                if (!last) {
-                    tmem_st16(acc_base + 2u * g, w);
-                } else if (row_ok) {
-                    if (vec && lim >= g + 8) {
+                    for (int j = 0; j < 8; ++j) {
+                        double sq = widen_exact(hv[j]);
+                        if (dg && col + j < lim) sq = __dadd_rn(sq, widen_exact(lrow[2 * (col + j)]));   // exact
+                        const double cprev = (q > 0) ? __hiloint2double((int)w[2 * j + 1], (int)w[2 * j]) : 0.0;
+                        const double out = __dadd_rn(cprev, sq);
+                        w[2 * j] = (uint32_t)__double2loint(out);
+                        w[2 * j + 1] = (uint32_t)__double2hiint(out);
+                    }
+                    if (!last) {
+                        tmem_st16(tacc + 2u * (uint32_t)col, w);
+                    } else if (vec && lim >= col + 8) {
 #pragma unroll
                         for (int j = 0; j < 8; j += 2)
-                            *reinterpret_cast<int4 *>(crow + g + j) =
+                            *reinterpret_cast<int4 *>(crow + col + j) =
                                 make_int4((int)w[2 * j], (int)w[2 * j + 1], (int)w[2 * j + 2], (int)w[2 * j + 3]);
                     } else {
 #pragma unroll
                         for (int j = 0; j < 8; ++j)
-                            if (g + j < lim) crow[g + j] = __hiloint2double((int)w[2 * j + 1], (int)w[2 * j]);
+                            if (col + j < lim) crow[col + j] = __hiloint2double((int)w[2 * j + 1], (int)w[2 * j]);
                     }
                 }
             }
             if (!last) tmem_st_wait();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(hempty);
         }
     }
     tc_fence_before();
