@@ -127,6 +127,39 @@ emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_
                         const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,
                         void *ws, size_t ws_bytes, emu_stream_t stream);
 
+/* Workspace bytes for emu_gemm_f32_host (mode 32) / emu_gemm_f64_host (mode
+ * 64): the header, the planes of A and B, staging space for the copied
+ * inputs (FP32: two row panels of A and two K-panels of B; FP64: A and B
+ * whole) and two row panels of C.  0 for negative sizes or another mode. */
+size_t emu_gemm_host_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K);
+
+/* The GEMMs of emu_gemm_f32 / emu_gemm_f64 (Algorithms 1 and 2, same kernels,
+ * bit-identical results) on operands in HOST memory: A (M x K, lda), B (K x N,
+ * ldb) and C (M x N, ldc) are host pointers, row-major; ws is a DEVICE
+ * workspace of at least emu_gemm_host_workspace_bytes bytes, 256-byte
+ * aligned.  The call enqueues the whole job and returns; C is complete when
+ * `stream` reaches the point after the call (synchronise it before reading
+ * C).  The host buffers must stay valid and unchanged until then.  Pinned
+ * (page-locked) host memory gives full copy speed and an asynchronous call;
+ * pageable memory works but the runtime then copies synchronously.
+ * Internally the copies, the split and the product-sum are pipelined over
+ * panels on streams that the library creates once per device (the current
+ * device must be the stream's device): FP32 copies B in K-panels and A in
+ * row panels, each split as soon as it lands, and multiplies row panels as
+ * their A rows arrive; FP64 copies A and B whole (its split needs the
+ * maximum over the whole operand, Eq. (fp64split)) and overlaps B's copy
+ * with A's split.  Finished row panels of C are copied back while the next
+ * is computed.  Concurrent calls on one device are serialised by the
+ * library.  The flag word (emu_read_flags on ws) reports the split and
+ * watchdog flags of the call.  Errors: as emu_gemm_f32 / emu_gemm_f64;
+ * EMU_ERR_MISALIGNED for a workspace not 256-byte aligned. */
+emu_status emu_gemm_f32_host(int64_t M, int64_t N, int64_t K, const float *A, int64_t lda,
+                             const float *B, int64_t ldb, float *C, int64_t ldc, void *ws,
+                             size_t ws_bytes, emu_stream_t stream);
+emu_status emu_gemm_f64_host(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda,
+                             const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,
+                             void *ws, size_t ws_bytes, emu_stream_t stream);
+
 /* Product-sum alone, from planes already split (A: [3][M][ldcomp],
  * B: [3][N][ldcomp], i.e. split with transpose = 1).  Eq. (fp32six),
  * Section 5.3.  ws: at least emu_split_workspace_bytes(32) (flag word). */

@@ -36,6 +36,9 @@ _SIGS = {
     "emu_prodsum_f32": ("i", ["l", "l", "l", "p", "p", "l", "p", "l", "p", "size", "p"]),
     "emu_prodsum_f64": ("i", ["l", "l", "l", "p", "p", "l", "p", "p", "i", "p", "l", "p", "size", "p"]),
     "emu_gemm_f64_noalloc": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "p"]),
+    "emu_gemm_host_workspace_bytes": ("size", ["i", "l", "l", "l"]),
+    "emu_gemm_f32_host": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "p", "size", "p"]),
+    "emu_gemm_f64_host": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "size", "p"]),
     "emu_read_flags": ("i", ["p", "p", "p"]),
     "emu_selftest_timeout": ("i", ["p", "size", "u32", "p"]),
     "emu_status_string": ("str", ["i"]),
@@ -87,6 +90,9 @@ emu_gemm_f64 = _mk("emu_gemm_f64")
 emu_prodsum_f32 = _mk("emu_prodsum_f32")
 emu_prodsum_f64 = _mk("emu_prodsum_f64")
 emu_gemm_f64_noalloc = _mk("emu_gemm_f64_noalloc")
+emu_gemm_host_workspace_bytes = _mk("emu_gemm_host_workspace_bytes")
+emu_gemm_f32_host = _mk("emu_gemm_f32_host")
+emu_gemm_f64_host = _mk("emu_gemm_f64_host")
 emu_read_flags = _mk("emu_read_flags")
 emu_selftest_timeout = _mk("emu_selftest_timeout")
 emu_status_string = _mk("emu_status_string")
@@ -174,6 +180,28 @@ def gemm_f64(A, B, nprod: int, C=None, ws=None, stream=None):
     ws = ws if ws is not None else workspace(emu_gemm_workspace_bytes(64, M, N, K), A.device)
     _check(emu_gemm_f64(M, N, K, A.data_ptr(), A.stride(0), B.data_ptr(), B.stride(0), C.data_ptr(), C.stride(0),
                         int(nprod), ws.data_ptr(), ws.numel(), _stream(stream)), "emu_gemm_f64")
+    return C, ws
+
+
+def gemm_host(A, B, nprod: int | None = None, C=None, ws=None, stream=None, device="cuda"):
+    """emu_gemm_f32_host / emu_gemm_f64_host: C = A.B with A, B, C in host
+    memory (CPU tensors; pinned ones give asynchronous full-speed copies).
+    FP32 inputs run Algorithm 1, FP64 inputs Algorithm 2 with nprod products.
+    Returns (C, ws) after enqueueing; synchronise the stream before reading C."""
+    torch = _torch()
+    M, K = A.shape
+    N = B.shape[1]
+    f64 = A.dtype == torch.float64
+    C = C if C is not None else torch.empty((M, N), dtype=A.dtype, pin_memory=True)
+    mode = 64 if f64 else 32
+    ws = ws if ws is not None else workspace(emu_gemm_host_workspace_bytes(mode, M, N, K), device)
+    if f64:
+        r = emu_gemm_f64_host(M, N, K, A.data_ptr(), A.stride(0), B.data_ptr(), B.stride(0), C.data_ptr(),
+                              C.stride(0), int(nprod), ws.data_ptr(), ws.numel(), _stream(stream))
+    else:
+        r = emu_gemm_f32_host(M, N, K, A.data_ptr(), A.stride(0), B.data_ptr(), B.stride(0), C.data_ptr(),
+                              C.stride(0), ws.data_ptr(), ws.numel(), _stream(stream))
+    _check(r, "emu_gemm_f64_host" if f64 else "emu_gemm_f32_host")
     return C, ws
 
 

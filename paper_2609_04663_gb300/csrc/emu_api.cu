@@ -1,18 +1,8 @@
 // C-ABI of the emulation library (declared in include/emu.h): argument
 // checks, workspace layout and the launch sequence of each entry point.
-#include "common.cuh"
+#include "launchers.cuh"
 
 namespace emu {
-cudaError_t launch_split_f32(const float *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
-                             uint16_t *comps, int64_t ldcomp, WsHeader *ws, cudaStream_t st);
-cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
-                             uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
-                             cudaStream_t st);
-cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
-                               int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st);
-cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
-                               int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
-                               int64_t ldc, uint32_t *flags, cudaStream_t st);
 
 // Watchdog self-test: one bounded wait on a barrier that nothing completes.
 namespace {

@@ -50,14 +50,15 @@ inline EncodeTiledFn encode_fn()
 
 // Tensor map over a plane set [S][rows][ldcomp] of BF16: dims (K, rows, S),
 // box (kb, box_rows, 1), swizzle matching a kb * 2-byte row.  Out-of-range
-// boxes (ragged M, N, K) read zeros.
+// boxes (ragged M, N, K) read zeros.  plane: distance between planes in
+// elements (0 = rows * ldcomp).
 inline bool make_plane_map(CUtensorMap *map, const uint16_t *planes, int64_t K, int64_t rows, int S, int64_t ldcomp,
-                    int kb, int box_rows)
+                    int kb, int box_rows, int64_t plane = 0)
 {
     EncodeTiledFn enc = encode_fn();
     if (!enc) return false;
     cuuint64_t dims[3] = {(cuuint64_t)K, (cuuint64_t)rows, (cuuint64_t)S};
-    cuuint64_t strides[2] = {(cuuint64_t)ldcomp * 2, (cuuint64_t)rows * ldcomp * 2};
+    cuuint64_t strides[2] = {(cuuint64_t)ldcomp * 2, (cuuint64_t)(plane ? plane : rows * ldcomp) * 2};
     cuuint32_t box[3] = {(cuuint32_t)kb, (cuuint32_t)box_rows, 1};
     cuuint32_t estr[3] = {1, 1, 1};
     const CUtensorMapSwizzle swz = (kb == 64) ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;

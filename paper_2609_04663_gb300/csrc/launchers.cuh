@@ -1,0 +1,31 @@
+// Host-side launch functions of the kernels, shared by the C-ABI translation
+// units (emu_api.cu, noalloc.cu, host_api.cu).  Each enqueues its kernels on
+// `st` and returns the launch error; device-side failures set flag bits.
+#pragma once
+
+#include "common.cuh"
+
+namespace emu {
+
+// Eq. (fp32split): X [rows][ldx] FP32 -> 3 BF16 planes of [transpose ? cols : rows][ldcomp].
+// plane: distance between planes in elements (0 = dense: (transpose ? cols : rows) * ldcomp).
+cudaError_t launch_split_f32(const float *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
+                             uint16_t *comps, int64_t ldcomp, WsHeader *ws, cudaStream_t st, int64_t plane = 0);
+
+// Eq. (fp64split): X -> 6 BF16 planes and the level exponents v_out[6]; `slot`
+// selects the header's per-operand state (0 = A, 1 = B).
+cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
+                             uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
+                             cudaStream_t st);
+
+// Product-sums from K-major planes; a_plane: distance between the A planes in
+// elements (0 = dense: M * ldcomp), so that a row panel of a larger plane set
+// can be multiplied on its own.
+cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
+                               int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
+                               int64_t a_plane = 0);
+cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
+                               int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
+                               int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane = 0);
+
+}  // namespace emu

@@ -16,16 +16,7 @@
 // host threads) race on it.
 #include <mutex>
 
-#include "common.cuh"
-
-namespace emu {
-cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
-                             uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
-                             cudaStream_t st);
-cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
-                               int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
-                               int64_t ldc, uint32_t *flags, cudaStream_t st);
-}  // namespace emu
+#include "launchers.cuh"
 
 using namespace emu;
 

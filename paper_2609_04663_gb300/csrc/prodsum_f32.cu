@@ -13,6 +13,7 @@
 #include <cstdlib>
 
 #include "gemm_common.cuh"
+#include "launchers.cuh"
 
 namespace emu {
 
@@ -150,11 +151,11 @@ prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
 
 template <int BN, int KB, int STAGES>
 cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
-                    float *C, int64_t ldc, uint32_t *flags, cudaStream_t st)
+                    float *C, int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane)
 {
     using Cfg = F32Cfg<BN, KB, STAGES>;
     CUtensorMap ta, tb;
-    if (!make_plane_map(&ta, Ap, K, M, 3, ldcomp, KB, kBM) || !make_plane_map(&tb, Bp, K, N, 3, ldcomp, KB, BN))
+    if (!make_plane_map(&ta, Ap, K, M, 3, ldcomp, KB, kBM, a_plane) || !make_plane_map(&tb, Bp, K, N, 3, ldcomp, KB, BN))
         return cudaErrorInvalidValue;
     auto kern = prodsum_f32_kernel<BN, KB, STAGES>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
@@ -170,14 +171,15 @@ cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
 // by default; EMU_F32_TILE=128x128 selects 128 x 128 with 64-wide K-blocks
 // (128-byte swizzle, 2 stages).
 cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
-                               int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st)
+                               int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
+                               int64_t a_plane)
 {
     static const bool narrow = [] {
         const char *e = std::getenv("EMU_F32_TILE");
         return e && e[0] == '1' && e[1] == '2' && e[2] == '8' && e[3] == 'x' && e[4] == '1';
     }();
-    if (narrow) return run_f32<128, 64, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st);
-    return run_f32<256, 32, 3>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st);
+    if (narrow) return run_f32<128, 64, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane);
+    return run_f32<256, 32, 3>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane);
 }
 
 }  // namespace emu

@@ -31,6 +31,7 @@
 // setmaxnreg moves registers between the warpgroups.  Every wait is bounded
 // and reports EMU_FLAG_TIMEOUT instead of hanging.
 #include "gemm_common.cuh"
+#include "launchers.cuh"
 
 namespace emu {
 
@@ -438,11 +439,12 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
 
 template <int NPROD>
 cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
-                    const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, uint32_t *flags, cudaStream_t st)
+                    const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
+                    int64_t a_plane)
 {
     using Cfg = F64Cfg;
     CUtensorMap ta, tb;
-    if (!make_plane_map(&ta, Ap, K, M, 6, ldcomp, Cfg::KB, kBM) || !make_plane_map(&tb, Bp, K, N, 6, ldcomp, Cfg::KB, Cfg::BN))
+    if (!make_plane_map(&ta, Ap, K, M, 6, ldcomp, Cfg::KB, kBM, a_plane) || !make_plane_map(&tb, Bp, K, N, 6, ldcomp, Cfg::KB, Cfg::BN))
         return cudaErrorInvalidValue;
     auto kern = prodsum_f64_kernel<NPROD>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
@@ -456,13 +458,13 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
 
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
-                               int64_t ldc, uint32_t *flags, cudaStream_t st)
+                               int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane)
 {
     switch (nprod) {
-    case 6: return run_f64<6>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st);
-    case 10: return run_f64<10>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st);
-    case 15: return run_f64<15>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st);
-    case 21: return run_f64<21>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st);
+    case 6: return run_f64<6>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st, a_plane);
+    case 10: return run_f64<10>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st, a_plane);
+    case 15: return run_f64<15>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st, a_plane);
+    case 21: return run_f64<21>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st, a_plane);
     default: return cudaErrorInvalidValue;
     }
 }

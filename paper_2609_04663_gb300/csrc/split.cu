@@ -16,7 +16,7 @@
 // checks the assumption level by level; only if it fails do the gated fix
 // kernels recompute the remaining levels literally.  The result is
 // identical to the literal definition in every case.
-#include "common.cuh"
+#include "launchers.cuh"
 
 namespace emu {
 
@@ -528,10 +528,10 @@ int grid_for(int64_t work_items, int max_blocks)
 
 // ----------------------------------------------------------- host launchers
 cudaError_t launch_split_f32(const float *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
-                             uint16_t *comps, int64_t ldcomp, WsHeader *ws, cudaStream_t st)
+                             uint16_t *comps, int64_t ldcomp, WsHeader *ws, cudaStream_t st, int64_t plane_stride)
 {
     if (rows == 0 || cols == 0) return cudaSuccess;
-    const int64_t plane = (transpose ? cols : rows) * ldcomp;
+    const int64_t plane = plane_stride ? plane_stride : (transpose ? cols : rows) * ldcomp;
     const int64_t tiles = ((rows + kTile - 1) / kTile) * ((cols + kTile - 1) / kTile);
     const int grid = grid_for(tiles, 152 * 16);
     const size_t sm = smem_bytes(3);

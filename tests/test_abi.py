@@ -64,3 +64,22 @@ def test_host_argument_checks_need_no_gpu(lib):
     assert emu.emu_gemm_f32(1 << 31, 4, 4, P, 4, P, 4, P, 4, P, 1 << 62, None) == 5  # size limit
     assert emu.emu_split_f64(P, 4, 4, 2, 0, P, 4, P, P, 4096, None) == 1              # ldx < cols
     assert emu.emu_selftest_timeout(P, 4096, 0, None) == 1
+    # host-buffer GEMMs: validation precedes every CUDA call
+    W = 256  # 256-byte aligned dummy workspace address
+    assert emu.emu_gemm_f32_host(4, 4, 4, P, 3, P, 4, P, 4, W, 1 << 40, None) == 1      # lda < K
+    assert emu.emu_gemm_f64_host(4, 4, 4, P, 4, P, 4, P, 4, 5, W, 1 << 40, None) == 1   # nprod
+    assert emu.emu_gemm_f32_host(4, 4, 4, P, 4, P, 4, P, 4, P, 1 << 40, None) == 2      # ws not 256-aligned
+    assert emu.emu_gemm_f32_host(4, 4, 4, P, 4, P, 4, P, 4, W, 64, None) == 3           # workspace
+    assert emu.emu_gemm_f64_host(4, 4, 4, 0, 4, P, 4, P, 4, 6, W, 1 << 40, None) == 1   # null A
+
+
+def test_host_workspace_sizes(lib):
+    M, N, K = 300, 200, 700
+    for mode in (32, 64):
+        need = emu.emu_gemm_host_workspace_bytes(mode, M, N, K)
+        assert need > emu.emu_gemm_workspace_bytes(mode, M, N, K)
+    assert emu.emu_gemm_host_workspace_bytes(16, M, N, K) == 0
+    assert emu.emu_gemm_host_workspace_bytes(32, -1, N, K) == 0
+    # FP64 stages both operands whole: at least 8 (MK + KN) bytes beyond the planes
+    assert emu.emu_gemm_host_workspace_bytes(64, M, N, K) >= emu.emu_gemm_workspace_bytes(64, M, N, K) + 8 * (M * K + K * N)
+
