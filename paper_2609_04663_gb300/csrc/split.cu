@@ -2,10 +2,13 @@
 // fixed six-slice simplified Ozaki split (Eq. (fp64split)), writing BF16
 // component planes row-major or transposed (K-major for the B operand).
 //
-// Both are HBM-bound elementwise passes.  A 64 x 64 tile of X is read with
-// coalesced vector loads, split in registers, staged in shared memory and
-// written as 16-byte chunks of whole plane rows, so the transposed B planes
-// are written as coalesced as the row-major A planes.
+// Both are HBM-bound elementwise passes.  The FP32 split works on element
+// pairs with the hardware BF16x2 conversion: row-major planes straight from
+// registers, transposed planes through a conflict-free shared-memory tile.
+// The FP64 split reads a 64 x 64 tile of X with coalesced vector loads,
+// splits it in registers, stages it in shared memory and writes 16-byte
+// chunks of whole plane rows, so transposed B planes are written as
+// coalesced as row-major A planes.
 //
 // FP64 level exponents need a whole-matrix max per level (v^(r) of
 // Eq. (fp64split)), i.e. six dependent grid-wide reductions.  The split does
@@ -27,17 +30,6 @@ constexpr int kSRow = kTile + 2;     // shared-memory row pitch in uint16 (odd w
 constexpr int kThreads = 256;
 
 // --------------------------------------------------------------- rounding
-// fl_BF16 of an FP32 value (round to nearest, ties to even) on its bit
-// pattern: add 0x7FFF plus the lowest kept bit, keep the upper half.
-__device__ __forceinline__ uint32_t bf16_rne_f32bits(float x)
-{
-    uint32_t u = __float_as_uint(x);
-    u += 0x7FFFu + ((u >> 16) & 1u);
-    return u >> 16;
-}
-
-__device__ __forceinline__ float bf16_as_float(uint32_t s) { return __uint_as_float(s << 16); }
-
 // fl_BF16 of an FP64 value, one rounding, by integer arithmetic on its bits:
 // the BF16 quantum is 2^(max(e, -126) - 7) for a leading-bit exponent e;
 // subnormal BF16 spacing 2^-133; overflow to infinity.
@@ -112,7 +104,7 @@ __device__ __forceinline__ uint16_t f64_level(double &R, int v, bool &bad)
         bad = true;
         s = bf16_rne_f64(Z);
     }
-    const double sv = (double)bf16_as_float(s);
+    const double sv = (double)__uint_as_float((uint32_t)s << 16);
     R = __dsub_rn(R, sv);
     return s;
 }
@@ -286,15 +278,16 @@ __device__ __forceinline__ void block_max_to(unsigned long long x, unsigned long
 }
 
 // ------------------------------------------------------------ tile kernel
-// MODE 0: FP32 split.  MODE 1: FP64 speculative split (v^(r) = v0 - 8r,
+// FP64 split.  MODE 1: speculative split (v^(r) = v0 - 8r,
 // records the maxima of |A^(r)|, r = 1..5).  MODE 2: FP64 rewrite with the
-// final levels (runs only when verification failed).
+// final levels (runs only when verification failed).  (T is double.)
 template <typename T, int MODE, bool TRANSPOSE>
 __global__ void __launch_bounds__(kThreads)
 split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
                   uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
 {
-    constexpr int NS = (MODE == 0) ? 3 : 6;
+    static_assert(MODE == 1 || MODE == 2, "FP64 split modes only");
+    constexpr int NS = 6;
     extern __shared__ __align__(16) uint16_t smdyn[];    // [NS][kTile][kSRow]
     auto sm = [&](int r, int row, int col) -> uint16_t & {
         return smdyn[((size_t)r * kTile + row) * kSRow + col];
@@ -312,7 +305,7 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
     }
 
     unsigned long long mx[5] = {0, 0, 0, 0, 0};         // max |A^(r)| as bit patterns
-    uint32_t badmask = 0, flagbits = 0;
+    uint32_t badmask = 0;
     const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;   // 16 x 16 threads
 
@@ -344,17 +337,7 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
             for (int e = 0; e < 4; ++e) {
                 const int lj = 4 * tx + e;
                 uint16_t s[NS];
-                if constexpr (MODE == 0) {
-                    float a = x[e];
-                    if (!isfinite(a)) flagbits |= EMU_FLAG_NONFINITE;
-#pragma unroll
-                    for (int r = 0; r < 3; ++r) {
-                        const uint32_t b = bf16_rne_f32bits(a);
-                        s[r] = (uint16_t)b;
-                        if ((b & 0x7F80u) == 0x7F80u) flagbits |= EMU_FLAG_SLICE;
-                        a = __fsub_rn(a, bf16_as_float(b));
-                    }
-                } else if constexpr (MODE == 1) {
+                if constexpr (MODE == 1) {
                     if (v[0] == kZeroLevel) {
 #pragma unroll
                         for (int r = 0; r < 6; ++r) s[r] = 0;
@@ -398,13 +381,8 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
         __syncthreads();
     }
 
-    if constexpr (MODE == 0) {
-        flagbits = __reduce_or_sync(0xFFFFFFFFu, flagbits);
-        if (flagbits && lane_id() == 0) atomicOr(&ws->flags, flagbits);
-    } else {
-        badmask = __reduce_or_sync(0xFFFFFFFFu, badmask);
-        if (badmask && lane_id() == 0) atomicOr(&ws->slice_bad[slot], MODE == 1 ? badmask : badmask << 8);
-    }
+    badmask = __reduce_or_sync(0xFFFFFFFFu, badmask);
+    if (badmask && lane_id() == 0) atomicOr(&ws->slice_bad[slot], MODE == 1 ? badmask : badmask << 8);
     if constexpr (MODE == 1) {
         // mx holds |A^(r)| in units of 2^(v0 - 50), below 2^53: exact as doubles
         const int F = (v[0] == kZeroLevel) ? 0 : v[0] - 50;
@@ -516,6 +494,152 @@ __global__ void f64_finalize_kernel(WsHeader *ws, int slot, int32_t *v_out)
     if (bad) atomicOr(&ws->flags, (uint32_t)EMU_FLAG_SLICE);
 }
 
+// ------------------------------------------------------ FP32 split kernels
+// Eq. (fp32split) on pairs of elements: the hardware conversion
+// cvt.rn.bf16x2.f32 rounds two FP32 values to BF16 (round to nearest, ties
+// to even, subnormals kept) and packs them into one 32-bit word, low element
+// in the low half.  The residual of each is an exact FP32 subtraction of its
+// slice, whose FP32 value is the BF16 bits shifted into the upper half.
+__device__ __forceinline__ uint32_t bf16x2_rn(float lo, float hi)
+{
+    uint32_t d;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+    return d;
+}
+
+// Three slice words (planes 0, 1, 2) of the element pair (x0, x1).
+__device__ __forceinline__ void split_pair(float x0, float x1, uint32_t &w0, uint32_t &w1, uint32_t &w2)
+{
+    w0 = bf16x2_rn(x0, x1);
+    const float r0 = __fsub_rn(x0, __uint_as_float(w0 << 16)), r1 = __fsub_rn(x1, __uint_as_float(w0 & 0xFFFF0000u));
+    w1 = bf16x2_rn(r0, r1);
+    const float q0 = __fsub_rn(r0, __uint_as_float(w1 << 16)), q1 = __fsub_rn(r1, __uint_as_float(w1 & 0xFFFF0000u));
+    w2 = bf16x2_rn(q0, q1);
+}
+
+// Flags of Eq. (fp32split)'s domain from the largest |x| bit pattern seen:
+// a non-finite input, and a slice that is not finite.  For a finite x the
+// only non-finite slice is slice 0 rounding up to infinity, which happens
+// exactly when |x| >= 0x7F7F8000 (half a BF16 ulp above the largest BF16).
+__device__ __forceinline__ void publish_f32_flags(uint32_t amax, WsHeader *ws)
+{
+    uint32_t f = (amax >= 0x7F800000u ? (uint32_t)EMU_FLAG_NONFINITE : 0u) |
+                 (amax >= 0x7F7F8000u ? (uint32_t)EMU_FLAG_SLICE : 0u);
+    f = __reduce_or_sync(0xFFFFFFFFu, f);
+    if (f && lane_id() == 0) atomicOr(&ws->flags, f);
+}
+
+// Row-major planes: thread = 8 consecutive elements of a row (two 16-byte
+// loads, one 16-byte store per plane), no shared memory.  Rows advance by
+// the grid's y dimension.
+__global__ void __launch_bounds__(kThreads)
+split_f32_rows_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                      uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws)
+{
+    const bool vin = ((ldx & 3) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
+    const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
+    const int64_t j0 = ((int64_t)blockIdx.x * kThreads + threadIdx.x) * 8;
+    uint32_t amax = 0;
+    if (j0 < cols) {
+        const bool full = j0 + 8 <= cols;
+        for (int64_t i = blockIdx.y; i < rows; i += gridDim.y) {
+            const float *src = X + i * ldx + j0;
+            float x[8];
+            if (vin && full) {
+                const float4 a = reinterpret_cast<const float4 *>(src)[0], b = reinterpret_cast<const float4 *>(src)[1];
+                x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) x[e] = (j0 + e < cols) ? src[e] : 0.0f;
+            }
+            uint32_t w[3][4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                amax = max(amax, max(__float_as_uint(x[2 * e]) & 0x7FFFFFFFu, __float_as_uint(x[2 * e + 1]) & 0x7FFFFFFFu));
+                split_pair(x[2 * e], x[2 * e + 1], w[0][e], w[1][e], w[2][e]);
+            }
+            uint16_t *dst = comps + i * ldcomp + j0;
+#pragma unroll
+            for (int r = 0; r < 3; ++r) {
+                if (vout && full) {
+                    *reinterpret_cast<uint4 *>(dst + r * plane) = make_uint4(w[r][0], w[r][1], w[r][2], w[r][3]);
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        if (j0 + e < cols) dst[r * plane + e] = (uint16_t)(w[r][e >> 1] >> (16 * (e & 1)));
+                }
+            }
+        }
+    }
+    publish_f32_flags(amax, ws);
+}
+
+// Transposed (K-major) planes: a 64 x 64 tile of X.  Warp q takes columns
+// 8q .. 8q+7, lane p rows 2p and 2p+1, so each slice word packs the two
+// elements that are adjacent in the transposed row; the words go to shared
+// memory (one bank per lane: conflict-free) and leave as 16-byte chunks of
+// whole transposed rows.
+__global__ void __launch_bounds__(kThreads)
+split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                           uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws)
+{
+    __shared__ __align__(16) uint32_t sm[3][kTile][kTile / 2];   // [plane][transposed row][word]
+    const bool vin = ((ldx & 3) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
+    const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
+    const int q = threadIdx.x >> 5, p = lane_id();
+    const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
+    uint32_t amax = 0;
+    for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
+        const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
+        const int64_t gj = c0 + 8 * q;
+        float x[2][8];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int64_t gi = r0 + 2 * p + h;
+            const float *src = X + gi * ldx + gj;
+            if (gi < rows && vin && gj + 8 <= cols) {
+                const float4 a = reinterpret_cast<const float4 *>(src)[0], b = reinterpret_cast<const float4 *>(src)[1];
+                x[h][0] = a.x; x[h][1] = a.y; x[h][2] = a.z; x[h][3] = a.w;
+                x[h][4] = b.x; x[h][5] = b.y; x[h][6] = b.z; x[h][7] = b.w;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) x[h][e] = (gi < rows && gj + e < cols) ? src[e] : 0.0f;
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            amax = max(amax, max(__float_as_uint(x[0][e]) & 0x7FFFFFFFu, __float_as_uint(x[1][e]) & 0x7FFFFFFFu));
+            uint32_t w0, w1, w2;
+            split_pair(x[0][e], x[1][e], w0, w1, w2);
+            sm[0][8 * q + e][p] = w0;
+            sm[1][8 * q + e][p] = w1;
+            sm[2][8 * q + e][p] = w2;
+        }
+        __syncthreads();
+        // 3 planes x 64 transposed rows x 8 chunks of 16 bytes
+#pragma unroll
+        for (int it = 0; it < 3 * kTile * 8 / kThreads; ++it) {
+            const int c = threadIdx.x + it * kThreads;
+            const int r = c >> 9, orow = (c >> 3) & 63, ch = c & 7;
+            const int64_t go = c0 + orow, gk = r0 + 8 * ch;
+            if (go < cols && gk < rows) {
+                const uint4 v = *reinterpret_cast<const uint4 *>(&sm[r][orow][4 * ch]);
+                uint16_t *dst = comps + r * plane + go * ldcomp + gk;
+                if (vout && gk + 8 <= rows) {
+                    *reinterpret_cast<uint4 *>(dst) = v;
+                } else {
+                    const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        if (gk + e < rows) dst[e] = (uint16_t)(wv[e >> 1] >> (16 * (e & 1)));
+                }
+            }
+        }
+        __syncthreads();
+    }
+    publish_f32_flags(amax, ws);
+}
+
 size_t smem_bytes(int ns) { return (size_t)ns * kTile * kSRow * sizeof(uint16_t); }
 
 int grid_for(int64_t work_items, int max_blocks)
@@ -532,13 +656,16 @@ cudaError_t launch_split_f32(const float *X, int64_t rows, int64_t cols, int64_t
 {
     if (rows == 0 || cols == 0) return cudaSuccess;
     const int64_t plane = plane_stride ? plane_stride : (transpose ? cols : rows) * ldcomp;
-    const int64_t tiles = ((rows + kTile - 1) / kTile) * ((cols + kTile - 1) / kTile);
-    const int grid = grid_for(tiles, 152 * 16);
-    const size_t sm = smem_bytes(3);
-    if (transpose)
-        split_tile_kernel<float, 0, true><<<grid, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, 0);
-    else
-        split_tile_kernel<float, 0, false><<<grid, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, 0);
+    if (transpose) {
+        const int64_t tiles = ((rows + kTile - 1) / kTile) * ((cols + kTile - 1) / kTile);
+        split_f32_transpose_kernel<<<grid_for(tiles, 152 * 8), kThreads, 0, st>>>(X, rows, cols, ldx, comps, ldcomp,
+                                                                                   plane, ws);
+    } else {
+        const int64_t bx = (cols + 8 * kThreads - 1) / (8 * kThreads);
+        const int64_t by = rows < 4096 ? rows : 4096;
+        split_f32_rows_kernel<<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, comps, ldcomp,
+                                                                                     plane, ws);
+    }
     return cudaGetLastError();
 }
 
