@@ -183,8 +183,8 @@ class Case:
         self.gemm_ws = None
         self.flop = 2.0 * M * N * K
         self.exec_flop = self.flop * (6 if self.mode == 32 else self.nprod)
-        # kernels of ours per step: FP32 split = 1 launch, FP64 split = 9, product-sum = 1
-        self.launches = (2 * 1 + 1) if self.mode == 32 else (2 * 9 + 1)
+        # kernels of ours per step: FP32 split = 1 launch, FP64 split = 10, product-sum = 1
+        self.launches = (2 * 1 + 1) if self.mode == 32 else (2 * 10 + 1)
         del np
 
     def split(self, stream):

@@ -396,8 +396,8 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
 
 // --------------------------------------------- row-segment FP64 passes
 // LEVEL = 0: max |x| and the input-domain checks of Eq. (bf16rangefp64).
-// LEVEL = L in 2..5: max |A^(L)| recomputed literally from x with the final
-// levels 0..L-1 (only when verification failed before level L).
+// LEVEL = L in 1..5: max |A^(L)| recomputed literally from x with the final
+// levels 0..L-1 (only when the trusted speculative levels end before L).
 template <int LEVEL>
 __global__ void __launch_bounds__(kThreads)
 f64_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, WsHeader *ws,
@@ -457,24 +457,31 @@ f64_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t
 
 // One thread: checks the speculative levels in order.  Level r's max from
 // the fused pass is literal as long as levels < r were right, so the first
-// mismatch r gives the true v^(r) directly; levels from r on are redone.
+// mismatch r gives the true v^(r) directly; levels after r are redone.  A
+// slice outside the BF16 normal range at level r (a domain violation, which
+// the finalizer flags) also ends the trusted levels at r: the fused pass
+// subtracts the exact projection Z there, while Eq. (fp64split) subtracts
+// fl_BF16(Z), so the literal passes redo the levels after r.
 __global__ void f64_verify_kernel(WsHeader *ws, int slot)
 {
     int ff = 6;
+    const uint32_t sb = ws->slice_bad[slot] & 0x3Fu;
+    const int badlvl = (sb && !(ws->flags & EMU_FLAG_NONFINITE)) ? __ffs(sb) - 1 : 6;
     const unsigned long long m0 = ws->maxbits[slot][0];
     if (m0 == 0) {
         for (int r = 0; r < 6; ++r) ws->v[slot][r] = kZeroLevel;
     } else {
         const int v0 = ceil_log2_bits(m0);
         ws->v[slot][0] = v0;
+        if (badlvl == 0) ff = 0;
         bool zero = false;
-        for (int r = 1; r < 6; ++r) {
+        for (int r = 1; r < 6 && ff == 6; ++r) {
             if (zero) { ws->v[slot][r] = kZeroLevel; continue; }
             const unsigned long long m = ws->maxbits[slot][r];
             if (m == 0) { ws->v[slot][r] = kZeroLevel; zero = true; continue; }
             const int vr = ceil_log2_bits(m);
             ws->v[slot][r] = vr;
-            if (vr != v0 - 8 * r) { ff = r; break; }
+            if (vr != v0 - 8 * r || r == badlvl) ff = r;
         }
     }
     ws->fix_from[slot] = ff;
@@ -492,6 +499,242 @@ __global__ void f64_finalize_kernel(WsHeader *ws, int slot, int32_t *v_out)
     const uint32_t sb = ws->slice_bad[slot];
     const uint32_t bad = (sb & keep & 0x3Fu) | ((sb >> 8) & ~keep & 0x3Fu);
     if (bad) atomicOr(&ws->flags, (uint32_t)EMU_FLAG_SLICE);
+}
+
+// ------------------------------------------ FP64 speculative pass kernels
+// The levels of spec_levels restated so that most steps are 32-bit: levels 0
+// and 1 have grids of 2^32 units or coarser and round on the upper word of
+// the fixed-point magnitude (the lower word only breaks ties and is carried
+// into the residual), level 2 rounds a value below 2^35 through its quotient
+// and remainder, and levels 3-5 work in 32 bits.  At each level the grid
+// splits |X| into t = |X| >> g and a remainder; rounding up (remainder above
+// half the grid, or exactly half with t odd) leaves the grid minus the
+// remainder with the opposite sign.  No range check is needed when
+// v0 >= -78: every nonzero slice then lies between 2^(v0 - 48) >= 2^-126 and
+// 2^v0 <= 2^127.  Results are bit-identical to spec_levels.
+__device__ __forceinline__ uint32_t bf16_of_level(uint32_t n, uint32_t sg, int eg)
+{
+    // n * 2^(eg - 127 - ...) as BF16: leading bit p of n (n <= 256), 7 bits below it
+    const int p = 31 - __clz(n | 1u);
+    const uint32_t out = (sg << 15) + ((uint32_t)(eg + p) << 7) + (((n << 7) >> p) & 0x7Fu);
+    return n ? out : 0u;
+}
+
+__device__ __forceinline__ void spec_levels_fast(double x, int F, uint32_t (&s)[6], uint32_t &badmask,
+                                                 unsigned long long &m1, unsigned long long &m2, uint32_t (&m)[3])
+{
+    const uint64_t b = (uint64_t)__double_as_longlong(x);
+    uint32_t sg = (uint32_t)(b >> 63);
+    const int E = (int)((b >> 52) & 0x7FFu);
+    uint64_t M = b & 0x000FFFFFFFFFFFFFull;
+    int Ee = E;
+    if (E == 0) Ee = 1; else M |= 1ull << 52;
+    if (E == 0x7FF) { badmask |= 1u; M = 0; }          // a non-finite slice 0
+    const int sh0 = (Ee - 1075) - F;
+    uint64_t a;
+    if (M == 0) a = 0;
+    else if (sh0 >= 0) a = sh0 < 12 ? (M << sh0) : (1ull << 62);
+    else if (sh0 > -64) a = (M >> (-sh0)) | ((M << (64 + sh0)) != 0 ? 1ull : 0ull);
+    else a = 1;
+    uint32_t H = (uint32_t)(a >> 32), L = (uint32_t)a;
+    // levels 0, 1: grid 2^(32 + gh) units, gh = 11 / 10 and 3 / 2
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+        if (r == 1) {
+            const unsigned long long cur = ((unsigned long long)H << 32) | L;
+            m1 = cur > m1 ? cur : m1;
+        }
+        const int gh = 11 - 8 * r - (int)sg;
+        const uint32_t t = H >> gh, rh = H & ((1u << gh) - 1u), hh = 1u << (gh - 1);
+        const bool up = (rh > hh) || (rh == hh && (L != 0u || (t & 1u)));
+        s[r] = bf16_of_level(t + (up ? 1u : 0u), sg, F + 32 + gh + 127);
+        if (up) { H = (1u << gh) - rh - (L != 0u ? 1u : 0u); L = 0u - L; sg ^= 1u; }
+        else H = rh;
+    }
+    // level 2: |X| < 2^35, grid 2^27 / 2^26
+    uint32_t Y;
+    {
+        const unsigned long long cur = ((unsigned long long)H << 32) | L;
+        m2 = cur > m2 ? cur : m2;
+        const int g = 27 - (int)sg;
+        const uint32_t t = (H << (32 - g)) | (L >> g), rem = L & ((1u << g) - 1u), half = 1u << (g - 1);
+        const bool up = rem > half || (rem == half && (t & 1u));
+        s[2] = bf16_of_level(t + (up ? 1u : 0u), sg, F + g + 127);
+        if (up) { Y = (1u << g) - rem; sg ^= 1u; } else Y = rem;
+    }
+    // levels 3-5: |X| <= 2^26
+#pragma unroll
+    for (int r = 3; r < 6; ++r) {
+        m[r - 3] = Y > m[r - 3] ? Y : m[r - 3];
+        const int g = 43 - 8 * r - (int)sg;
+        const uint32_t t = Y >> g, rem = Y & ((1u << g) - 1u), half = 1u << (g - 1);
+        const bool up = rem > half || (rem == half && (t & 1u));
+        s[r] = bf16_of_level(t + (up ? 1u : 0u), sg, F + g + 127);
+        if (up) { Y = (1u << g) - rem; sg ^= 1u; } else Y = rem;
+    }
+}
+
+// Per-thread state of the speculative pass: level maxima in units of 2^F.
+struct SpecState {
+    unsigned long long m1 = 0, m2 = 0;
+    uint32_t m[3] = {0, 0, 0};
+    uint32_t badmask = 0;
+};
+
+__device__ __forceinline__ void spec_element(double x, int v0, bool fast, uint32_t (&s)[6], SpecState &st)
+{
+    if (v0 == kZeroLevel) {
+#pragma unroll
+        for (int r = 0; r < 6; ++r) s[r] = 0;
+    } else if (fast) {
+        spec_levels_fast(x, v0 - 50, s, st.badmask, st.m1, st.m2, st.m);
+    } else {                                          // tiny matrices: the checked general form
+        uint16_t t[6];
+        unsigned long long mx[5] = {st.m1, st.m2, st.m[0], st.m[1], st.m[2]};
+        spec_levels(x, v0, t, st.badmask, mx);
+        st.m1 = mx[0]; st.m2 = mx[1];
+        st.m[0] = (uint32_t)mx[2]; st.m[1] = (uint32_t)mx[3]; st.m[2] = (uint32_t)mx[4];
+#pragma unroll
+        for (int r = 0; r < 6; ++r) s[r] = t[r];
+    }
+}
+
+// Block-wide publication of the slice flags and the level maxima (as FP64
+// bit patterns of |A^(r)|, r = 1..5).  Every thread of the block calls it.
+__device__ __forceinline__ void spec_publish(const SpecState &st, int v0, WsHeader *ws, int slot, unsigned long long *red)
+{
+    const uint32_t bm = __reduce_or_sync(0xFFFFFFFFu, st.badmask);
+    if (bm && lane_id() == 0) atomicOr(&ws->slice_bad[slot], bm);
+    const int F = (v0 == kZeroLevel) ? 0 : v0 - 50;
+    const unsigned long long mm[5] = {st.m1, st.m2, st.m[0], st.m[1], st.m[2]};
+#pragma unroll
+    for (int r = 0; r < 5; ++r) {
+        const double v = (double)mm[r] * pow2_d(F);                  // exact: below 2^53 units
+        block_max_to((unsigned long long)__double_as_longlong(v), &ws->maxbits[slot][r + 1], red);
+    }
+}
+
+__device__ __forceinline__ int spec_v0(const WsHeader *ws, int slot)
+{
+    const unsigned long long m0 = ws->maxbits[slot][0];
+    return m0 ? ceil_log2_bits(m0) : kZeroLevel;
+}
+
+// Row-major planes: thread = 4 consecutive entries of a row (two 16-byte
+// loads, one 8-byte store per plane), rows advancing by the grid's y size.
+__global__ void __launch_bounds__(kThreads)
+f64_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                     uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
+{
+    __shared__ unsigned long long red[kThreads / 32];
+    const int v0 = spec_v0(ws, slot);
+    const bool fast = v0 >= -78;
+    const bool vin = ((ldx & 1) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
+    const bool vout = ((ldcomp & 3) == 0) && ((plane & 3) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 7u) == 0);
+    const int64_t j0 = ((int64_t)blockIdx.x * kThreads + threadIdx.x) * 4;
+    SpecState st;
+    if (j0 < cols) {
+        const bool full = j0 + 4 <= cols;
+        for (int64_t i = blockIdx.y; i < rows; i += gridDim.y) {
+            const double *src = X + i * ldx + j0;
+            double x[4];
+            if (vin && full) {
+                const double2 a = reinterpret_cast<const double2 *>(src)[0], c = reinterpret_cast<const double2 *>(src)[1];
+                x[0] = a.x; x[1] = a.y; x[2] = c.x; x[3] = c.y;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) x[e] = (j0 + e < cols) ? src[e] : 0.0;
+            }
+            uint32_t w[6][2] = {};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                uint32_t sl[6];
+                spec_element(x[e], v0, fast, sl, st);
+#pragma unroll
+                for (int r = 0; r < 6; ++r) w[r][e >> 1] |= sl[r] << (16 * (e & 1));
+            }
+            uint16_t *dst = comps + i * ldcomp + j0;
+#pragma unroll
+            for (int r = 0; r < 6; ++r) {
+                if (vout && full) {
+                    *reinterpret_cast<uint2 *>(dst + r * plane) = make_uint2(w[r][0], w[r][1]);
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        if (j0 + e < cols) dst[r * plane + e] = (uint16_t)(w[r][e >> 1] >> (16 * (e & 1)));
+                }
+            }
+        }
+    }
+    spec_publish(st, v0, ws, slot, red);
+}
+
+// Transposed (K-major) planes: a 64 x 64 tile, warp q on columns 8q .. 8q+7,
+// lane p on rows 2p and 2p+1; each plane word packs the two entries adjacent
+// in the transposed row, staged one bank per lane and written as 16-byte
+// chunks of whole transposed rows.  Shared memory: [6][64][32] words.
+__global__ void __launch_bounds__(kThreads)
+f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                          uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
+{
+    extern __shared__ __align__(16) uint32_t smw[];                  // [6][kTile][kTile / 2]
+    __shared__ unsigned long long red[kThreads / 32];
+    const int v0 = spec_v0(ws, slot);
+    const bool fast = v0 >= -78;
+    const bool vin = ((ldx & 1) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
+    const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
+    const int q = threadIdx.x >> 5, p = lane_id();
+    const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
+    SpecState st;
+    for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
+        const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
+        const int64_t gj = c0 + 8 * q;
+        double x[2][8];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int64_t gi = r0 + 2 * p + h;
+            const double *src = X + gi * ldx + gj;
+            if (gi < rows && vin && gj + 8 <= cols) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const double2 a = reinterpret_cast<const double2 *>(src)[k];
+                    x[h][2 * k] = a.x; x[h][2 * k + 1] = a.y;
+                }
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) x[h][e] = (gi < rows && gj + e < cols) ? src[e] : 0.0;
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            uint32_t s0[6], s1[6];
+            spec_element(x[0][e], v0, fast, s0, st);
+            spec_element(x[1][e], v0, fast, s1, st);
+#pragma unroll
+            for (int r = 0; r < 6; ++r) smw[(r * kTile + 8 * q + e) * (kTile / 2) + p] = s0[r] | (s1[r] << 16);
+        }
+        __syncthreads();
+#pragma unroll 4
+        for (int it = 0; it < 6 * kTile * 8 / kThreads; ++it) {
+            const int c = threadIdx.x + it * kThreads;
+            const int r = c >> 9, orow = (c >> 3) & 63, ch = c & 7;
+            const int64_t go = c0 + orow, gk = r0 + 8 * ch;
+            if (go < cols && gk < rows) {
+                const uint4 v = *reinterpret_cast<const uint4 *>(&smw[(r * kTile + orow) * (kTile / 2) + 4 * ch]);
+                uint16_t *dst = comps + r * plane + go * ldcomp + gk;
+                if (vout && gk + 8 <= rows) {
+                    *reinterpret_cast<uint4 *>(dst) = v;
+                } else {
+                    const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        if (gk + e < rows) dst[e] = (uint16_t)(wv[e >> 1] >> (16 * (e & 1)));
+                }
+            }
+        }
+        __syncthreads();
+    }
+    spec_publish(st, v0, ws, slot, red);
 }
 
 // ------------------------------------------------------ FP32 split kernels
@@ -640,6 +883,8 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
     publish_f32_flags(amax, ws);
 }
 
+constexpr size_t kSpecTransposeSmem = 6 * kTile * (kTile / 2) * sizeof(uint32_t);
+
 size_t smem_bytes(int ns) { return (size_t)ns * kTile * kSRow * sizeof(uint16_t); }
 
 int grid_for(int64_t work_items, int max_blocks)
@@ -682,19 +927,25 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
         const size_t sm = smem_bytes(6);
         cudaError_t e = cudaSuccess;
         if (transpose) {
-            e = cudaFuncSetAttribute(split_tile_kernel<double, 1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+            e = cudaFuncSetAttribute(f64_spec_transpose_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)kSpecTransposeSmem);
             if (e == cudaSuccess) e = cudaFuncSetAttribute(split_tile_kernel<double, 2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
         } else {
-            e = cudaFuncSetAttribute(split_tile_kernel<double, 1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-            if (e == cudaSuccess) e = cudaFuncSetAttribute(split_tile_kernel<double, 2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+            e = cudaFuncSetAttribute(split_tile_kernel<double, 2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
         }
         if (e != cudaSuccess) return e;
         f64_max_kernel<0><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
-        if (transpose)
-            split_tile_kernel<double, 1, true><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot);
-        else
-            split_tile_kernel<double, 1, false><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot);
+        if (transpose) {
+            f64_spec_transpose_kernel<<<gt, kThreads, kSpecTransposeSmem, st>>>(X, rows, cols, ldx, comps, ldcomp,
+                                                                            plane, ws, slot);
+        } else {
+            const int64_t bx = (cols + 4 * kThreads - 1) / (4 * kThreads);
+            const int64_t by = rows < 4096 ? rows : 4096;
+            f64_spec_rows_kernel<<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, comps,
+                                                                                       ldcomp, plane, ws, slot);
+        }
         f64_verify_kernel<<<1, 1, 0, st>>>(ws, slot);
+        f64_max_kernel<1><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
         f64_max_kernel<2><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
         f64_max_kernel<3><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
         f64_max_kernel<4><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);

@@ -142,3 +142,13 @@ def test_split_fullsize_fp64_scaled_b_transposed_bitexact(dev):
     want, wv, _ = oracle.split_f64(B)
     assert np.array_equal(v.cpu().numpy(), wv)
     assert np.array_equal(planes_np(planes), want.transpose(0, 2, 1))
+
+
+@pytest.mark.parametrize("scale_exp", [-70, -77, -78, -79, -100, 100, 126])
+@pytest.mark.parametrize("transpose", [False, True])
+def test_split_f64_scales_bitexact(dev, scale_exp, transpose):
+    """Uniform data scaled by 2^e: the split takes its 32-bit fast form for
+    v0 >= -78 and its checked general form below (where low slices leave the
+    BF16 normal range and are flagged); both must match the oracle."""
+    X = synth.uniform_f64(7, 0, (130, 75)) * 2.0**scale_exp
+    _check_f64(X, dev, transpose, pad=3)
