@@ -512,12 +512,23 @@ __global__ void f64_finalize_kernel(WsHeader *ws, int slot, int32_t *v_out)
 // remainder with the opposite sign.  No range check is needed when
 // v0 >= -78: every nonzero slice then lies between 2^(v0 - 48) >= 2^-126 and
 // 2^v0 <= 2^127.  Results are bit-identical to spec_levels.
-__device__ __forceinline__ uint32_t bf16_of_level(uint32_t n, uint32_t sg, int eg)
+// BF16 bits of (-1)^sg * n * 2^e for an integer 0 <= n <= 256 whose value is
+// a normal BF16 (guaranteed on the fast path): n is converted exactly to FP32
+// (2^23 + n by bits, minus 2^23), whose upper half is the BF16 of n; adding e
+// to the exponent field and the sign gives the slice.
+__device__ __forceinline__ uint32_t bf16_of_level(uint32_t n, uint32_t sg, int e)
 {
-    // n * 2^(eg - 127 - ...) as BF16: leading bit p of n (n <= 256), 7 bits below it
-    const int p = 31 - __clz(n | 1u);
-    const uint32_t out = (sg << 15) + ((uint32_t)(eg + p) << 7) + (((n << 7) >> p) & 0x7Fu);
+    const float fn = __fsub_rn(__uint_as_float(0x4B000000u | n), 8388608.0f);
+    const uint32_t out = (__float_as_uint(fn) >> 16) + ((uint32_t)e << 7) + (sg << 15);
     return n ? out : 0u;
+}
+
+// BF16 bits of an FP32 value z (a multiple of the level's grid with at most
+// nine significant bits, or zero) scaled by 2^F.
+__device__ __forceinline__ uint32_t bf16_of_scaled(float z, int F)
+{
+    const uint32_t zb = __float_as_uint(z);
+    return (zb & 0x7FFFFFFFu) ? (zb >> 16) + ((uint32_t)F << 7) : 0u;
 }
 
 __device__ __forceinline__ void spec_levels_fast(double x, int F, uint32_t (&s)[6], uint32_t &badmask,
@@ -546,10 +557,12 @@ __device__ __forceinline__ void spec_levels_fast(double x, int F, uint32_t (&s)[
         }
         const int gh = 11 - 8 * r - (int)sg;
         const uint32_t t = H >> gh, rh = H & ((1u << gh) - 1u), hh = 1u << (gh - 1);
-        const bool up = (rh > hh) || (rh == hh && (L != 0u || (t & 1u)));
-        s[r] = bf16_of_level(t + (up ? 1u : 0u), sg, F + 32 + gh + 127);
-        if (up) { H = (1u << gh) - rh - (L != 0u ? 1u : 0u); L = 0u - L; sg ^= 1u; }
-        else H = rh;
+        const uint32_t lnz = (uint32_t)(L != 0u);
+        const uint32_t up = (uint32_t)(rh > hh) | ((uint32_t)(rh == hh) & (lnz | (t & 1u)));
+        s[r] = bf16_of_level(t + up, sg, F + 32 + gh);
+        H = up ? (1u << gh) - rh - lnz : rh;
+        L = up ? 0u - L : L;
+        sg ^= up;
     }
     // level 2: |X| < 2^35, grid 2^27 / 2^26
     uint32_t Y;
@@ -558,19 +571,34 @@ __device__ __forceinline__ void spec_levels_fast(double x, int F, uint32_t (&s)[
         m2 = cur > m2 ? cur : m2;
         const int g = 27 - (int)sg;
         const uint32_t t = (H << (32 - g)) | (L >> g), rem = L & ((1u << g) - 1u), half = 1u << (g - 1);
-        const bool up = rem > half || (rem == half && (t & 1u));
-        s[2] = bf16_of_level(t + (up ? 1u : 0u), sg, F + g + 127);
-        if (up) { Y = (1u << g) - rem; sg ^= 1u; } else Y = rem;
+        const uint32_t up = (uint32_t)(rem > half) | ((uint32_t)(rem == half) & t & 1u);
+        s[2] = bf16_of_level(t + up, sg, F + g);
+        Y = up ? (1u << g) - rem : rem;
+        sg ^= up;
     }
-    // levels 3-5: |X| <= 2^26
-#pragma unroll
-    for (int r = 3; r < 6; ++r) {
-        m[r - 3] = Y > m[r - 3] ? Y : m[r - 3];
-        const int g = 43 - 8 * r - (int)sg;
+    // level 3: |X| <= 2^26, grid 2^19 / 2^18
+    {
+        m[0] = Y > m[0] ? Y : m[0];
+        const int g = 19 - (int)sg;
         const uint32_t t = Y >> g, rem = Y & ((1u << g) - 1u), half = 1u << (g - 1);
-        const bool up = rem > half || (rem == half && (t & 1u));
-        s[r] = bf16_of_level(t + (up ? 1u : 0u), sg, F + g + 127);
-        if (up) { Y = (1u << g) - rem; sg ^= 1u; } else Y = rem;
+        const uint32_t up = (uint32_t)(rem > half) | ((uint32_t)(rem == half) & t & 1u);
+        s[3] = bf16_of_level(t + up, sg, F + g);
+        Y = up ? (1u << g) - rem : rem;
+        sg ^= up;
+    }
+    // levels 4, 5: |X| <= 2^18, exact in FP32; the add-subtract projection
+    // with C = 1.5 * 2^(23 + g) rounds to the grid 2^g to nearest, ties to even
+    float y = __fsub_rn(__uint_as_float(0x4B000000u | Y), 8388608.0f);
+    y = sg ? -y : y;
+#pragma unroll
+    for (int r = 4; r < 6; ++r) {
+        const float ay = fabsf(y);
+        m[r - 3] = max(m[r - 3], (uint32_t)ay);                   // exact: an integer below 2^24
+        const float C = (y < 0.0f) ? (r == 4 ? 12884901888.0f : 50331648.0f)      // 1.5 * 2^33, 1.5 * 2^25
+                                   : (r == 4 ? 25769803776.0f : 100663296.0f);    // 1.5 * 2^34, 1.5 * 2^26
+        const float z = __fsub_rn(__fadd_rn(y, C), C);
+        s[r] = bf16_of_scaled(z, F);
+        y = __fsub_rn(y, z);
     }
 }
 
@@ -605,12 +633,25 @@ __device__ __forceinline__ void spec_publish(const SpecState &st, int v0, WsHead
 {
     const uint32_t bm = __reduce_or_sync(0xFFFFFFFFu, st.badmask);
     if (bm && lane_id() == 0) atomicOr(&ws->slice_bad[slot], bm);
-    const int F = (v0 == kZeroLevel) ? 0 : v0 - 50;
-    const unsigned long long mm[5] = {st.m1, st.m2, st.m[0], st.m[1], st.m[2]};
+    // maxima in units (integers, so the reduction needs no conversion); one
+    // thread converts the block's five maxima to FP64 bit patterns
+    unsigned long long mm[5] = {st.m1, st.m2, st.m[0], st.m[1], st.m[2]};
+    const int w = threadIdx.x >> 5;
 #pragma unroll
     for (int r = 0; r < 5; ++r) {
-        const double v = (double)mm[r] * pow2_d(F);                  // exact: below 2^53 units
-        block_max_to((unsigned long long)__double_as_longlong(v), &ws->maxbits[slot][r + 1], red);
+        mm[r] = warp_max(mm[r]);
+        if (lane_id() == 0) red[r * (kThreads / 32) + w] = mm[r];
+    }
+    __syncthreads();
+    if (threadIdx.x < 5) {
+        const int r = threadIdx.x;
+        unsigned long long m = 0;
+        for (int i = 0; i < kThreads / 32; ++i) m = red[r * (kThreads / 32) + i] > m ? red[r * (kThreads / 32) + i] : m;
+        if (m) {
+            const int F = (v0 == kZeroLevel) ? 0 : v0 - 50;
+            const double v = (double)m * pow2_d(F);                   // exact: below 2^53 units
+            atomicMax(&ws->maxbits[slot][r + 1], (unsigned long long)__double_as_longlong(v));
+        }
     }
 }
 
@@ -626,7 +667,7 @@ __global__ void __launch_bounds__(kThreads)
 f64_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
                      uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
 {
-    __shared__ unsigned long long red[kThreads / 32];
+    __shared__ unsigned long long red[5 * (kThreads / 32)];
     const int v0 = spec_v0(ws, slot);
     const bool fast = v0 >= -78;
     const bool vin = ((ldx & 1) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
@@ -678,7 +719,7 @@ f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t co
                           uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
 {
     extern __shared__ __align__(16) uint32_t smw[];                  // [6][kTile][kTile / 2]
-    __shared__ unsigned long long red[kThreads / 32];
+    __shared__ unsigned long long red[5 * (kThreads / 32)];
     const int v0 = spec_v0(ws, slot);
     const bool fast = v0 >= -78;
     const bool vin = ((ldx & 1) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
@@ -939,8 +980,10 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
             f64_spec_transpose_kernel<<<gt, kThreads, kSpecTransposeSmem, st>>>(X, rows, cols, ldx, comps, ldcomp,
                                                                             plane, ws, slot);
         } else {
+            // about eight blocks per SM, each over several rows
             const int64_t bx = (cols + 4 * kThreads - 1) / (4 * kThreads);
-            const int64_t by = rows < 4096 ? rows : 4096;
+            const int64_t want = (152 * 8 + bx - 1) / bx;
+            const int64_t by = rows < want ? rows : (want < 65535 ? want : 65535);
             f64_spec_rows_kernel<<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, comps,
                                                                                        ldcomp, plane, ws, slot);
         }
