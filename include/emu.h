@@ -80,7 +80,7 @@ size_t emu_split_workspace_bytes(int mode);
 
 /* FP32 three-slice split, Eq. (fp32split) / Algorithm 1 (Split_FP32):
  *   A_r = fl_BF16(A^(r)), A^(r+1) = fl32(A^(r) - A_r), r = 0, 1, 2,
- * fl_BF16 = round to nearest, ties to even (Section 4.1).
+ * fl_BF16 = round to nearest, ties to even (Section 4.2).
  * X: rows x cols FP32, leading dimension ldx (elements, >= cols).
  * transpose = 0: comps holds 3 planes [rows][ldcomp] (ldcomp >= cols);
  * transpose = 1: comps holds 3 planes [cols][ldcomp] (ldcomp >= rows).
@@ -109,7 +109,7 @@ size_t emu_gemm_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K);
 /* FP32-mode emulated GEMM, Algorithm 1: C (M x N, ldc) = A (M x K, lda) . B
  * (K x N, ldb), all FP32 row-major.  Splits A and B into the workspace, then
  * runs the tensor-core product-sum: the 6 products of Eq. (fp32six) are
- * accumulated in one FP32 accumulator over all of K (Section 5.3, FP32
+ * accumulated in one FP32 accumulator over all of K (Section 6.3, FP32
  * reconstruction), so C matches the oracle within FP32 reordering error. */
 emu_status emu_gemm_f32(int64_t M, int64_t N, int64_t K, const float *A, int64_t lda,
                         const float *B, int64_t ldb, float *C, int64_t ldc, void *ws,
@@ -118,7 +118,7 @@ emu_status emu_gemm_f32(int64_t M, int64_t N, int64_t K, const float *A, int64_t
 /* FP64-mode emulated GEMM, Algorithm 2: C = A . B for FP64 inputs, nprod in
  * {6, 10, 15, 21}.  Products are taken in Algorithm 2's diagonal order; for
  * each, the FP32 component product fl32(A_i B_j) is formed on the tensor
- * cores per K-chunk of 256 (every chunk partial is exact, Section 4.5), the
+ * cores per K-chunk of 256 (every chunk partial is exact, Section 5.2), the
  * partials are summed exactly, and the total is added once into the FP64
  * result: C <- fl64(C + fl32(A_i B_j)).  C equals the oracle's product-outer
  * order bit for bit.  C also serves as the FP64 accumulator while the kernel
@@ -162,7 +162,7 @@ emu_status emu_gemm_f64_host(int64_t M, int64_t N, int64_t K, const double *A, i
 
 /* Product-sum alone, from planes already split (A: [3][M][ldcomp],
  * B: [3][N][ldcomp], i.e. split with transpose = 1).  Eq. (fp32six),
- * Section 5.3.  ws: at least emu_split_workspace_bytes(32) (flag word). */
+ * Section 6.3.  ws: at least emu_split_workspace_bytes(32) (flag word). */
 emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acomps,
                            const uint16_t *Bcomps, int64_t ldcomp, float *C, int64_t ldc,
                            void *ws, size_t ws_bytes, emu_stream_t stream);

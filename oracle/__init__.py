@@ -74,7 +74,7 @@ def _load():
 
 
 def fl_bf16(x: float) -> int:
-    """fl_BF16 of one value (Section 4.1), as a BF16 bit pattern."""
+    """fl_BF16 of one value (Section 4.2), as a BF16 bit pattern."""
     return int(_load().oracle_fl_bf16(float(x)))
 
 
@@ -179,7 +179,7 @@ def ref_dd(A: np.ndarray, B: np.ndarray, rows=None):
 
 
 def errors(C_hat: np.ndarray, hi: np.ndarray, lo: np.ndarray, absAB: np.ndarray | None = None):
-    """Accuracy metrics of Section 6.3 against a double-double reference.
+    """Accuracy metrics of Section 7.3 against a double-double reference.
 
     e_F (Eq. (froerror)), e_max = max |C_hat - C_ref|, and, when |A||B| is
     given, e_scaled (Eq. (scalederror)) over entries with a nonzero

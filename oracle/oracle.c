@@ -20,18 +20,18 @@
  *
  * Readings of points the paper leaves open (each listed in the design doc):
  *   - fl_BF16 rounds to nearest, ties to even, with BF16 subnormals and
- *     overflow to infinity (Section 4.1 says "round-to-nearest").
+ *     overflow to infinity (Section 4.2 says "round-to-nearest").
  *   - v^(r) of Eq. (fp64split) is one scalar per operand and level: the max is
  *     taken over the whole matrix, as the equation is written.
- *   - K-chunk = B_K = 256 (Section 5.1); the last chunk may be shorter.
+ *   - K-chunk = B_K = 256 (Section 6.1); the last chunk may be shorter.
  *   - FP32 mode: inside one chunk the six products are interleaved per 32-wide
  *     K step in the operand-reuse order of Eq. (fp32reuseorder), one FP32
  *     accumulator per chunk, chunk results added into an FP32 output
- *     accumulator (Section 5.3, reconstruction of the FP32 path).
+ *     accumulator (Section 6.3, reconstruction of the FP32 path).
  *   - FP64 mode, two summation orders of the same exact FP32 chunk partials:
  *     ORDER_CHUNK_OUTER: chunk outer, products inner in diagonal order (l
  *       ascending, i ascending within a diagonal), each partial widened and
- *       added in FP64 (the per-panel reconstruction of Section 5.3);
+ *       added in FP64 (the per-panel reconstruction of Section 6.3);
  *     ORDER_PRODUCT_OUTER: products in diagonal order outer, as Algorithm 2
  *       is written (C <- fl64(C + fl32(A_i B_j))): the FP32 component product
  *       is formed per K-chunk and its chunk partials are summed exactly (they
@@ -50,10 +50,10 @@
 #define ORACLE_ZERO_LEVEL INT32_MIN /* v^(r) of an all-zero residual */
 #define ORACLE_ORDER_CHUNK_OUTER 0
 #define ORACLE_ORDER_PRODUCT_OUTER 1
-#define ORACLE_KCHUNK 256           /* B_K of Section 5.1 */
+#define ORACLE_KCHUNK 256           /* B_K of Section 6.1 */
 
 /* ------------------------------------------------------------------------ */
-/* fl_BF16 (Section 4.1): keep an 8-bit significand (implicit bit included), */
+/* fl_BF16 (Section 4.2): keep an 8-bit significand (implicit bit included), */
 /* round to nearest, ties to even.  Written from the definition: find the    */
 /* binade, scale to an integer significand, round, scale back.               */
 /* ------------------------------------------------------------------------ */
@@ -240,10 +240,10 @@ static float *expand_bt(const uint16_t *Bp, int s, int64_t K, int64_t N)
 
 /* ------------------------------------------------------------------------ */
 /* FP32-mode product-sum, Eq. (fp32six) with the blocked FP32 reconstruction */
-/* of Section 5.3: per K-chunk an FP32 accumulator takes the six products    */
+/* of Section 6.3: per K-chunk an FP32 accumulator takes the six products    */
 /* (interleaved per 32-wide step, Eq. (fp32reuseorder)); each chunk result   */
 /* is added into the FP32 output accumulator.  Every product of two BF16    */
-/* values is exact in FP32 (Section 4.5); only the additions round.         */
+/* values is exact in FP32 (Section 5.2); only the additions round.         */
 /* ------------------------------------------------------------------------ */
 void oracle_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                         int64_t r0, int64_t nr, float *C)
@@ -281,7 +281,7 @@ void oracle_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, con
 /* chunk partial P = fl32(sum_k A_i B_j) is formed in FP32 (k ascending).    */
 /* Slices lie on the grid of Eq. (fp64split): integers times 2^(v-8) of     */
 /* magnitude <= 256, so a BF16 product is <= 2^16 units and a 256-long chunk */
-/* <= 2^24 units: P is exact (Section 4.5 extended to the chunk).            */
+/* <= 2^24 units: P is exact (Section 5.2 extended to the chunk).            */
 /*   order 0 (chunk outer): for chunk, for pair: C = fl64(C + (double)P).    */
 /*   order 1 (product outer): for pair: S = sum over chunks of (double)P --  */
 /*     exact in FP64, a sum of integers in one unit below 2^53 units -- then */
@@ -334,7 +334,7 @@ void oracle_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, con
 }
 
 /* ------------------------------------------------------------------------ */
-/* Double-double reference product (for the accuracy metrics of Section 6.3, */
+/* Double-double reference product (for the accuracy metrics of Section 7.3, */
 /* Eqs. (froerror), (scalederror)): sum_k A[m,k] B[k,n] with an error-free   */
 /* product (TwoProd via fma) and error-free additions (TwoSum), Dekker/Knuth */
 /* style.  Returns hi + lo per element, rows [r0, r0+nr).                    */

@@ -28,7 +28,7 @@ struct WsHeader {
 constexpr size_t kWsHeaderBytes = 512;
 static_assert(sizeof(WsHeader) <= kWsHeaderBytes, "workspace header too large");
 
-constexpr int kKChunk = 256;              // B_K of the paper (Section 5.1)
+constexpr int kKChunk = 256;              // B_K of the paper (Section 6.1)
 constexpr int32_t kZeroLevel = INT32_MIN;
 
 // Watchdog limit of a bounded wait inside the GEMM kernels (nanoseconds).

@@ -1,6 +1,6 @@
 // FP32-mode tensor-core product-sum (sm_103a: TMA -> shared memory ->
 // tcgen05 BF16 MMAs with the FP32 accumulator in tensor memory), Eq. (fp32six)
-// and the FP32 reconstruction of Section 5.3.
+// and the FP32 reconstruction of Section 6.3.
 //
 // One CTA owns a 128 x BN tile of C.  Each pipeline stage holds the three A
 // slices and the three B slices of one K-block; the six retained products of

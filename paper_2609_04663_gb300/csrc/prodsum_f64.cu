@@ -1,7 +1,7 @@
 // FP64-mode tensor-core product-sum, Eq. (fp64reconstruction) / Algorithm 2.
 //
 // Products are taken in Algorithm 2's diagonal order (outer loop); for each
-// product the K dimension is walked in chunks of 256 (B_K of Section 5.1).
+// product the K dimension is walked in chunks of 256 (B_K of Section 6.1).
 // Every chunk partial fl32(A_i B_j) is formed on the tensor cores in its own
 // TMEM buffer (two rotating 128-column buffers).  The partials are exact:
 // slice entries are integers times 2^(v-8) of magnitude <= 256, so a chunk

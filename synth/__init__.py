@@ -5,7 +5,7 @@ SplitMix64 counter generator in ``synth.c`` and the input recipes used by the
 tests and by ``bench.py``.  The CPU oracle and the CUDA path are both fed the
 very same host arrays produced here.
 
-Input classes (Section 6.3 of the paper, "Input Matrices and Accuracy
+Input classes (Section 7.3 of the paper, "Input Matrices and Accuracy
 Metrics"): uniform random entries in [-1, 1] (the class the paper reports),
 and the "scaled" class ``(u - 0.5) * exp(phi * g)`` clamped into the BF16
 exponent range.  Matrix A is drawn first (row-major), then B continues the

@@ -251,7 +251,7 @@ def test_product_sets_match_paper():
 
 # ------------------------------------------------------- product-sum pins
 def test_fp64_chunk_partials_are_exact():
-    """Section 4.5: BF16 x BF16 products are exact in FP32; with slices on the
+    """Section 5.2: BF16 x BF16 products are exact in FP32; with slices on the
     grid of Eq. (fp64split) every 256-long chunk partial is exact too."""
     for X, Y in [synth.gemm_inputs("f64", 24, 20, 600, 1),
                  synth.gemm_inputs("f64_scaled", 16, 16, 520, 5, phi=4.0),
@@ -410,7 +410,7 @@ def test_accuracy_magnitudes_uniform_n256():
 
 
 def test_fp32_kchunk_is_256():
-    """B_K = 256 (Section 5.1) fixes where FP32 rounding happens: each chunk
+    """B_K = 256 (Section 6.1) fixes where FP32 rounding happens: each chunk
     is accumulated on its own, then added into the output accumulator.
     Row 0: 256 ones then 256 x 2^-22.  Per-chunk: 256 + 256*2^-22 = 256 + 2^-14
     (exact); one long accumulator would round every 2^-22 away (ulp(256) = 2^-15).
