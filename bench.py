@@ -136,12 +136,23 @@ def peaks():
         return {"bf16_sustained": 1700.0, "bf16_burst": 1900.0, "hbm": 6800.0, "source": "fallback"}
 
 
+def code_digest(path: str) -> str:
+    """sha256 prefix of a CUDA source with comments and whitespace removed, so
+    that a comment edit does not invalidate counters taken on the same code."""
+    import re
+    text = open(path).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", "", text)
+    text = re.sub(r"\s+", "", text)
+    return hashlib.sha256(text.encode()).hexdigest()[:16]
+
+
 def kernel_traffic(kernel: str, workload_name: str):
     """DRAM bytes per launch from the committed ncu summary, if it was taken on
-    the current source of the kernel (else None)."""
+    the current code of the kernel (else None)."""
     src = os.path.join(ROOT, "paper_2609_04663_gb300", "csrc", kernel + ".cu")
     try:
-        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        digest = code_digest(src)
         with open(os.path.join(ROOT, "profiles", "traffic.txt")) as f:
             for line in f:
                 t = line.split()
