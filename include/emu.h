@@ -127,6 +127,33 @@ emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_
                         const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,
                         void *ws, size_t ws_bytes, emu_stream_t stream);
 
+/* General GEMM (the "more complete BLAS semantics" of Section 9's future
+ * work): C (M x N, ldc) <- alpha * op(A) op(B) + beta * C, all row-major.
+ * op(X) is X as stored (EMU_OP_N) or its transpose (EMU_OP_T): with opA = N,
+ * A is M x K (lda >= K), with opA = T it is stored K x M (lda >= M); with
+ * opB = N, B is K x N (ldb >= N), with opB = T it is stored N x K (ldb >= K).
+ * The product P = op(A) op(B) is the emulated one of emu_gemm_f32 (Algorithm
+ * 1) or emu_gemm_f64 (Algorithm 2, nprod products), from the same kernels:
+ * the split writes op(A) and op(B) into the same K-major planes whichever
+ * way they are stored.  Then, each operation rounded once in FP32 / FP64
+ * (no fused multiply-add): alpha = 1 and beta = 0 gives C = P (written
+ * directly, bit-identical to emu_gemm_*); beta = 0 gives C = fl(alpha * P)
+ * without reading C; otherwise C = fl(fl(alpha * P) + fl(beta * C)).  K = 0
+ * gives P = 0.  ws: device workspace of at least
+ * emu_gemm_ex_workspace_bytes (the GEMM workspace plus an M x N product
+ * buffer), 16-byte aligned.  Errors as emu_gemm_*; EMU_ERR_INVALID_ARG also
+ * for an op other than EMU_OP_N / EMU_OP_T. */
+#define EMU_OP_N 0
+#define EMU_OP_T 1
+size_t emu_gemm_ex_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K);
+emu_status emu_gemm_ex_f32(int opA, int opB, int64_t M, int64_t N, int64_t K, float alpha,
+                           const float *A, int64_t lda, const float *B, int64_t ldb, float beta,
+                           float *C, int64_t ldc, void *ws, size_t ws_bytes, emu_stream_t stream);
+emu_status emu_gemm_ex_f64(int opA, int opB, int64_t M, int64_t N, int64_t K, double alpha,
+                           const double *A, int64_t lda, const double *B, int64_t ldb, double beta,
+                           double *C, int64_t ldc, int nprod, void *ws, size_t ws_bytes,
+                           emu_stream_t stream);
+
 /* Workspace bytes for emu_gemm_f32_host (mode 32) / emu_gemm_f64_host (mode
  * 64): the header, the planes of A and B, staging space for the copied
  * inputs (FP32: two row panels of A and two K-panels of B; FP64: A and B

@@ -164,6 +164,35 @@ def gemm_f64(A: np.ndarray, B: np.ndarray, nprod: int, rows=None, order: str = "
     return prodsum_f64(Ap, Bp, nprod, rows=rows, order=order), fa | fb
 
 
+def gemm_ex(opA: int, opB: int, alpha, A: np.ndarray, B: np.ndarray, beta, C: np.ndarray | None = None,
+            nprod: int | None = None):
+    """General GEMM C <- alpha op(A) op(B) + beta C (the BLAS semantics that
+    Section 9 leaves as future work), row-major, op = 1 transposes the stored
+    matrix.  P = op(A) op(B) is Algorithm 1 (FP32 inputs) or Algorithm 2 with
+    nprod products (FP64 inputs); the epilogue rounds each operation once in
+    the input format: alpha = 1, beta = 0 gives P; beta = 0 gives alpha * P
+    (C not read); otherwise (alpha * P) + (beta * C).  Returns (C, flags)."""
+    f64 = A.dtype == np.float64
+    dt = np.float64 if f64 else np.float32
+    Ae = np.ascontiguousarray(A.T if opA else A)
+    Be = np.ascontiguousarray(B.T if opB else B)
+    M, K = Ae.shape
+    N = Be.shape[1]
+    if K == 0:
+        P, flags = np.zeros((M, N), dtype=dt), 0
+    elif f64:
+        P, flags = gemm_f64(Ae, Be, nprod)
+    else:
+        P, flags = gemm_f32(Ae, Be)
+    a, b = dt(alpha), dt(beta)
+    if a == 1 and b == 0:
+        return P, flags
+    aP = a * P                                   # one rounding in the input format
+    if b == 0:
+        return aP, flags
+    return aP + b * np.asarray(C, dtype=dt), flags
+
+
 def ref_dd(A: np.ndarray, B: np.ndarray, rows=None):
     """Double-double reference A.B (rows [r0, r1)): returns (hi, lo)."""
     A = np.ascontiguousarray(A, dtype=np.float64)

@@ -23,6 +23,7 @@ EMU_OK = 0
 STATUS = {0: "ok", 1: "invalid argument", 2: "misaligned", 3: "workspace too small", 4: "CUDA error",
           5: "unsupported size"}
 FLAG_NONFINITE, FLAG_RANGE, FLAG_SLICE, FLAG_TIMEOUT = 0x1, 0x2, 0x4, 0x8
+OP_N, OP_T = 0, 1
 ZERO_LEVEL = -(2 ** 31)
 
 _SIGS = {
@@ -37,6 +38,9 @@ _SIGS = {
     "emu_prodsum_f64": ("i", ["l", "l", "l", "p", "p", "l", "p", "p", "i", "p", "l", "p", "size", "p"]),
     "emu_gemm_f64_noalloc": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "p"]),
     "emu_gemm_host_workspace_bytes": ("size", ["i", "l", "l", "l"]),
+    "emu_gemm_ex_workspace_bytes": ("size", ["i", "l", "l", "l"]),
+    "emu_gemm_ex_f32": ("i", ["i", "i", "l", "l", "l", "f", "p", "l", "p", "l", "f", "p", "l", "p", "size", "p"]),
+    "emu_gemm_ex_f64": ("i", ["i", "i", "l", "l", "l", "d", "p", "l", "p", "l", "d", "p", "l", "i", "p", "size", "p"]),
     "emu_gemm_f32_host": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "p", "size", "p"]),
     "emu_gemm_f64_host": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "size", "p"]),
     "emu_read_flags": ("i", ["p", "p", "p"]),
@@ -44,7 +48,7 @@ _SIGS = {
     "emu_status_string": ("str", ["i"]),
 }
 _CT = {"i": ctypes.c_int, "l": ctypes.c_int64, "p": ctypes.c_void_p, "size": ctypes.c_size_t,
-       "u32": ctypes.c_uint32, "str": ctypes.c_char_p}
+       "u32": ctypes.c_uint32, "str": ctypes.c_char_p, "f": ctypes.c_float, "d": ctypes.c_double}
 
 
 class EmuError(RuntimeError):
@@ -91,6 +95,9 @@ emu_prodsum_f32 = _mk("emu_prodsum_f32")
 emu_prodsum_f64 = _mk("emu_prodsum_f64")
 emu_gemm_f64_noalloc = _mk("emu_gemm_f64_noalloc")
 emu_gemm_host_workspace_bytes = _mk("emu_gemm_host_workspace_bytes")
+emu_gemm_ex_workspace_bytes = _mk("emu_gemm_ex_workspace_bytes")
+emu_gemm_ex_f32 = _mk("emu_gemm_ex_f32")
+emu_gemm_ex_f64 = _mk("emu_gemm_ex_f64")
 emu_gemm_f32_host = _mk("emu_gemm_f32_host")
 emu_gemm_f64_host = _mk("emu_gemm_f64_host")
 emu_read_flags = _mk("emu_read_flags")
@@ -180,6 +187,28 @@ def gemm_f64(A, B, nprod: int, C=None, ws=None, stream=None):
     ws = ws if ws is not None else workspace(emu_gemm_workspace_bytes(64, M, N, K), A.device)
     _check(emu_gemm_f64(M, N, K, A.data_ptr(), A.stride(0), B.data_ptr(), B.stride(0), C.data_ptr(), C.stride(0),
                         int(nprod), ws.data_ptr(), ws.numel(), _stream(stream)), "emu_gemm_f64")
+    return C, ws
+
+
+def gemm_ex(A, B, opA: int = OP_N, opB: int = OP_N, alpha: float = 1.0, beta: float = 0.0, C=None,
+            nprod: int | None = None, ws=None, stream=None):
+    """emu_gemm_ex_*: C <- alpha op(A) op(B) + beta C for device tensors A, B
+    as stored (op = OP_T reads the stored matrix transposed).  FP32 tensors
+    run Algorithm 1, FP64 tensors Algorithm 2 with nprod products."""
+    torch = _torch()
+    M, K = (A.shape[1], A.shape[0]) if opA == OP_T else (A.shape[0], A.shape[1])
+    N = B.shape[0] if opB == OP_T else B.shape[1]
+    f64 = A.dtype == torch.float64
+    C = C if C is not None else torch.zeros((M, N), dtype=A.dtype, device=A.device)
+    ws = ws if ws is not None else workspace(emu_gemm_ex_workspace_bytes(64 if f64 else 32, M, N, K), A.device)
+    if f64:
+        r = emu_gemm_ex_f64(opA, opB, M, N, K, float(alpha), A.data_ptr(), A.stride(0), B.data_ptr(), B.stride(0),
+                            float(beta), C.data_ptr(), C.stride(0), int(nprod), ws.data_ptr(), ws.numel(),
+                            _stream(stream))
+    else:
+        r = emu_gemm_ex_f32(opA, opB, M, N, K, float(alpha), A.data_ptr(), A.stride(0), B.data_ptr(), B.stride(0),
+                            float(beta), C.data_ptr(), C.stride(0), ws.data_ptr(), ws.numel(), _stream(stream))
+    _check(r, "emu_gemm_ex_f64" if f64 else "emu_gemm_ex_f32")
     return C, ws
 
 

@@ -163,6 +163,92 @@ emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_
     return cuda_status(e);
 }
 
+size_t emu_gemm_ex_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K)
+{
+    if (M < 0 || N < 0 || K < 0 || (mode != 32 && mode != 64)) return 0;
+    return gemm_ws_bytes(mode == 64 ? 6 : 3, M, N, K) + (size_t)round_up(M * N * (mode == 64 ? 8 : 4), 256);
+}
+
+}  // extern "C"
+
+namespace {
+
+// Shared body of the general GEMMs: validation, the splits of op(A) and
+// op(B) into K-major planes (the split's transpose flag absorbs op), the
+// product-sum into C (alpha = 1, beta = 0) or into the workspace product
+// buffer followed by the epilogue.
+template <typename T>
+emu_status gemm_ex(int opA, int opB, int64_t M, int64_t N, int64_t K, T alpha, const T *A, int64_t lda, const T *B,
+                   int64_t ldb, T beta, T *C, int64_t ldc, int nprod, void *ws, size_t ws_bytes, cudaStream_t st)
+{
+    constexpr bool f64 = sizeof(T) == 8;
+    constexpr int S = f64 ? 6 : 3;
+    if ((opA != EMU_OP_N && opA != EMU_OP_T) || (opB != EMU_OP_N && opB != EMU_OP_T)) return EMU_ERR_INVALID_ARG;
+    if (M < 0 || N < 0 || K < 0 || !ws) return EMU_ERR_INVALID_ARG;
+    const int64_t a_cols = opA == EMU_OP_N ? K : M, b_cols = opB == EMU_OP_N ? N : K;
+    if (lda < (a_cols > 0 ? a_cols : 1) || ldb < (b_cols > 0 ? b_cols : 1) || ldc < (N > 0 ? N : 1))
+        return EMU_ERR_INVALID_ARG;
+    if (M >= kMaxDim || N >= kMaxDim || K >= kMaxDim) return EMU_ERR_UNSUPPORTED;
+    if (f64 && nprod != 6 && nprod != 10 && nprod != 15 && nprod != 21) return EMU_ERR_INVALID_ARG;
+    if (M > 0 && N > 0 && (!C || (K > 0 && (!A || !B)))) return EMU_ERR_INVALID_ARG;
+    if (ws_bytes < emu_gemm_ex_workspace_bytes(f64 ? 64 : 32, M, N, K)) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
+    if (e != cudaSuccess) return EMU_ERR_CUDA;
+    if (M == 0 || N == 0) return EMU_OK;
+    const int64_t ldk = gemm_ldk(K);
+    char *w = static_cast<char *>(ws);
+    uint16_t *Ap = reinterpret_cast<uint16_t *>(w + kWsHeaderBytes);
+    uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(S * M * ldk * 2, 256));
+    T *P = reinterpret_cast<T *>(reinterpret_cast<char *>(Bp) + round_up(S * N * ldk * 2, 256));
+    const bool direct = (alpha == T(1) && beta == T(0));
+    T *out = direct ? C : P;
+    const int64_t ldo = direct ? ldc : N;
+    if (K == 0) {
+        e = cudaMemset2DAsync(out, (size_t)ldo * sizeof(T), 0, (size_t)N * sizeof(T), (size_t)M, st);
+    } else {
+        // op(A) -> planes [S][M][ldk]; op(B) -> planes [S][N][ldk]
+        const bool ta = opA == EMU_OP_T, tb = opB == EMU_OP_N;
+        const int64_t ar = ta ? K : M, ac = ta ? M : K, br = tb ? K : N, bc = tb ? N : K;
+        if constexpr (f64) {
+            e = launch_split_f64(A, ar, ac, lda, ta, Ap, ldk, h->vout[0], h, 0, st);
+            if (e == cudaSuccess) e = launch_split_f64(B, br, bc, ldb, tb, Bp, ldk, h->vout[1], h, 1, st);
+            if (e == cudaSuccess)
+                e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, out, ldo, &h->flags, st);
+        } else {
+            e = launch_split_f32(A, ar, ac, lda, ta, Ap, ldk, h, st);
+            if (e == cudaSuccess) e = launch_split_f32(B, br, bc, ldb, tb, Bp, ldk, h, st);
+            if (e == cudaSuccess) e = launch_prodsum_f32(M, N, K, Ap, Bp, ldk, out, ldo, &h->flags, st);
+        }
+    }
+    if (e == cudaSuccess && !direct) {
+        if constexpr (f64) e = launch_axpby_f64(P, N, C, ldc, M, N, alpha, beta, st);
+        else e = launch_axpby_f32(P, N, C, ldc, M, N, alpha, beta, st);
+    }
+    return cuda_status(e);
+}
+
+}  // namespace
+
+extern "C" {
+
+emu_status emu_gemm_ex_f32(int opA, int opB, int64_t M, int64_t N, int64_t K, float alpha, const float *A, int64_t lda,
+                           const float *B, int64_t ldb, float beta, float *C, int64_t ldc, void *ws, size_t ws_bytes,
+                           emu_stream_t stream)
+{
+    return gemm_ex<float>(opA, opB, M, N, K, alpha, A, lda, B, ldb, beta, C, ldc, 0, ws, ws_bytes,
+                          reinterpret_cast<cudaStream_t>(stream));
+}
+
+emu_status emu_gemm_ex_f64(int opA, int opB, int64_t M, int64_t N, int64_t K, double alpha, const double *A,
+                           int64_t lda, const double *B, int64_t ldb, double beta, double *C, int64_t ldc, int nprod,
+                           void *ws, size_t ws_bytes, emu_stream_t stream)
+{
+    return gemm_ex<double>(opA, opB, M, N, K, alpha, A, lda, B, ldb, beta, C, ldc, nprod, ws, ws_bytes,
+                           reinterpret_cast<cudaStream_t>(stream));
+}
+
 emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acomps, const uint16_t *Bcomps,
                            int64_t ldcomp, float *C, int64_t ldc, void *ws, size_t ws_bytes, emu_stream_t stream)
 {

@@ -28,4 +28,10 @@ cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *
                                int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
                                int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane = 0);
 
+// General-GEMM epilogue: C <- fl(fl(alpha P) + fl(beta C)) (beta = 0: C <- fl(alpha P), C not read).
+cudaError_t launch_axpby_f32(const float *P, int64_t ldp, float *C, int64_t ldc, int64_t M, int64_t N, float alpha,
+                             float beta, cudaStream_t st);
+cudaError_t launch_axpby_f64(const double *P, int64_t ldp, double *C, int64_t ldc, int64_t M, int64_t N,
+                             double alpha, double beta, cudaStream_t st);
+
 }  // namespace emu

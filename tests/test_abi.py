@@ -83,3 +83,16 @@ def test_host_workspace_sizes(lib):
     # FP64 stages both operands whole: at least 8 (MK + KN) bytes beyond the planes
     assert emu.emu_gemm_host_workspace_bytes(64, M, N, K) >= emu.emu_gemm_workspace_bytes(64, M, N, K) + 8 * (M * K + K * N)
 
+
+def test_gemm_ex_argument_checks_need_no_gpu(lib):
+    P = 16
+    big = 1 << 40
+    assert emu.emu_gemm_ex_f32(2, 0, 4, 4, 4, 1.0, P, 4, P, 4, 0.0, P, 4, P, big, None) == 1   # op
+    assert emu.emu_gemm_ex_f32(1, 0, 4, 4, 8, 1.0, P, 3, P, 4, 0.0, P, 4, P, big, None) == 1   # op(A) = T: lda >= M
+    assert emu.emu_gemm_ex_f32(0, 1, 4, 5, 8, 1.0, P, 8, P, 7, 0.0, P, 5, P, big, None) == 1   # op(B) = T: ldb >= K
+    assert emu.emu_gemm_ex_f64(0, 0, 4, 4, 4, 1.0, P, 4, P, 4, 0.0, P, 4, 7, P, big, None) == 1  # nprod
+    assert emu.emu_gemm_ex_f64(0, 0, 4, 4, 4, 1.0, P, 4, P, 4, 0.0, P, 4, 6, P, 64, None) == 3   # workspace
+    assert emu.emu_gemm_ex_workspace_bytes(32, 10, 20, 30) == (
+        emu.emu_gemm_workspace_bytes(32, 10, 20, 30) + (10 * 20 * 4 + 255) // 256 * 256)
+    assert emu.emu_gemm_ex_workspace_bytes(48, 10, 20, 30) == 0
+

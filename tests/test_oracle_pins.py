@@ -467,3 +467,46 @@ def test_fp64_orders_agree_within_fp64_rounding():
         assert np.all(np.abs(Cc - Cp) <= 2 * nprod * nch * 2.0**-53 * absP)
         ec, ep = oracle.errors(Cc, hi, lo), oracle.errors(Cp, hi, lo)
         assert ep["e_F"] <= 1.01 * ec["e_F"] + 1e-300
+
+
+# ----------------------------------------------------- general GEMM (gemm_ex)
+def _exact_ex(A_eff, B_eff, alpha, beta, C):
+    """alpha op(A) op(B) + beta C in exact rational arithmetic."""
+    from fractions import Fraction
+    M, K = A_eff.shape
+    N = B_eff.shape[1]
+    out = np.empty((M, N), dtype=object)
+    for i in range(M):
+        for j in range(N):
+            p = sum(Fraction(float(A_eff[i, k])) * Fraction(float(B_eff[k, j])) for k in range(K))
+            out[i, j] = Fraction(alpha) * p + (Fraction(beta) * Fraction(float(C[i, j])) if beta != 0 else 0)
+    return out
+
+
+@pytest.mark.parametrize("dtype,nprod", [(np.float32, None), (np.float64, 6)])
+@pytest.mark.parametrize("opA,opB", [(0, 0), (0, 1), (1, 0), (1, 1)])
+def test_gemm_ex_exact_on_small_integers(dtype, nprod, opA, opB):
+    """Small integers are BF16-exact (one slice), so the emulated product is
+    A B exactly (K <= 256 keeps FP32 sums exact); with alpha, beta powers of
+    two the epilogue is exact too.  The oracle must then return
+    alpha op(A) op(B) + beta C exactly, for each placement of the operands."""
+    rng = np.random.default_rng(17 + 2 * opA + opB)
+    M, N, K = 7, 5, 40
+    A_eff = rng.integers(-16, 17, size=(M, K)).astype(dtype)
+    B_eff = rng.integers(-16, 17, size=(K, N)).astype(dtype)
+    C = rng.integers(-100, 101, size=(M, N)).astype(dtype)
+    A = np.ascontiguousarray(A_eff.T) if opA else A_eff
+    B = np.ascontiguousarray(B_eff.T) if opB else B_eff
+    for alpha, beta in [(1.0, 0.0), (0.5, -2.0), (-4.0, 0.25), (2.0, 0.0)]:
+        got, flags = oracle.gemm_ex(opA, opB, alpha, A, B, beta, C, nprod=nprod)
+        assert flags == 0 and got.dtype == dtype
+        want = _exact_ex(A_eff, B_eff, alpha, beta, C)
+        assert all(got[i, j] == float(want[i, j]) for i in range(M) for j in range(N)), (alpha, beta)
+
+
+def test_gemm_ex_beta_zero_does_not_read_c():
+    A, B = synth.gemm_inputs("f64", 9, 6, 30, 5)
+    C = np.full((9, 6), np.nan)
+    got, _ = oracle.gemm_ex(0, 0, 3.0, A, B, 0.0, C, nprod=10)
+    P, _ = oracle.gemm_f64(A, B, 10)
+    assert np.array_equal(got, 3.0 * P)
