@@ -190,7 +190,8 @@ class Case:
         self.Bp = torch.empty((s, N, self.ldk), dtype=torch.int16, device=dev)
         self.v = torch.empty(12, dtype=torch.int32, device=dev)
         self.C = torch.empty((M, N), dtype=torch.float32 if self.mode == 32 else torch.float64, device=dev)
-        self.ws = emu.workspace(emu.emu_split_workspace_bytes(self.mode), dev)
+        self.ws = emu.workspace(max(emu.emu_split_workspace_bytes(self.mode),
+                                    emu.emu_prodsum_workspace_bytes(self.mode, M, N)), dev)
         self.gemm_ws = None
         self.flop = 2.0 * M * N * K
         self.exec_flop = self.flop * (6 if self.mode == 32 else self.nprod)

@@ -103,7 +103,9 @@ emu_status emu_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ld
                          size_t ws_bytes, emu_stream_t stream);
 
 /* Workspace bytes for emu_gemm_f32 (mode 32) / emu_gemm_f64 (mode 64):
- * the flag word plus the slice planes of A (M x K) and B (K x N). */
+ * the flag word plus the slice planes of A (M x K) and B (K x N), and in
+ * mode 64 the product-sum's FP64 accumulator (8 bytes per element of C,
+ * rounded up to 128 x 128 tiles). */
 size_t emu_gemm_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K);
 
 /* FP32-mode emulated GEMM, Algorithm 1: C (M x N, ldc) = A (M x K, lda) . B
@@ -194,6 +196,12 @@ emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
                            const uint16_t *Bcomps, int64_t ldcomp, float *C, int64_t ldc,
                            void *ws, size_t ws_bytes, emu_stream_t stream);
 
+/* Workspace bytes for emu_prodsum_f32 (mode 32: the flag word) and
+ * emu_prodsum_f64 (mode 64: the flag word and the FP64 accumulator of the
+ * product-outer sum, 8 bytes per element of C rounded up to 128 x 128
+ * tiles).  0 for negative sizes or another mode. */
+size_t emu_prodsum_workspace_bytes(int mode, int64_t M, int64_t N);
+
 /* Product-sum alone for FP64 mode, Eq. (fp64reconstruction), summed as in
  * emu_gemm_f64: A planes [6][M][ldcomp], B planes [6][N][ldcomp]; nprod in
  * {6, 10, 15, 21}.  vA, vB: the device arrays of level exponents v^(0..5)
@@ -202,7 +210,7 @@ emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
  * partial with one FP32 addition while the running sum stays below 2^24
  * units (provably exact); both may be NULL, and then every addition is done
  * as an error-free TwoSum (same result, slower).  ws: at least
- * emu_split_workspace_bytes(64). */
+ * emu_prodsum_workspace_bytes(64, M, N) (flag word and FP64 accumulator). */
 emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acomps,
                            const uint16_t *Bcomps, int64_t ldcomp, const int32_t *vA,
                            const int32_t *vB, int nprod, double *C, int64_t ldc, void *ws,
@@ -214,11 +222,12 @@ emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
  * whole device memory budget and forbid allocation calls after start-up, or
  * latency-critical paths that cannot accept the implicit synchronisation of
  * cudaMalloc.  It computes exactly what emu_gemm_f64 computes (same kernels,
- * same results), with its scratch (flag word, level maxima, BF16 planes) in a
- * static device array of EMU_NOALLOC_SCRATCH_BYTES that every GPU loading
- * the library holds until the library is unloaded.
- * Limit: 512 + 12 * (M + N) * roundup(K, 8) bytes (256-byte rounding per
- * operand) must fit the array, e.g. M = N = K = 1024; larger problems
+ * same results), with its scratch (flag word, level maxima, BF16 planes,
+ * FP64 accumulator) in a static device array of EMU_NOALLOC_SCRATCH_BYTES
+ * that every GPU loading the library holds until the library is unloaded.
+ * Limit: 512 + 12 * (M + N) * roundup(K, 8) bytes of planes (256-byte
+ * rounding per operand) plus 8 * roundup(M, 128) * roundup(N, 128) bytes of
+ * accumulator must fit the array, e.g. M = N = K = 1024; larger problems
  * return EMU_ERR_UNSUPPORTED before any work is enqueued.
  * flags_out: device pointer receiving the EMU_FLAG_* word of this call
  * (may be NULL).  The first call on each device looks up the array's device
@@ -226,7 +235,7 @@ emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
  * stream capture.  All calls on a device share the array: calls whose work
  * may overlap on the GPU (different streams or host threads without
  * ordering) race and must be serialised by the caller. */
-#define EMU_NOALLOC_SCRATCH_BYTES (32u << 20)
+#define EMU_NOALLOC_SCRATCH_BYTES (40u << 20)
 emu_status emu_gemm_f64_noalloc(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda,
                                 const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,
                                 uint32_t *flags_out, emu_stream_t stream);

@@ -39,6 +39,7 @@ _SIGS = {
     "emu_gemm_f64_noalloc": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "p"]),
     "emu_gemm_host_workspace_bytes": ("size", ["i", "l", "l", "l"]),
     "emu_gemm_ex_workspace_bytes": ("size", ["i", "l", "l", "l"]),
+    "emu_prodsum_workspace_bytes": ("size", ["i", "l", "l"]),
     "emu_gemm_ex_f32": ("i", ["i", "i", "l", "l", "l", "f", "p", "l", "p", "l", "f", "p", "l", "p", "size", "p"]),
     "emu_gemm_ex_f64": ("i", ["i", "i", "l", "l", "l", "d", "p", "l", "p", "l", "d", "p", "l", "i", "p", "size", "p"]),
     "emu_gemm_f32_host": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "p", "size", "p"]),
@@ -96,6 +97,7 @@ emu_prodsum_f64 = _mk("emu_prodsum_f64")
 emu_gemm_f64_noalloc = _mk("emu_gemm_f64_noalloc")
 emu_gemm_host_workspace_bytes = _mk("emu_gemm_host_workspace_bytes")
 emu_gemm_ex_workspace_bytes = _mk("emu_gemm_ex_workspace_bytes")
+emu_prodsum_workspace_bytes = _mk("emu_prodsum_workspace_bytes")
 emu_gemm_ex_f32 = _mk("emu_gemm_ex_f32")
 emu_gemm_ex_f64 = _mk("emu_gemm_ex_f64")
 emu_gemm_f32_host = _mk("emu_gemm_f32_host")
@@ -249,7 +251,7 @@ def prodsum_f64(Ap, Bp, M: int, N: int, K: int, nprod: int, vA=None, vB=None, C=
     vA, vB: the level exponents emu_split_f64 returned for A and B (or None)."""
     torch = _torch()
     C = C if C is not None else torch.empty((M, N), dtype=torch.float64, device=Ap.device)
-    ws = ws if ws is not None else workspace(emu_split_workspace_bytes(64), Ap.device)
+    ws = ws if ws is not None else workspace(emu_prodsum_workspace_bytes(64, M, N), Ap.device)
     _check(emu_prodsum_f64(M, N, K, Ap.data_ptr(), Bp.data_ptr(), Ap.shape[2],
                            vA.data_ptr() if vA is not None else None, vB.data_ptr() if vB is not None else None,
                            int(nprod), C.data_ptr(), C.stride(0), ws.data_ptr(), ws.numel(), _stream(stream)),

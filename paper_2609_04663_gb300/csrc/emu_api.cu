@@ -62,10 +62,21 @@ emu_status zero_c(T *C, int64_t M, int64_t N, int64_t ldc, cudaStream_t st)
     return cuda_status(cudaMemset2DAsync(C, (size_t)ldc * sizeof(T), 0, (size_t)N * sizeof(T), (size_t)M, st));
 }
 
+// GEMM workspace: header, A planes [s][M][ldk], B planes [s][N][ldk], and in
+// FP64 mode the product-sum's FP64 accumulator.
 size_t gemm_ws_bytes(int s, int64_t M, int64_t N, int64_t K)
 {
     const int64_t ldk = gemm_ldk(K);
-    return kWsHeaderBytes + (size_t)round_up((int64_t)s * M * ldk * 2, 256) + (size_t)round_up((int64_t)s * N * ldk * 2, 256);
+    return kWsHeaderBytes + (size_t)round_up((int64_t)s * M * ldk * 2, 256) +
+           (size_t)round_up((int64_t)s * N * ldk * 2, 256) + (s == 6 ? f64_acc_bytes(M, N) : 0);
+}
+
+// The FP64 accumulator that follows the planes of a GEMM workspace.
+double *gemm_acc(void *ws, int64_t M, int64_t N, int64_t K)
+{
+    const int64_t ldk = gemm_ldk(K);
+    return reinterpret_cast<double *>(static_cast<char *>(ws) + kWsHeaderBytes + round_up(6 * M * ldk * 2, 256) +
+                                      round_up(6 * N * ldk * 2, 256));
 }
 
 }  // namespace
@@ -159,8 +170,15 @@ emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_
     e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st);
     if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st);
     if (e == cudaSuccess)
-        e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, C, ldc, &h->flags, st);
+        e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, C, ldc, gemm_acc(ws, M, N, K),
+                               &h->flags, st);
     return cuda_status(e);
+}
+
+size_t emu_prodsum_workspace_bytes(int mode, int64_t M, int64_t N)
+{
+    if (M < 0 || N < 0 || (mode != 32 && mode != 64)) return 0;
+    return kWsHeaderBytes + (mode == 64 ? f64_acc_bytes(M, N) : 0);
 }
 
 size_t emu_gemm_ex_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K)
@@ -201,7 +219,8 @@ emu_status gemm_ex(int opA, int opB, int64_t M, int64_t N, int64_t K, T alpha, c
     char *w = static_cast<char *>(ws);
     uint16_t *Ap = reinterpret_cast<uint16_t *>(w + kWsHeaderBytes);
     uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(S * M * ldk * 2, 256));
-    T *P = reinterpret_cast<T *>(reinterpret_cast<char *>(Bp) + round_up(S * N * ldk * 2, 256));
+    T *P = reinterpret_cast<T *>(reinterpret_cast<char *>(Bp) + round_up(S * N * ldk * 2, 256) +
+                                 (f64 ? f64_acc_bytes(M, N) : 0));
     const bool direct = (alpha == T(1) && beta == T(0));
     T *out = direct ? C : P;
     const int64_t ldo = direct ? ldc : N;
@@ -215,7 +234,8 @@ emu_status gemm_ex(int opA, int opB, int64_t M, int64_t N, int64_t K, T alpha, c
             e = launch_split_f64(A, ar, ac, lda, ta, Ap, ldk, h->vout[0], h, 0, st);
             if (e == cudaSuccess) e = launch_split_f64(B, br, bc, ldb, tb, Bp, ldk, h->vout[1], h, 1, st);
             if (e == cudaSuccess)
-                e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, out, ldo, &h->flags, st);
+                e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, out, ldo,
+                                       gemm_acc(ws, M, N, K), &h->flags, st);
         } else {
             e = launch_split_f32(A, ar, ac, lda, ta, Ap, ldk, h, st);
             if (e == cudaSuccess) e = launch_split_f32(B, br, bc, ldb, tb, Bp, ldk, h, st);
@@ -274,7 +294,7 @@ emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
     if (M < 0 || N < 0 || K < 0 || ldc < (N > 0 ? N : 1) || !ws) return EMU_ERR_INVALID_ARG;
     if (nprod != 6 && nprod != 10 && nprod != 15 && nprod != 21) return EMU_ERR_INVALID_ARG;
     if (M >= kMaxDim || N >= kMaxDim || K >= kMaxDim) return EMU_ERR_UNSUPPORTED;
-    if (ws_bytes < kWsHeaderBytes) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (ws_bytes < emu_prodsum_workspace_bytes(64, M, N)) return EMU_ERR_WORKSPACE_TOO_SMALL;
     if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     WsHeader *h = static_cast<WsHeader *>(ws);
@@ -285,7 +305,8 @@ emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
     emu_status s = check_planes(Acomps, Bcomps, ldcomp, K);
     if (s != EMU_OK) return s;
     if ((vA == nullptr) != (vB == nullptr)) return EMU_ERR_INVALID_ARG;
-    return cuda_status(launch_prodsum_f64(M, N, K, Acomps, Bcomps, ldcomp, vA, vB, nprod, C, ldc, &h->flags, st));
+    double *acc = reinterpret_cast<double *>(static_cast<char *>(ws) + kWsHeaderBytes);
+    return cuda_status(launch_prodsum_f64(M, N, K, Acomps, Bcomps, ldcomp, vA, vB, nprod, C, ldc, acc, &h->flags, st));
 }
 
 emu_status emu_read_flags(const void *ws, uint32_t *host_flags, emu_stream_t stream)

@@ -79,11 +79,11 @@ struct Geometry {
 };
 
 // Workspace layout (each part 256-byte aligned): header, A planes [s][M][ldk],
-// B planes [s][N][ldk], A staging, B staging, C ring of two row panels.
-// FP32 stages two row panels of A and two K-panels of B; FP64 stages A and B
-// whole.
+// B planes [s][N][ldk], A staging, B staging, C ring of two row panels, and in
+// FP64 mode one product-sum accumulator per ring slot.  FP32 stages two row
+// panels of A and two K-panels of B; FP64 stages A and B whole.
 struct Layout {
-    size_t ap, bp, ast, bst, cring, total;
+    size_t ap, bp, ast, bst, cring, acc, total;
     Layout(int mode, int64_t M, int64_t N, int64_t K)
     {
         const Geometry g(M, K);
@@ -95,7 +95,8 @@ struct Layout {
         const int64_t b_stage = mode == 64 ? K * N : 2 * g.Kp * N;
         bst = ast + (size_t)round_up(a_stage * esz, 256);
         cring = bst + (size_t)round_up(b_stage * esz, 256);
-        total = cring + (size_t)round_up(2 * g.Mp * N * esz, 256);
+        acc = cring + (size_t)round_up(2 * g.Mp * N * esz, 256);
+        total = acc + (mode == 64 ? 2 * f64_acc_bytes(g.Mp, N) : 0);   // FP64 accumulators of the two ring slots
     }
 };
 
@@ -282,9 +283,10 @@ emu_status emu_gemm_f64_host(int64_t M, int64_t N, int64_t K, const double *A, i
         if (e == cudaSuccess) e = cudaStreamWaitEvent(cx->comp[1], split, 0);
     }
     auto prepare = [](int64_t, int64_t, int64_t, cudaStream_t) -> cudaError_t { return cudaSuccess; };
-    auto compute = [&](int64_t, int64_t m0, int64_t mp, double *cr, cudaStream_t cs) -> cudaError_t {
+    auto compute = [&](int64_t i, int64_t m0, int64_t mp, double *cr, cudaStream_t cs) -> cudaError_t {
         if (K == 0) return cudaMemsetAsync(cr, 0, (size_t)mp * N * 8, cs);
-        return launch_prodsum_f64(mp, N, K, Ap + m0 * g.ldk, Bp, g.ldk, h->vout[0], h->vout[1], nprod, cr, N,
+        double *acc = reinterpret_cast<double *>(w + L.acc + (i & 1) * f64_acc_bytes(g.Mp, N));
+        return launch_prodsum_f64(mp, N, K, Ap + m0 * g.ldk, Bp, g.ldk, h->vout[0], h->vout[1], nprod, cr, N, acc,
                                   &h->flags, cs, a_plane);
     };
     if (e == cudaSuccess) e = row_panels(*cx, ne, g, M, N, C, ldc, cring, prepare, compute);

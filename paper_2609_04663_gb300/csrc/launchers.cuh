@@ -24,9 +24,16 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
 cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
                                int64_t a_plane = 0);
+// acc: FP64 accumulator scratch of f64_acc_bytes(M, N) bytes (16-byte aligned).
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
-                               int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane = 0);
+                               int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane = 0);
+
+// Bytes of the FP64 product-sum's accumulator: one 128 x 128 FP64 tile per CTA tile.
+inline size_t f64_acc_bytes(int64_t M, int64_t N)
+{
+    return (size_t)((M + 127) / 128) * (size_t)((N + 127) / 128) * 128u * 128u * sizeof(double);
+}
 
 // General-GEMM epilogue: C <- fl(fl(alpha P) + fl(beta C)) (beta = 0: C <- fl(alpha P), C not read).
 cudaError_t launch_axpby_f32(const float *P, int64_t ldp, float *C, int64_t ldc, int64_t M, int64_t N, float alpha,

@@ -9,7 +9,7 @@
 // same split and product-sum kernels as emu_gemm_f64 with their scratch (flag
 // word, level maxima, BF16 planes) in the file-scope device array below.
 //
-// The array is EMU_NOALLOC_SCRATCH_BYTES (32 MiB) on every GPU that loads the
+// The array is EMU_NOALLOC_SCRATCH_BYTES (40 MiB) on every GPU that loads the
 // library, for as long as the library stays loaded.  All calls on a device
 // share it: each call clears the parts that must start at zero and overwrites
 // the rest, and calls whose work overlaps on the GPU (other streams, other
@@ -60,10 +60,11 @@ extern "C" emu_status emu_gemm_f64_noalloc(int64_t M, int64_t N, int64_t K, cons
     if (lda < (K > 0 ? K : 1) || ldb < (N > 0 ? N : 1) || ldc < (N > 0 ? N : 1)) return EMU_ERR_INVALID_ARG;
     if (nprod != 6 && nprod != 10 && nprod != 15 && nprod != 21) return EMU_ERR_INVALID_ARG;
     if (M > 0 && N > 0 && (!C || (K > 0 && (!A || !B)))) return EMU_ERR_INVALID_ARG;
-    // scratch: header, then 6 A planes [M][ldk] and 6 B planes [N][ldk] of BF16
+    // scratch: header, 6 A planes [M][ldk] and 6 B planes [N][ldk] of BF16, FP64 accumulator
     const int64_t ldk = round_up(K < 1 ? 1 : K, 8);
     const int64_t a_bytes = round_up(6 * M * ldk * 2, 256);
-    const int64_t need = (int64_t)kWsHeaderBytes + a_bytes + round_up(6 * N * ldk * 2, 256);
+    const int64_t b_bytes = round_up(6 * N * ldk * 2, 256);
+    const int64_t need = (int64_t)kWsHeaderBytes + a_bytes + b_bytes + (int64_t)f64_acc_bytes(M, N);
     if (M >= ((int64_t)1 << 31) || N >= ((int64_t)1 << 31) || K >= ((int64_t)1 << 31) ||
         need > (int64_t)EMU_NOALLOC_SCRATCH_BYTES)
         return EMU_ERR_UNSUPPORTED;
@@ -82,7 +83,9 @@ extern "C" emu_status emu_gemm_f64_noalloc(int64_t M, int64_t N, int64_t K, cons
             e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st);
             if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st);
             if (e == cudaSuccess)
-                e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, C, ldc, &h->flags, st);
+                e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, C, ldc,
+                                       reinterpret_cast<double *>(scratch + kWsHeaderBytes + a_bytes + b_bytes),
+                                       &h->flags, st);
         }
     }
     if (e == cudaSuccess && flags_out)

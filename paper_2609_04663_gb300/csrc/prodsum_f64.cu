@@ -16,14 +16,17 @@
 // the other); (hi, lo) is renormalised by another TwoSum whenever lo reaches
 // 2^23 u, so the additions into lo are exact for any K.
 //
-// A finished product's sums go through a 64 KB shared-memory hand-off to four
-// fold warps, which add hi + lo (exact in FP64) once into the FP64
-// accumulator in the upper 256 TMEM columns: C <- fl64(C + fl32(A_i B_j)),
-// Algorithm 2's step.  GB300's FP64 pipe does two adds per clock per SM, so
-// a product's 128 x 128 FP64 adds take as long as several chunk partials; with
-// the fold in its own warps the drain warps go straight on to the next
-// product and the tensor cores keep running.  The result is bit-identical to
-// the oracle in its product-outer order.
+// A finished product's sums go through a 128-column TMEM hand-off area to
+// four fold warps, which add hi + lo (exact in FP64) once into the FP64
+// accumulator: C <- fl64(C + fl32(A_i B_j)), Algorithm 2's step.  GB300's
+// FP64 pipe does two adds per clock per SM, so a product's 128 x 128 FP64
+// adds take as long as several chunk partials; with the fold in its own warps
+// the drain warps go straight on to the next product and the tensor cores
+// keep running.  The FP64 accumulator lives in a workspace buffer (tile by
+// tile, 128 KB per CTA, L2-resident while the tile runs), which leaves TMEM
+// for three partial buffers and the hand-off and shared memory for three
+// 64 KB operand stages.  The result is bit-identical to the oracle in its
+// product-outer order.
 //
 // Warp roles: warp 0 lane 0 issues TMA loads, warp 1 owns TMEM and lane 0
 // issues the MMAs, warps 4-19 drain (four per TMEM lane quarter, 32 columns
@@ -46,17 +49,15 @@ __constant__ int8_t kDiag[21][2] = {{0, 0}, {0, 1}, {1, 0}, {0, 2}, {1, 1}, {2, 
 struct F64Cfg {
     // A stage holds SUB K-blocks of 64 (one 128-byte swizzle row each) of the
     // A slice and of the B slice.
-    static constexpr int BN = 128, KB = 64, SUB = 2, STAGES = 2, NBUF = 2;
+    static constexpr int BN = 128, KB = 64, SUB = 2, STAGES = 3, NBUF = 3;
     static constexpr int KSPAN = KB * SUB;                          // K per stage
     static constexpr int A_SUB = kBM * KB * 2, B_SUB = BN * KB * 2; // one 64-wide K-block tile
     static constexpr int A_TILE = A_SUB * SUB, B_TILE = B_SUB * SUB;
     static constexpr int STAGE = A_TILE + B_TILE;
     static constexpr uint32_t SWZ = 2u, SBO = 1024u;              // 128-byte swizzle
-    // hand-off of a product's sums: [128 rows][128 columns] FP32, 16-byte
-    // chunks of a row XOR-swizzled by (row & 7); then one low-part mask byte
-    // per (row, drain column quarter)
-    static constexpr int HAND_OFF = STAGES * STAGE;
-    static constexpr int MASK_OFF = HAND_OFF + kBM * BN * 4;
+    // one low-part mask byte per (row, drain column quarter) of the product
+    // being handed off
+    static constexpr int MASK_OFF = STAGES * STAGE;
     static constexpr int BAR_OFF = MASK_OFF + kBM * 4;
     // barriers: full/empty per stage, tfull/tempty per buffer, hand-off
     // full/empty, done; then the TMEM address slot
@@ -69,9 +70,10 @@ struct F64Cfg {
     // Register split: the launch reserves 768 x 80 (six warps per SMSP);
     // 128 x 32 (control) + 512 x 96 (drain) + 128 x 64 (fold) = 61440 = 768 x 80.
     static constexpr int REG_CTRL = 32, REG_DRAIN = 96, REG_FOLD = 64, REG_LAUNCH = 80;
-    static constexpr uint32_t ACC_COL = NBUF * BN;                 // FP64 accumulator: 2 words per column
+    static constexpr uint32_t HP_COL = NBUF * BN;                  // hand-off area: one FP32 word per column
 };
-static_assert(F64Cfg::ACC_COL + 2 * F64Cfg::BN == 512, "TMEM budget: 2 partial buffers + FP64 accumulator");
+static_assert(F64Cfg::HP_COL + F64Cfg::BN == 512, "TMEM budget: 3 partial buffers + hand-off area");
+static_assert(kBM == 128 && F64Cfg::BN == 128, "f64_acc_bytes assumes 128 x 128 tiles");
 static_assert(kKChunk % F64Cfg::KSPAN == 0, "a K-chunk is a whole number of stages");
 static_assert(8 * F64Cfg::NBARS + 8 <= 256, "barrier area");
 static_assert(F64Cfg::SMEM <= 232448, "shared memory per CTA");
@@ -168,30 +170,11 @@ __device__ __forceinline__ float two_sum(float a, float b, float &e)
     return s;
 }
 
-__device__ __forceinline__ void sts_v4(uint32_t addr, float a, float b, float c, float d)
-{
-    asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d) : "memory");
-}
-
-__device__ __forceinline__ float4 lds_v4(uint32_t addr)
-{
-    float4 v;
-    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr) : "memory");
-    return v;
-}
-
-// Shared-memory address of 16-byte chunk `c` (columns 4c .. 4c+3) of row r
-// of the hand-off area.
-__device__ __forceinline__ uint32_t hand_addr(uint32_t hand, int r, int c)
-{
-    return hand + (uint32_t)(r * 512 + ((c ^ (r & 7)) << 4));
-}
-
 template <int NPROD>
 __global__ void __launch_bounds__(F64Cfg::THREADS, 1)
 prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    int M, int N, int K, const int32_t *__restrict__ vA, const int32_t *__restrict__ vB,
-                   double *__restrict__ C, int64_t ldc, uint32_t *flags)
+                   double *__restrict__ C, int64_t ldc, double *__restrict__ acc, uint32_t *flags)
 {
     using Cfg = F64Cfg;
     extern __shared__ uint8_t smem_raw[];
@@ -201,7 +184,7 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     const uint32_t full0 = base + Cfg::BAR_OFF, empty0 = full0 + 8u * Cfg::STAGES;
     const uint32_t tfull0 = empty0 + 8u * Cfg::STAGES, tempty0 = tfull0 + 8u * Cfg::NBUF;
     const uint32_t hfull = tempty0 + 8u * Cfg::NBUF, hempty = hfull + 8u, done_bar = hempty + 8u;
-    const uint32_t hand = base + Cfg::HAND_OFF, hmask = base + Cfg::MASK_OFF;
+    const uint32_t hmask = base + Cfg::MASK_OFF;
     volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(base_ptr + Cfg::BAR_OFF + 8 * Cfg::NBARS);
 
     const int warp = threadIdx.x >> 5, lane = lane_id();
@@ -294,6 +277,7 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
         const int cq = (warp - Cfg::FIRST_DRAIN) >> 2;                   // column quarter
         const int r = quarter * 32 + lane;                               // tile row of this thread
         const uint32_t tcol = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(cq * Cfg::COLS);
+        const uint32_t thp = tcol + Cfg::HP_COL;                         // this thread's hand-off columns
         const int row = m0 + r;
         double *crow = C + (int64_t)row * ldc + n0 + cq * Cfg::COLS;
         const int lim = row < M ? N - (n0 + cq * Cfg::COLS) : 0;        // valid columns of this thread
@@ -362,9 +346,15 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                 if (!ok) break;
             }
 #pragma unroll
-            for (int k = 0; k < Cfg::COLS / 4; ++k)
-                sts_v4(hand_addr(hand, r, cq * (Cfg::COLS / 4) + k), hi[4 * k], hi[4 * k + 1], hi[4 * k + 2], hi[4 * k + 3]);
+            for (int h = 0; h < Cfg::COLS; h += 16) {
+                uint32_t w[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) w[j] = __float_as_uint(hi[h + j]);
+                tmem_st16(thp + (uint32_t)h, w);
+            }
+            tmem_st_wait();
             asm volatile("st.shared.u8 [%0], %1;" ::"r"(hmask + (uint32_t)(r * 4 + cq)), "r"(dirty) : "memory");
+            tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(hfull);
         }
@@ -373,57 +363,61 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
         // ---------------- fold: C <- fl64(C + (hi + lo)) per product, in product order
         const int quarter = warp & 3;
         const int r = quarter * 32 + lane;
-        const uint32_t tacc = tmem + ((uint32_t)(quarter * 32) << 16) + Cfg::ACC_COL;
+        const uint32_t thp = tmem + ((uint32_t)(quarter * 32) << 16) + Cfg::HP_COL;
         const int row = m0 + r;
         double *crow = C + (int64_t)row * ldc + n0;
+        // this tile's accumulator, column-major: a warp's 32 rows of a column are contiguous
+        double *tacc = acc + ((size_t)tm * tiles_n + tn) * (size_t)(kBM * Cfg::BN) + r;
         const int lim = row < M ? N - n0 : 0;
         const bool vec = ((ldc & 1) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15u) == 0);
         for (int q = 0; q < NPROD; ++q) {
             const bool ok = mbar_wait(hfull, (uint32_t)(q & 1), flags);
             __syncwarp();
             if (!ok) break;
-            const bool last = (q == NPROD - 1);
+            tc_fence_after();
+            const bool first = (q == 0), last = (q == NPROD - 1);
             const float *lrow = reinterpret_cast<const float *>(crow) + (q & 1);
+            double nxt[8];                                   // accumulator of the next 8 columns (prefetched)
+            if (!first) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) nxt[j] = tacc[j * kBM];
+            }
 #pragma unroll 1
-            for (int cq = 0; cq < 4; ++cq) {
+            for (int col = 0; col < Cfg::BN; col += 8) {
+                double cur[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) cur[j] = nxt[j];
+                if (!first && col + 8 < Cfg::BN) {
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) nxt[j] = tacc[(col + 8 + j) * kBM];
+                }
+                uint32_t hv[8];
+                tmem_ld8(thp + (uint32_t)col, hv);
                 uint32_t mask;
-                asm volatile("ld.shared.u8 %0, [%1];" : "=r"(mask) : "r"(hmask + (uint32_t)(r * 4 + cq)) : "memory");
+                asm volatile("ld.shared.u8 %0, [%1];" : "=r"(mask) : "r"(hmask + (uint32_t)(r * 4 + (col >> 5))) : "memory");
+                const bool dg = (mask >> ((col >> 4) & 1)) & 1u;   // 16-column group of these 8 columns
+                tmem_ld_wait();
+                double out[8];
 #pragma unroll
-                for (int k = 0; k < 8; k += 2) {
-                    const int col = cq * 32 + 4 * k;                 // 8 columns: chunks k, k + 1
-                    const float4 h0 = lds_v4(hand_addr(hand, r, cq * 8 + k));
-                    const float4 h1 = lds_v4(hand_addr(hand, r, cq * 8 + k + 1));
-                    const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
-                    uint32_t w[16];
-                    if (q > 0) {
-                        tmem_ld16(tacc + 2u * (uint32_t)col, w);
-                        tmem_ld_wait();
-                    }
-                    const bool dg = (mask >> (k / 4)) & 1u;      // 16-column group of these 8 columns
+                for (int j = 0; j < 8; ++j) {
+                    double sq = widen_exact(__uint_as_float(hv[j]));
+                    if (dg && col + j < lim) sq = __dadd_rn(sq, widen_exact(lrow[2 * (col + j)]));   // exact
+                    out[j] = first ? sq : __dadd_rn(cur[j], sq);
+                }
+                if (!last) {
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        double sq = widen_exact(hv[j]);
-                        if (dg && col + j < lim) sq = __dadd_rn(sq, widen_exact(lrow[2 * (col + j)]));   // exact
-                        const double cprev = (q > 0) ? __hiloint2double((int)w[2 * j + 1], (int)w[2 * j]) : 0.0;
-                        const double out = __dadd_rn(cprev, sq);
-                        w[2 * j] = (uint32_t)__double2loint(out);
-                        w[2 * j + 1] = (uint32_t)__double2hiint(out);
-                    }
-                    if (!last) {
-                        tmem_st16(tacc + 2u * (uint32_t)col, w);
-                    } else if (vec && lim >= col + 8) {
+                    for (int j = 0; j < 8; ++j) tacc[(col + j) * kBM] = out[j];
+                } else if (vec && lim >= col + 8) {
 #pragma unroll
-                        for (int j = 0; j < 8; j += 2)
-                            *reinterpret_cast<int4 *>(crow + col + j) =
-                                make_int4((int)w[2 * j], (int)w[2 * j + 1], (int)w[2 * j + 2], (int)w[2 * j + 3]);
-                    } else {
+                    for (int j = 0; j < 8; j += 2)
+                        *reinterpret_cast<double2 *>(crow + col + j) = make_double2(out[j], out[j + 1]);
+                } else {
 #pragma unroll
-                        for (int j = 0; j < 8; ++j)
-                            if (col + j < lim) crow[col + j] = __hiloint2double((int)w[2 * j + 1], (int)w[2 * j]);
-                    }
+                    for (int j = 0; j < 8; ++j)
+                        if (col + j < lim) crow[col + j] = out[j];
                 }
             }
-            if (!last) tmem_st_wait();
+            tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(hempty);
         }
@@ -439,8 +433,8 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
 
 template <int NPROD>
 cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
-                    const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
-                    int64_t a_plane)
+                    const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, double *acc, uint32_t *flags,
+                    cudaStream_t st, int64_t a_plane)
 {
     using Cfg = F64Cfg;
     CUtensorMap ta, tb;
@@ -450,7 +444,7 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
     const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + Cfg::BN - 1) / Cfg::BN);
-    kern<<<(unsigned)tiles, Cfg::THREADS, Cfg::SMEM, st>>>(ta, tb, (int)M, (int)N, (int)K, vA, vB, C, ldc, flags);
+    kern<<<(unsigned)tiles, Cfg::THREADS, Cfg::SMEM, st>>>(ta, tb, (int)M, (int)N, (int)K, vA, vB, C, ldc, acc, flags);
     return cudaGetLastError();
 }
 
@@ -458,13 +452,13 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
 
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
-                               int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane)
+                               int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane)
 {
     switch (nprod) {
-    case 6: return run_f64<6>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st, a_plane);
-    case 10: return run_f64<10>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st, a_plane);
-    case 15: return run_f64<15>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st, a_plane);
-    case 21: return run_f64<21>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, flags, st, a_plane);
+    case 6: return run_f64<6>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
+    case 10: return run_f64<10>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
+    case 15: return run_f64<15>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
+    case 21: return run_f64<21>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
     default: return cudaErrorInvalidValue;
     }
 }

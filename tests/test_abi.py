@@ -96,3 +96,13 @@ def test_gemm_ex_argument_checks_need_no_gpu(lib):
         emu.emu_gemm_workspace_bytes(32, 10, 20, 30) + (10 * 20 * 4 + 255) // 256 * 256)
     assert emu.emu_gemm_ex_workspace_bytes(48, 10, 20, 30) == 0
 
+
+
+def test_prodsum_workspace_sizes_and_check(lib):
+    assert emu.emu_prodsum_workspace_bytes(32, 300, 200) == emu.emu_split_workspace_bytes(32)
+    # FP64: the header plus one 128 x 128 FP64 accumulator tile per CTA tile
+    assert emu.emu_prodsum_workspace_bytes(64, 300, 200) == emu.emu_split_workspace_bytes(64) + 3 * 2 * 128 * 128 * 8
+    assert emu.emu_prodsum_workspace_bytes(64, -1, 2) == 0
+    P = 16
+    small = emu.emu_split_workspace_bytes(64)
+    assert emu.emu_prodsum_f64(300, 200, 64, P, P, 64, P, P, 6, P, 200, P, small, None) == 3
