@@ -426,7 +426,8 @@ def gpu_arm(args, rank, world, local):
                 "frac": achieved / pk["bf16_burst"],
                 "peak_source": f"{pk['source']} bf16 burst (cuBLAS 8192^3); sustained {pk['bf16_sustained']}",
                 "kernel": "prodsum_f32_kernel" if case.mode == 32 else "prodsum_f64_kernel",
-                "traffic": kernel_traffic("prodsum_f32" if case.mode == 32 else "prodsum_f64", name)}
+                "traffic": kernel_traffic("prodsum_f32" if case.mode == 32 else "prodsum_f64",
+                                          name if case.mode == 32 else f"{name}_np{case.nprod}")}
     flags = case.emu.read_flags(case.ws)
     e2e = None if args.no_e2e else time_e2e(case, max(2, min(args.steps, 5)), 1, world)
     split_gbs = case.split_bytes() / (split_ms / 1e3) / 1e9
