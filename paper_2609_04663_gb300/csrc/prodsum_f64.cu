@@ -84,16 +84,26 @@ static_assert(128 * F64Cfg::REG_CTRL + 512 * F64Cfg::REG_DRAIN + 128 * F64Cfg::R
 template <uint32_t R> __device__ __forceinline__ void regs_dec() { asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R)); }
 template <uint32_t R> __device__ __forceinline__ void regs_inc() { asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(R)); }
 
-// Exact FP32 -> FP64 widening of a normal or zero value by bit operations
-// (rebias the exponent, shift the significand); other values take the
-// conversion instruction.
+// Exact FP32 -> FP64 widening by integer operations only (on GB300 a
+// conversion instruction would occupy the FP64 pipe, which the fold's adds
+// need): rebias the exponent and shift the significand of a normal value;
+// normalise a subnormal by its leading bit; keep zeros, infinities and NaN
+// payloads.
 __device__ __forceinline__ double widen_exact(float x)
 {
     const uint32_t u = __float_as_uint(x);
-    const uint32_t ex = (u >> 23) & 0xFFu;
-    if ((u & 0x7FFFFFFFu) == 0u) return __hiloint2double((int)(u & 0x80000000u), 0);
-    if (ex == 0u || ex == 0xFFu) return (double)x;
-    return __hiloint2double((int)((u & 0x80000000u) | ((ex + 896u) << 20) | ((u & 0x7FFFFFu) >> 3)), (int)(u << 29));
+    const uint32_t sign = u & 0x80000000u, ex = (u >> 23) & 0xFFu, m = u & 0x7FFFFFu;
+    uint32_t e = ex + 896u, f = m;                     // normal: exponent rebased from bias 127 to 1023
+    if (ex == 0xFFu) e = 0x7FFu;                       // infinity / NaN
+    if (ex == 0u) {
+        if (m == 0u) { e = 0u; }                       // zero
+        else {                                         // subnormal: m * 2^-149, leading bit at p
+            const int p = 31 - __clz(m);
+            e = (uint32_t)(p + 874);                   // p - 149 + 1023
+            f = (m << (23 - p)) & 0x7FFFFFu;
+        }
+    }
+    return __hiloint2double((int)(sign | (e << 20) | (f >> 3)), (int)(f << 29));
 }
 
 
