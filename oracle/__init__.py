@@ -110,6 +110,37 @@ def split_f64(X: np.ndarray):
     return planes, v, int(flags)
 
 
+def split_f64_rows(X: np.ndarray):
+    """Eq. (fp64split) with one set of levels per row: the standard Ozaki
+    scaling of Eq. (ozakiscaled) on row vectors (Section 4.3).  Each row is
+    split exactly as the whole-matrix split splits a one-row matrix.  Returns
+    (planes uint16 [6, rows, cols], v int32 [rows, 6], flags)."""
+    X = np.ascontiguousarray(X, dtype=np.float64)
+    rows, cols = X.shape
+    planes = np.zeros((6, rows, cols), dtype=np.uint16)
+    v = np.empty((rows, 6), dtype=np.int32)
+    flags = 0
+    for i in range(rows):
+        p, vi, f = split_f64(X[i:i + 1])
+        planes[:, i:i + 1, :] = p
+        v[i] = vi
+        flags |= f
+    return planes, v, flags
+
+
+def gemm_f64_rowcol(A: np.ndarray, B: np.ndarray, nprod: int, rows=None):
+    """Algorithm 2 with per-row levels for A and per-column levels for B: the
+    slices of A are split row by row, those of B column by column (rows of
+    B^T), and the product-sum is Algorithm 2's product-outer sum.  Returns
+    (C, flags)."""
+    Ap, _, fa = split_f64_rows(A)
+    Bt, _, fb = split_f64_rows(np.ascontiguousarray(B.T))
+    Bp = np.ascontiguousarray(Bt.transpose(0, 2, 1))
+    if rows is not None:
+        Ap = Ap[:, rows[0]:rows[1]]
+    return prodsum_f64(Ap, Bp, nprod), fa | fb
+
+
 def products(mode: int, nprod: int):
     """Executed (i, j) order: FP32 reuse chain, or FP64 diagonal order."""
     buf = np.zeros(2 * 21, dtype=np.int32)

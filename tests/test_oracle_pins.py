@@ -510,3 +510,67 @@ def test_gemm_ex_beta_zero_does_not_read_c():
     got, _ = oracle.gemm_ex(0, 0, 3.0, A, B, 0.0, C, nprod=10)
     P, _ = oracle.gemm_f64(A, B, 10)
     assert np.array_equal(got, 3.0 * P)
+
+
+# --------------------------------------- per-row / per-column levels (NEXT-2)
+def test_split_rows_commutes_with_power_of_two_row_scaling():
+    """With one set of levels per row, scaling a row by 2^e scales every slice
+    of that row by 2^e and shifts its levels by e, exactly.  A split that
+    shared levels across rows would round the small rows on the large rows'
+    grid and fail this."""
+    rng = np.random.default_rng(31)
+    U = synth.uniform_f64(31, 0, (12, 40))
+    e = rng.integers(-60, 60, size=12)
+    X = U * np.ldexp(1.0, e)[:, None]
+    P, v, f = oracle.split_f64_rows(X)
+    Pu, vu, fu = oracle.split_f64_rows(U)
+    assert f == fu == 0
+    vals = (P.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    vals_u = (Pu.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    assert np.array_equal(vals, vals_u * np.ldexp(1.0, e)[None, :, None])
+    assert np.array_equal(v, vu + e[:, None])
+
+
+def test_split_rows_levels_are_the_row_maxima():
+    """v[i, r] = ceil(log2 max_j |A^(r)_ij|) row by row, and a row that is
+    exact after r slices stops there (zero levels), independently of other rows."""
+    X = synth.uniform_f64(32, 0, (5, 30))
+    X[2] = np.round(X[2] * 64)                      # integers: one slice
+    P, v, _ = oracle.split_f64_rows(X)
+    for i in range(5):
+        R = X[i].copy()
+        for r in range(6):
+            m = np.max(np.abs(R))
+            if m == 0:
+                assert v[i, r] == oracle.ZERO_LEVEL
+                continue
+            assert 2.0 ** (v[i, r] - 1) < m <= 2.0 ** v[i, r]
+            R = R - (P[r, i].astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    assert v[2, 1] == oracle.ZERO_LEVEL
+
+
+def test_gemm_rowcol_commutes_with_row_and_column_scaling():
+    """Per-row levels for A and per-column levels for B make the emulated
+    product of D_A U and V D_B (D diagonal powers of two) equal to
+    D_A (U V) D_B exactly, with every chunk partial exact in its own unit; one
+    level per matrix instead rounds the small rows and columns on the large
+    ones' grid and loses them (far larger scaled error, same product count)."""
+    M, N, K = 24, 20, 300
+    U, V = synth.gemm_inputs("f64", M, N, K, 4)
+    rng = np.random.default_rng(33)
+    ea, eb = rng.integers(-40, 41, size=M), rng.integers(-40, 41, size=N)
+    A, B = U * np.ldexp(1.0, ea)[:, None], V * np.ldexp(1.0, eb)[None, :]
+    Ap, _, _ = oracle.split_f64_rows(A)
+    Bt, _, _ = oracle.split_f64_rows(np.ascontiguousarray(B.T))
+    _, bad = oracle.prodsum_f64(Ap, np.ascontiguousarray(Bt.transpose(0, 2, 1)), 21, check_exact=True)
+    assert bad == 0
+    for nprod in (6, 10, 21):
+        C1, f1 = oracle.gemm_f64_rowcol(A, B, nprod)
+        C0, f0 = oracle.gemm_f64_rowcol(U, V, nprod)
+        assert f1 == f0 == 0
+        assert np.array_equal(C1, C0 * np.ldexp(1.0, ea)[:, None] * np.ldexp(1.0, eb)[None, :])
+    hi, lo = oracle.ref_dd(A, B)
+    absab = np.abs(A) @ np.abs(B)
+    e_rc = oracle.errors(oracle.gemm_f64_rowcol(A, B, 10)[0], hi, lo, absab)["e_scaled"]
+    e_gl = oracle.errors(oracle.gemm_f64(A, B, 10)[0], hi, lo, absab)["e_scaled"]
+    assert e_rc < 1e-3 * e_gl, (e_rc, e_gl)
