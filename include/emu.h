@@ -102,6 +102,36 @@ emu_status emu_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ld
                          uint16_t *comps, int64_t ldcomp, int32_t *v_out, void *ws,
                          size_t ws_bytes, emu_stream_t stream);
 
+/* Eq. (fp64split) with one set of six levels per plane row instead of one per
+ * matrix: the vector scaling of the standard Ozaki scheme (Eq.
+ * (ozakiscaled), Section 4.3).  Plane rows are the rows of X (transpose = 0)
+ * or its columns (transpose = 1, K-major planes for the B operand), so a
+ * GEMM gets levels per row of A and per column of B.  Each vector is split
+ * exactly as the whole-matrix split would split it alone, so rows and columns
+ * of very different magnitudes keep their own precision; results are
+ * bit-identical to the oracle's split_f64_rows.  comps: 6 planes
+ * [6][plane rows][ldcomp]; v_out: device int32 [6][plane rows]
+ * (level-major; EMU_ZERO_LEVEL once a vector's residual is zero); ws: at
+ * least emu_split_f64_rowcol_workspace_bytes(plane rows).  Flags as
+ * emu_split_f64. */
+size_t emu_split_f64_rowcol_workspace_bytes(int64_t plane_rows);
+emu_status emu_split_f64_rowcol(const double *X, int64_t rows, int64_t cols, int64_t ldx,
+                                int transpose, uint16_t *comps, int64_t ldcomp, int32_t *v_out,
+                                void *ws, size_t ws_bytes, emu_stream_t stream);
+
+/* FP64-mode GEMM (Algorithm 2, same product-outer sum as emu_gemm_f64)
+ * with levels per row of A and per column of B (emu_split_f64_rowcol).
+ * Every chunk partial stays exact in the unit of its own output element, so
+ * C equals the oracle's gemm_f64_rowcol bit for bit.  Row and column scaling
+ * by powers of two commutes with it exactly, which the whole-matrix levels
+ * of emu_gemm_f64 cannot offer.  ws: at least
+ * emu_gemm_f64_rowcol_workspace_bytes (the GEMM workspace plus the levels).
+ * Errors as emu_gemm_f64. */
+size_t emu_gemm_f64_rowcol_workspace_bytes(int64_t M, int64_t N, int64_t K);
+emu_status emu_gemm_f64_rowcol(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda,
+                               const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,
+                               void *ws, size_t ws_bytes, emu_stream_t stream);
+
 /* Workspace bytes for emu_gemm_f32 (mode 32) / emu_gemm_f64 (mode 64):
  * the flag word plus the slice planes of A (M x K) and B (K x N), and in
  * mode 64 the product-sum's FP64 accumulator (8 bytes per element of C,

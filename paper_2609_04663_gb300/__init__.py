@@ -40,6 +40,10 @@ _SIGS = {
     "emu_gemm_host_workspace_bytes": ("size", ["i", "l", "l", "l"]),
     "emu_gemm_ex_workspace_bytes": ("size", ["i", "l", "l", "l"]),
     "emu_prodsum_workspace_bytes": ("size", ["i", "l", "l"]),
+    "emu_split_f64_rowcol_workspace_bytes": ("size", ["l"]),
+    "emu_split_f64_rowcol": ("i", ["p", "l", "l", "l", "i", "p", "l", "p", "p", "size", "p"]),
+    "emu_gemm_f64_rowcol_workspace_bytes": ("size", ["l", "l", "l"]),
+    "emu_gemm_f64_rowcol": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "size", "p"]),
     "emu_gemm_ex_f32": ("i", ["i", "i", "l", "l", "l", "f", "p", "l", "p", "l", "f", "p", "l", "p", "size", "p"]),
     "emu_gemm_ex_f64": ("i", ["i", "i", "l", "l", "l", "d", "p", "l", "p", "l", "d", "p", "l", "i", "p", "size", "p"]),
     "emu_gemm_f32_host": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "p", "size", "p"]),
@@ -98,6 +102,10 @@ emu_gemm_f64_noalloc = _mk("emu_gemm_f64_noalloc")
 emu_gemm_host_workspace_bytes = _mk("emu_gemm_host_workspace_bytes")
 emu_gemm_ex_workspace_bytes = _mk("emu_gemm_ex_workspace_bytes")
 emu_prodsum_workspace_bytes = _mk("emu_prodsum_workspace_bytes")
+emu_split_f64_rowcol_workspace_bytes = _mk("emu_split_f64_rowcol_workspace_bytes")
+emu_split_f64_rowcol = _mk("emu_split_f64_rowcol")
+emu_gemm_f64_rowcol_workspace_bytes = _mk("emu_gemm_f64_rowcol_workspace_bytes")
+emu_gemm_f64_rowcol = _mk("emu_gemm_f64_rowcol")
 emu_gemm_ex_f32 = _mk("emu_gemm_ex_f32")
 emu_gemm_ex_f64 = _mk("emu_gemm_ex_f64")
 emu_gemm_f32_host = _mk("emu_gemm_f32_host")
@@ -166,6 +174,34 @@ def split_f64(X, transpose: bool = False, ldcomp: int | None = None, ws=None, st
     _check(emu_split_f64(X.data_ptr(), rows, cols, X.stride(0), int(transpose), planes.data_ptr(), ldcomp,
                          v.data_ptr(), ws.data_ptr(), ws.numel(), _stream(stream)), "emu_split_f64")
     return planes, v, ws
+
+
+def split_f64_rowcol(X, transpose: bool = False, ldcomp: int | None = None, ws=None, stream=None):
+    """emu_split_f64_rowcol: levels per row of X (per column when transposed).
+    Returns (planes int16 [6, plane_rows, ldcomp], v int32 [6, plane_rows] (device), ws)."""
+    torch = _torch()
+    rows, cols = X.shape
+    prow, pcols = (cols, rows) if transpose else (rows, cols)
+    ldcomp = ldcomp or pcols
+    planes = torch.zeros((6, prow, ldcomp), dtype=torch.int16, device=X.device)
+    v = torch.empty((6, prow), dtype=torch.int32, device=X.device)
+    ws = ws if ws is not None else workspace(emu_split_f64_rowcol_workspace_bytes(prow), X.device)
+    _check(emu_split_f64_rowcol(X.data_ptr(), rows, cols, X.stride(0), int(transpose), planes.data_ptr(), ldcomp,
+                                v.data_ptr(), ws.data_ptr(), ws.numel(), _stream(stream)), "emu_split_f64_rowcol")
+    return planes, v, ws
+
+
+def gemm_f64_rowcol(A, B, nprod: int, C=None, ws=None, stream=None):
+    """emu_gemm_f64_rowcol: Algorithm 2 with levels per row of A and per column of B."""
+    torch = _torch()
+    M, K = A.shape
+    N = B.shape[1]
+    C = C if C is not None else torch.empty((M, N), dtype=torch.float64, device=A.device)
+    ws = ws if ws is not None else workspace(emu_gemm_f64_rowcol_workspace_bytes(M, N, K), A.device)
+    _check(emu_gemm_f64_rowcol(M, N, K, A.data_ptr(), A.stride(0), B.data_ptr(), B.stride(0), C.data_ptr(),
+                               C.stride(0), int(nprod), ws.data_ptr(), ws.numel(), _stream(stream)),
+           "emu_gemm_f64_rowcol")
+    return C, ws
 
 
 def gemm_f32(A, B, C=None, ws=None, stream=None):

@@ -269,6 +269,71 @@ emu_status emu_gemm_ex_f64(int opA, int opB, int64_t M, int64_t N, int64_t K, do
                            reinterpret_cast<cudaStream_t>(stream));
 }
 
+size_t emu_split_f64_rowcol_workspace_bytes(int64_t plane_rows)
+{
+    if (plane_rows < 0) return 0;
+    return kWsHeaderBytes + (size_t)round_up(plane_rows * 8, 256);
+}
+
+emu_status emu_split_f64_rowcol(const double *X, int64_t rows, int64_t cols, int64_t ldx, int transpose,
+                                uint16_t *comps, int64_t ldcomp, int32_t *v_out, void *ws, size_t ws_bytes,
+                                emu_stream_t stream)
+{
+    if (rows < 0 || cols < 0 || ldx < (cols > 0 ? cols : 1) || !ws || !v_out) return EMU_ERR_INVALID_ARG;
+    const int64_t prow = transpose ? cols : rows;
+    if (ldcomp < (transpose ? rows : cols) || ldcomp < 1) return EMU_ERR_INVALID_ARG;
+    if (rows > 0 && cols > 0 && (!X || !comps)) return EMU_ERR_INVALID_ARG;
+    if (rows >= kMaxDim || cols >= kMaxDim) return EMU_ERR_UNSUPPORTED;
+    if (ws_bytes < emu_split_f64_rowcol_workspace_bytes(prow)) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
+    auto *maxbits = reinterpret_cast<unsigned long long *>(static_cast<char *>(ws) + kWsHeaderBytes);
+    if (e == cudaSuccess) e = launch_split_f64_rc(X, rows, cols, ldx, transpose != 0, comps, ldcomp, v_out, maxbits, h, st);
+    return cuda_status(e);
+}
+
+size_t emu_gemm_f64_rowcol_workspace_bytes(int64_t M, int64_t N, int64_t K)
+{
+    if (M < 0 || N < 0 || K < 0) return 0;
+    return gemm_ws_bytes(6, M, N, K) + (size_t)round_up(6 * (M + N) * 4, 256) +
+           (size_t)round_up((M > N ? M : N) * 8, 256);
+}
+
+emu_status emu_gemm_f64_rowcol(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda, const double *B,
+                               int64_t ldb, double *C, int64_t ldc, int nprod, void *ws, size_t ws_bytes,
+                               emu_stream_t stream)
+{
+    emu_status s = check_gemm_dims(M, N, K, lda, ldb, ldc);
+    if (s != EMU_OK) return s;
+    if (nprod != 6 && nprod != 10 && nprod != 15 && nprod != 21) return EMU_ERR_INVALID_ARG;
+    if (!ws || (M > 0 && N > 0 && (!C || (K > 0 && (!A || !B))))) return EMU_ERR_INVALID_ARG;
+    if (ws_bytes < emu_gemm_f64_rowcol_workspace_bytes(M, N, K)) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
+    if (e != cudaSuccess) return EMU_ERR_CUDA;
+    if (M == 0 || N == 0) return EMU_OK;
+    if (K == 0) return zero_c(C, M, N, ldc, st);
+    const int64_t ldk = gemm_ldk(K);
+    char *w = static_cast<char *>(ws);
+    uint16_t *Ap = reinterpret_cast<uint16_t *>(w + kWsHeaderBytes);
+    uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(6 * M * ldk * 2, 256));
+    char *tail = w + gemm_ws_bytes(6, M, N, K);                    // after the planes and the accumulator
+    int32_t *vA = reinterpret_cast<int32_t *>(tail);
+    int32_t *vB = vA + 6 * M;
+    auto *maxbits = reinterpret_cast<unsigned long long *>(tail + round_up(6 * (M + N) * 4, 256));
+    // A by rows (plane rows = rows of A), B by columns (plane rows = columns of B)
+    e = launch_split_f64_rc(A, M, K, lda, false, Ap, ldk, vA, maxbits, h, st);
+    if (e == cudaSuccess) e = launch_split_f64_rc(B, K, N, ldb, true, Bp, ldk, vB, maxbits, h, st);
+    if (e == cudaSuccess)
+        e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, vA, vB, nprod, C, ldc, gemm_acc(ws, M, N, K), &h->flags, st, 0,
+                               true);
+    return cuda_status(e);
+}
+
 emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acomps, const uint16_t *Bcomps,
                            int64_t ldcomp, float *C, int64_t ldc, void *ws, size_t ws_bytes, emu_stream_t stream)
 {

@@ -18,6 +18,13 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
                              uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
                              cudaStream_t st);
 
+// Eq. (fp64split) with one set of levels per plane row (an input row, or an
+// input column when transposed): v_out[6][plane rows] (level-major),
+// maxbits: scratch of 8 bytes per plane row.
+cudaError_t launch_split_f64_rc(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
+                                uint16_t *comps, int64_t ldcomp, int32_t *v_out, unsigned long long *maxbits,
+                                WsHeader *ws, cudaStream_t st);
+
 // Product-sums from K-major planes; a_plane: distance between the A planes in
 // elements (0 = dense: M * ldcomp), so that a row panel of a larger plane set
 // can be multiplied on its own.
@@ -25,9 +32,11 @@ cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *
                                int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
                                int64_t a_plane = 0);
 // acc: FP64 accumulator scratch of f64_acc_bytes(M, N) bytes (16-byte aligned).
+// rowcol: vA / vB are levels per row of A ([6][M]) and per column of B ([6][N]).
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
-                               int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane = 0);
+                               int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane = 0,
+                               bool rowcol = false);
 
 // Bytes of the FP64 product-sum's accumulator: one 128 x 128 FP64 tile per CTA tile.
 inline size_t f64_acc_bytes(int64_t M, int64_t N)

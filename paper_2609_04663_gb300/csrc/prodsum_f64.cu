@@ -114,14 +114,40 @@ __device__ __forceinline__ double widen_exact(float x)
 // exact.  0 (always take the error-free path, renormalising every time) when
 // the levels are unknown or the bound is not a normal float; +inf for a
 // product of an all-zero slice.
-__device__ __forceinline__ float exact_bound(const int32_t *vA, const int32_t *vB, int i, int j)
+__device__ __forceinline__ float bound_of_levels(int a, int b)
 {
-    if (!vA) return 0.0f;
-    const int a = vA[i], b = vB[j];
     if (a == kZeroLevel || b == kZeroLevel) return __int_as_float(0x7F800000);
     const int e = a + b + 8;                          // 2^24 * 2^(a + b - 16)
     if (e < -126 || e > 127) return 0.0f;
     return __int_as_float((e + 127) << 23);
+}
+
+__device__ __forceinline__ float exact_bound(const int32_t *vA, const int32_t *vB, int i, int j)
+{
+    if (!vA) return 0.0f;
+    return bound_of_levels(vA[i], vB[j]);
+}
+
+// The same bound with levels per row of A (vA[6][M]) and per column of B
+// (vB[6][N]), the vector scaling of Eq. (ozakiscaled): element (row, col) has
+// unit 2^(vA_i[row] + vB_j[col] - 16), so a thread summing columns col0 ..
+// col0 + ncols - 1 of one row may add plainly below 2^24 of the smallest of
+// its units (a column or row whose slice is all zero contributes nothing).
+__device__ __forceinline__ float exact_bound_rowcol(const int32_t *vA, const int32_t *vB, int M, int N, int i, int j,
+                                                    int row, int col0, int ncols)
+{
+    const int a = row < M ? vA[(int64_t)i * M + row] : kZeroLevel;
+    if (a == kZeroLevel) return __int_as_float(0x7F800000);
+    int bmin = 0x7FFFFFFF;
+    for (int c = 0; c < ncols; ++c) {
+        const int col = col0 + c;
+        if (col < N) {
+            const int b = vB[(int64_t)j * N + col];
+            if (b != kZeroLevel) bmin = b < bmin ? b : bmin;
+        }
+    }
+    if (bmin == 0x7FFFFFFF) return __int_as_float(0x7F800000);
+    return bound_of_levels(a, bmin);
 }
 
 // 16 consecutive 32-bit TMEM columns of this thread's lane: load / store.
@@ -180,7 +206,7 @@ __device__ __forceinline__ float two_sum(float a, float b, float &e)
     return s;
 }
 
-template <int NPROD>
+template <int NPROD, bool ROWCOL>
 __global__ void __launch_bounds__(F64Cfg::THREADS, 1)
 prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    int M, int N, int K, const int32_t *__restrict__ vA, const int32_t *__restrict__ vB,
@@ -297,7 +323,9 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
 #pragma unroll
             for (int j = 0; j < Cfg::COLS; ++j) hi[j] = 0.0f;
             uint32_t dirty = 0;                           // 16-column groups whose low part lives in C
-            const float bound = exact_bound(vA, vB, kDiag[q][0], kDiag[q][1]);
+            const float bound = ROWCOL ? exact_bound_rowcol(vA, vB, M, N, kDiag[q][0], kDiag[q][1], row,
+                                                            n0 + cq * Cfg::COLS, Cfg::COLS)
+                                       : exact_bound(vA, vB, kDiag[q][0], kDiag[q][1]);
             for (int c = 0; c < nch; ++c) {
                 const int t = q * nch + c, b = t % Cfg::NBUF;
                 ok = mbar_wait(tfull0 + 8u * b, (uint32_t)((t / Cfg::NBUF) & 1), flags);
@@ -441,7 +469,7 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     }
 }
 
-template <int NPROD>
+template <int NPROD, bool ROWCOL>
 cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
                     const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, double *acc, uint32_t *flags,
                     cudaStream_t st, int64_t a_plane)
@@ -450,7 +478,7 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
     CUtensorMap ta, tb;
     if (!make_plane_map(&ta, Ap, K, M, 6, ldcomp, Cfg::KB, kBM, a_plane) || !make_plane_map(&tb, Bp, K, N, 6, ldcomp, Cfg::KB, Cfg::BN))
         return cudaErrorInvalidValue;
-    auto kern = prodsum_f64_kernel<NPROD>;
+    auto kern = prodsum_f64_kernel<NPROD, ROWCOL>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
     const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + Cfg::BN - 1) / Cfg::BN);
@@ -462,13 +490,18 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
 
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
-                               int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane)
+                               int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
+                               bool rowcol)
 {
     switch (nprod) {
-    case 6: return run_f64<6>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
-    case 10: return run_f64<10>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
-    case 15: return run_f64<15>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
-    case 21: return run_f64<21>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
+    case 6: return rowcol ? run_f64<6, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane)
+                   : run_f64<6, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
+    case 10: return rowcol ? run_f64<10, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane)
+                   : run_f64<10, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
+    case 15: return rowcol ? run_f64<15, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane)
+                   : run_f64<15, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
+    case 21: return rowcol ? run_f64<21, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane)
+                   : run_f64<21, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
     default: return cudaErrorInvalidValue;
     }
 }

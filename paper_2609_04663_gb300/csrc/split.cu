@@ -278,33 +278,29 @@ __device__ __forceinline__ void block_max_to(unsigned long long x, unsigned long
 }
 
 // ------------------------------------------------------------ tile kernel
-// FP64 split.  MODE 1: speculative split (v^(r) = v0 - 8r,
-// records the maxima of |A^(r)|, r = 1..5).  MODE 2: FP64 rewrite with the
-// final levels (runs only when verification failed).  (T is double.)
+// Literal FP64 plane pass (T is double).  MODE 2: rewrite with the final
+// whole-matrix levels (runs only when verification failed).  MODE 3: levels
+// per plane row (per input row, or per input column when transposed), read
+// from vrc[6][plane rows].
 template <typename T, int MODE, bool TRANSPOSE>
 __global__ void __launch_bounds__(kThreads)
 split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
-                  uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
+                  uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot,
+                  const int32_t *__restrict__ vrc)
 {
-    static_assert(MODE == 1 || MODE == 2, "FP64 split modes only");
+    static_assert(MODE == 2 || MODE == 3, "literal FP64 split modes only");
     constexpr int NS = 6;
     extern __shared__ __align__(16) uint16_t smdyn[];    // [NS][kTile][kSRow]
     auto sm = [&](int r, int row, int col) -> uint16_t & {
         return smdyn[((size_t)r * kTile + row) * kSRow + col];
     };
-    __shared__ unsigned long long red[kThreads / 32];
 
     int v[6] = {0, 0, 0, 0, 0, 0};
-    if constexpr (MODE == 1) {
-        const unsigned long long m0 = ws->maxbits[slot][0];
-        const int v0 = m0 ? ceil_log2_bits(m0) : kZeroLevel;
-        for (int r = 0; r < 6; ++r) v[r] = (v0 == kZeroLevel) ? kZeroLevel : v0 - 8 * r;
-    } else if constexpr (MODE == 2) {
+    if constexpr (MODE == 2) {
         if (ws->fix_from[slot] >= 6) return;     // speculation held: nothing to redo
         final_levels(ws, slot, 6, v);
     }
-
-    unsigned long long mx[5] = {0, 0, 0, 0, 0};         // max |A^(r)| as bit patterns
+    const int64_t nvec = TRANSPOSE ? cols : rows;        // plane rows (MODE 3's level vectors)
     uint32_t badmask = 0;
     const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;   // 16 x 16 threads
@@ -337,21 +333,21 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
             for (int e = 0; e < 4; ++e) {
                 const int lj = 4 * tx + e;
                 uint16_t s[NS];
-                if constexpr (MODE == 1) {
-                    if (v[0] == kZeroLevel) {
+                int vv[6];
+                if constexpr (MODE == 3) {
+                    const int64_t vec = TRANSPOSE ? c0 + lj : gi;
 #pragma unroll
-                        for (int r = 0; r < 6; ++r) s[r] = 0;
-                    } else {
-                        spec_levels(x[e], v[0], s, badmask, mx);
-                    }
+                    for (int r = 0; r < 6; ++r) vv[r] = vec < nvec ? vrc[r * nvec + vec] : kZeroLevel;
                 } else {
-                    double R = x[e];
 #pragma unroll
-                    for (int r = 0; r < 6; ++r) {
-                        bool bad = false;
-                        s[r] = f64_level_int(R, v[r], bad);
-                        if (bad) badmask |= 1u << r;
-                    }
+                    for (int r = 0; r < 6; ++r) vv[r] = v[r];
+                }
+                double R = x[e];
+#pragma unroll
+                for (int r = 0; r < 6; ++r) {
+                    bool bad = false;
+                    s[r] = f64_level_int(R, vv[r], bad);
+                    if (bad) badmask |= 1u << r;
                 }
 #pragma unroll
                 for (int r = 0; r < NS; ++r) {
@@ -382,15 +378,9 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
     }
 
     badmask = __reduce_or_sync(0xFFFFFFFFu, badmask);
-    if (badmask && lane_id() == 0) atomicOr(&ws->slice_bad[slot], MODE == 1 ? badmask : badmask << 8);
-    if constexpr (MODE == 1) {
-        // mx holds |A^(r)| in units of 2^(v0 - 50), below 2^53: exact as doubles
-        const int F = (v[0] == kZeroLevel) ? 0 : v[0] - 50;
-#pragma unroll
-        for (int r = 0; r < 5; ++r) {
-            const double m = (double)mx[r] * pow2_d(F);
-            block_max_to((unsigned long long)__double_as_longlong(m), &ws->maxbits[slot][r + 1], red);
-        }
+    if (badmask && lane_id() == 0) {
+        if constexpr (MODE == 2) atomicOr(&ws->slice_bad[slot], badmask << 8);
+        else atomicOr(&ws->flags, (uint32_t)EMU_FLAG_SLICE);
     }
 }
 
@@ -924,6 +914,77 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
     publish_f32_flags(amax, ws);
 }
 
+// ------------------------------ FP64 split with levels per row / per column
+// The vector scaling of Eq. (ozakiscaled): each plane row (an input row, or
+// an input column when the planes are transposed) gets its own six levels
+// v^(r) = ceil(log2 max |X^(r)|) over that vector.  Literal form: level L's
+// maxima come from a pass that recomputes levels 0 .. L-1 from x with the
+// vector's final levels; a one-thread-per-vector kernel turns them into
+// v[L][vector]; the tile kernel (MODE 3) then writes all six planes.
+
+// Max |X^(L)| per vector.  Not transposed: one warp per row, lanes striding
+// along it.  Transposed: one thread per column over a range of rows, the
+// block's columns contiguous, maxima merged with atomicMax.  Level 0 also
+// checks the input domain of Eq. (bf16rangefp64).
+template <bool TRANSPOSE>
+__global__ void __launch_bounds__(kThreads)
+rc_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, int L,
+              const int32_t *__restrict__ vrc, unsigned long long *maxbits, int64_t rows_per_block, WsHeader *ws)
+{
+    constexpr unsigned long long kLo = 0x3810000000000000ull, kHi = 0x47EFE00000000000ull;
+    constexpr unsigned long long kInf = 0x7FF0000000000000ull;
+    const int64_t nvec = TRANSPOSE ? cols : rows;
+    uint32_t flagbits = 0;
+    auto take = [&](double R, const int (&v)[6], unsigned long long &m) {
+        bool bad = false;
+        for (int l = 0; l < L; ++l) (void)f64_level_int(R, v[l], bad);
+        const unsigned long long ab = (unsigned long long)__double_as_longlong(R) & 0x7FFFFFFFFFFFFFFFull;
+        if (L == 0) {
+            if (ab >= kInf) flagbits |= EMU_FLAG_NONFINITE;
+            else if (ab != 0 && (ab < kLo || ab > kHi)) flagbits |= EMU_FLAG_RANGE;
+            if (ab <= kInf) m = ab > m ? ab : m;                      // NaN never wins
+        } else {
+            m = ab > m ? ab : m;
+        }
+    };
+    int v[6] = {0, 0, 0, 0, 0, 0};
+    if (!TRANSPOSE) {
+        const int64_t nwarps = (int64_t)gridDim.x * (kThreads / 32);
+        for (int64_t i = (int64_t)blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5); i < rows; i += nwarps) {
+            for (int l = 0; l < L; ++l) v[l] = vrc[l * nvec + i];
+            unsigned long long m = 0;
+            for (int64_t j = lane_id(); j < cols; j += 32) take(X[i * ldx + j], v, m);
+            m = warp_max(m);
+            if (lane_id() == 0) maxbits[i] = m;
+        }
+    } else {
+        const int64_t j = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+        const int64_t i0 = (int64_t)blockIdx.y * rows_per_block;
+        const int64_t i1 = i0 + rows_per_block < rows ? i0 + rows_per_block : rows;
+        if (j < cols) {
+            for (int l = 0; l < L; ++l) v[l] = vrc[l * nvec + j];
+            unsigned long long m = 0;
+            for (int64_t i = i0; i < i1; ++i) take(X[i * ldx + j], v, m);
+            if (m) atomicMax(&maxbits[j], m);
+        }
+    }
+    flagbits = __reduce_or_sync(0xFFFFFFFFu, flagbits);
+    if (flagbits && lane_id() == 0) atomicOr(&ws->flags, flagbits);
+}
+
+// v[L][vector] from the maxima of level L; a vector whose previous level was
+// already zero stays zero (Section 4.3's early stop).  Clears the maxima.
+__global__ void rc_levels_kernel(int L, unsigned long long *maxbits, int32_t *vrc, int64_t nvec)
+{
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += (int64_t)gridDim.x * blockDim.x) {
+        const unsigned long long m = maxbits[i];
+        int v = m ? ceil_log2_bits(m) : kZeroLevel;
+        if (L > 0 && vrc[(L - 1) * nvec + i] == kZeroLevel) v = kZeroLevel;
+        vrc[L * nvec + i] = v;
+        maxbits[i] = 0;
+    }
+}
+
 constexpr size_t kSpecTransposeSmem = 6 * kTile * (kTile / 2) * sizeof(uint32_t);
 
 size_t smem_bytes(int ns) { return (size_t)ns * kTile * kSRow * sizeof(uint16_t); }
@@ -994,13 +1055,62 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
         f64_max_kernel<4><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
         f64_max_kernel<5><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
         if (transpose)
-            split_tile_kernel<double, 2, true><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot);
+            split_tile_kernel<double, 2, true><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, nullptr);
         else
-            split_tile_kernel<double, 2, false><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot);
+            split_tile_kernel<double, 2, false><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, nullptr);
     } else {
         f64_verify_kernel<<<1, 1, 0, st>>>(ws, slot);
     }
     f64_finalize_kernel<<<1, 1, 0, st>>>(ws, slot, v_out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_split_f64_rc(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
+                                uint16_t *comps, int64_t ldcomp, int32_t *v_out, unsigned long long *maxbits,
+                                WsHeader *ws, cudaStream_t st)
+{
+    const int64_t nvec = transpose ? cols : rows;
+    const int64_t plane = nvec * ldcomp;
+    if (rows == 0 || cols == 0) {
+        if (nvec == 0) return cudaSuccess;
+        // an empty vector has no nonzero entry: every level is zero
+        cudaError_t e = cudaMemsetAsync(maxbits, 0, (size_t)nvec * 8, st);
+        for (int L = 0; L < 6 && e == cudaSuccess; ++L) {
+            rc_levels_kernel<<<grid_for((nvec + 255) / 256, 152 * 4), 256, 0, st>>>(L, maxbits, v_out, nvec);
+            e = cudaGetLastError();
+        }
+        return e;
+    }
+    const size_t sm = smem_bytes(6);
+    cudaError_t e = transpose
+        ? cudaFuncSetAttribute(split_tile_kernel<double, 3, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm)
+        : cudaFuncSetAttribute(split_tile_kernel<double, 3, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e == cudaSuccess) e = cudaMemsetAsync(maxbits, 0, (size_t)nvec * 8, st);
+    const int lgrid = grid_for((nvec + 255) / 256, 152 * 4);
+    for (int L = 0; L < 6 && e == cudaSuccess; ++L) {
+        if (transpose) {
+            // blocks of 256 columns, each over a range of rows: about eight blocks per SM
+            const int64_t bx = (cols + kThreads - 1) / kThreads;
+            int64_t by = (152 * 8 + bx - 1) / bx;
+            by = by < rows ? by : rows;
+            by = by < 65535 ? by : 65535;
+            const int64_t rpb = (rows + by - 1) / by;
+            rc_max_kernel<true><<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, L, v_out,
+                                                                                     maxbits, rpb, ws);
+        } else {
+            rc_max_kernel<false><<<grid_for((rows + 7) / 8, 152 * 8), kThreads, 0, st>>>(X, rows, cols, ldx, L, v_out,
+                                                                                        maxbits, 0, ws);
+        }
+        rc_levels_kernel<<<lgrid, 256, 0, st>>>(L, maxbits, v_out, nvec);
+        e = cudaGetLastError();
+    }
+    if (e != cudaSuccess) return e;
+    const int64_t tiles = ((rows + kTile - 1) / kTile) * ((cols + kTile - 1) / kTile);
+    const int gt = grid_for(tiles, 152 * 8);
+    if (transpose)
+        split_tile_kernel<double, 3, true><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, 0, v_out);
+    else
+        split_tile_kernel<double, 3, false><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, 0, v_out);
     return cudaGetLastError();
 }
 

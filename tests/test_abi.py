@@ -106,3 +106,14 @@ def test_prodsum_workspace_sizes_and_check(lib):
     P = 16
     small = emu.emu_split_workspace_bytes(64)
     assert emu.emu_prodsum_f64(300, 200, 64, P, P, 64, P, P, 6, P, 200, P, small, None) == 3
+
+
+def test_rowcol_argument_checks_need_no_gpu(lib):
+    P = 16
+    assert emu.emu_split_f64_rowcol_workspace_bytes(100) == emu.emu_split_workspace_bytes(64) + 1024
+    assert emu.emu_split_f64_rowcol(P, 100, 8, 8, 0, P, 8, P, P, 600, None) == 3           # workspace
+    assert emu.emu_split_f64_rowcol(P, 100, 8, 8, 0, P, 8, 0, P, 1 << 20, None) == 1       # no v_out
+    need = emu.emu_gemm_f64_rowcol_workspace_bytes(300, 200, 700)
+    assert need > emu.emu_gemm_workspace_bytes(64, 300, 200, 700)
+    assert emu.emu_gemm_f64_rowcol(300, 200, 700, P, 700, P, 200, P, 200, 6, P, need - 1, None) == 3
+    assert emu.emu_gemm_f64_rowcol(4, 4, 4, P, 4, P, 4, P, 4, 11, P, 1 << 30, None) == 1      # nprod
