@@ -17,7 +17,7 @@ namespace emu {
 // GEMM workspace continues with the A planes, then the B planes.
 struct WsHeader {
     uint32_t flags;                       // EMU_FLAG_* of the current call
-    uint32_t pad0;
+    uint32_t fix_any;                     // split with per-vector levels: some vector needs the literal passes
     unsigned long long maxbits[2][6];     // speculative-pass maxima |A^(r)| (FP64 bits)
     unsigned long long fixmax[2][6];      // maxima of the fix passes
     int32_t v[2][6];                      // final level exponents

@@ -272,7 +272,7 @@ emu_status emu_gemm_ex_f64(int opA, int opB, int64_t M, int64_t N, int64_t K, do
 size_t emu_split_f64_rowcol_workspace_bytes(int64_t plane_rows)
 {
     if (plane_rows < 0) return 0;
-    return kWsHeaderBytes + (size_t)round_up(plane_rows * 8, 256);
+    return kWsHeaderBytes + (size_t)round_up((int64_t)rc_scratch_bytes(plane_rows), 256);
 }
 
 emu_status emu_split_f64_rowcol(const double *X, int64_t rows, int64_t cols, int64_t ldx, int transpose,
@@ -289,8 +289,8 @@ emu_status emu_split_f64_rowcol(const double *X, int64_t rows, int64_t cols, int
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     WsHeader *h = static_cast<WsHeader *>(ws);
     cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
-    auto *maxbits = reinterpret_cast<unsigned long long *>(static_cast<char *>(ws) + kWsHeaderBytes);
-    if (e == cudaSuccess) e = launch_split_f64_rc(X, rows, cols, ldx, transpose != 0, comps, ldcomp, v_out, maxbits, h, st);
+    void *scratch = static_cast<char *>(ws) + kWsHeaderBytes;
+    if (e == cudaSuccess) e = launch_split_f64_rc(X, rows, cols, ldx, transpose != 0, comps, ldcomp, v_out, scratch, h, 0, st);
     return cuda_status(e);
 }
 
@@ -298,7 +298,7 @@ size_t emu_gemm_f64_rowcol_workspace_bytes(int64_t M, int64_t N, int64_t K)
 {
     if (M < 0 || N < 0 || K < 0) return 0;
     return gemm_ws_bytes(6, M, N, K) + (size_t)round_up(6 * (M + N) * 4, 256) +
-           (size_t)round_up((M > N ? M : N) * 8, 256);
+           (size_t)round_up((int64_t)rc_scratch_bytes(M > N ? M : N), 256);
 }
 
 emu_status emu_gemm_f64_rowcol(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda, const double *B,
@@ -324,10 +324,11 @@ emu_status emu_gemm_f64_rowcol(int64_t M, int64_t N, int64_t K, const double *A,
     char *tail = w + gemm_ws_bytes(6, M, N, K);                    // after the planes and the accumulator
     int32_t *vA = reinterpret_cast<int32_t *>(tail);
     int32_t *vB = vA + 6 * M;
-    auto *maxbits = reinterpret_cast<unsigned long long *>(tail + round_up(6 * (M + N) * 4, 256));
-    // A by rows (plane rows = rows of A), B by columns (plane rows = columns of B)
-    e = launch_split_f64_rc(A, M, K, lda, false, Ap, ldk, vA, maxbits, h, st);
-    if (e == cudaSuccess) e = launch_split_f64_rc(B, K, N, ldb, true, Bp, ldk, vB, maxbits, h, st);
+    void *scratch = tail + round_up(6 * (M + N) * 4, 256);
+    // A by rows (plane rows = rows of A), B by columns (plane rows = columns of B);
+    // the two splits run in order on the stream and share the scratch
+    e = launch_split_f64_rc(A, M, K, lda, false, Ap, ldk, vA, scratch, h, 0, st);
+    if (e == cudaSuccess) e = launch_split_f64_rc(B, K, N, ldb, true, Bp, ldk, vB, scratch, h, 1, st);
     if (e == cudaSuccess)
         e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, vA, vB, nprod, C, ldc, gemm_acc(ws, M, N, K), &h->flags, st, 0,
                                true);

@@ -19,11 +19,13 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
                              cudaStream_t st);
 
 // Eq. (fp64split) with one set of levels per plane row (an input row, or an
-// input column when transposed): v_out[6][plane rows] (level-major),
-// maxbits: scratch of 8 bytes per plane row.
+// input column when transposed): v_out[6][plane rows] (level-major);
+// scratch: rc_scratch_bytes(plane rows) bytes, 8-byte aligned; slot: the
+// header's per-operand state (0 = A, 1 = B).
 cudaError_t launch_split_f64_rc(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
-                                uint16_t *comps, int64_t ldcomp, int32_t *v_out, unsigned long long *maxbits,
-                                WsHeader *ws, cudaStream_t st);
+                                uint16_t *comps, int64_t ldcomp, int32_t *v_out, void *scratch, WsHeader *ws,
+                                int slot, cudaStream_t st);
+inline size_t rc_scratch_bytes(int64_t plane_rows) { return (size_t)plane_rows * 28; }
 
 // Product-sums from K-major planes; a_plane: distance between the A planes in
 // elements (0 = dense: M * ldcomp), so that a row panel of a larger plane set

@@ -286,7 +286,7 @@ template <typename T, int MODE, bool TRANSPOSE>
 __global__ void __launch_bounds__(kThreads)
 split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
                   uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot,
-                  const int32_t *__restrict__ vrc)
+                  const int32_t *__restrict__ vrc, const int32_t *__restrict__ ff)
 {
     static_assert(MODE == 2 || MODE == 3, "literal FP64 split modes only");
     constexpr int NS = 6;
@@ -301,6 +301,10 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
         final_levels(ws, slot, 6, v);
     }
     const int64_t nvec = TRANSPOSE ? cols : rows;        // plane rows (MODE 3's level vectors)
+    // MODE 3 rewrites only the vectors whose speculative levels failed (ff < 6)
+    if constexpr (MODE == 3) {
+        if (ws->fix_any == 0) return;
+    }
     uint32_t badmask = 0;
     const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;   // 16 x 16 threads
@@ -366,6 +370,7 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
             const int orow = rem / (kTile / 8), ch = rem % (kTile / 8);
             const int64_t go = orow0 + orow, gc = ocol0 + 8 * ch;
             if (go >= orows || gc >= ocols) continue;
+            if (MODE == 3 && ff[go] >= 6) continue;
             uint16_t *dst = comps + r * plane + go * ldcomp + gc;
             const uint32_t *w = reinterpret_cast<const uint32_t *>(&sm(r, orow, 8 * ch));
             if (gc + 8 <= ocols && ((reinterpret_cast<uintptr_t>(dst) & 15u) == 0)) {
@@ -929,8 +934,12 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
 template <bool TRANSPOSE>
 __global__ void __launch_bounds__(kThreads)
 rc_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, int L,
-              const int32_t *__restrict__ vrc, unsigned long long *maxbits, int64_t rows_per_block, WsHeader *ws)
+              const int32_t *__restrict__ vrc, unsigned long long *maxbits, int64_t rows_per_block, WsHeader *ws,
+              const int32_t *__restrict__ ff)
 {
+    // ff (fix passes only): levels <= ff[vector] are final; nothing to do for
+    // vectors with ff >= L, and nothing at all unless some vector failed
+    if (ff && ws->fix_any == 0) return;
     constexpr unsigned long long kLo = 0x3810000000000000ull, kHi = 0x47EFE00000000000ull;
     constexpr unsigned long long kInf = 0x7FF0000000000000ull;
     const int64_t nvec = TRANSPOSE ? cols : rows;
@@ -951,6 +960,7 @@ rc_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t 
     if (!TRANSPOSE) {
         const int64_t nwarps = (int64_t)gridDim.x * (kThreads / 32);
         for (int64_t i = (int64_t)blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5); i < rows; i += nwarps) {
+            if (ff && ff[i] >= L) continue;
             for (int l = 0; l < L; ++l) v[l] = vrc[l * nvec + i];
             unsigned long long m = 0;
             for (int64_t j = lane_id(); j < cols; j += 32) take(X[i * ldx + j], v, m);
@@ -961,7 +971,7 @@ rc_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t 
         const int64_t j = (int64_t)blockIdx.x * kThreads + threadIdx.x;
         const int64_t i0 = (int64_t)blockIdx.y * rows_per_block;
         const int64_t i1 = i0 + rows_per_block < rows ? i0 + rows_per_block : rows;
-        if (j < cols) {
+        if (j < cols && !(ff && ff[j] >= L)) {
             for (int l = 0; l < L; ++l) v[l] = vrc[l * nvec + j];
             unsigned long long m = 0;
             for (int64_t i = i0; i < i1; ++i) take(X[i * ldx + j], v, m);
@@ -974,14 +984,206 @@ rc_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t 
 
 // v[L][vector] from the maxima of level L; a vector whose previous level was
 // already zero stays zero (Section 4.3's early stop).  Clears the maxima.
-__global__ void rc_levels_kernel(int L, unsigned long long *maxbits, int32_t *vrc, int64_t nvec)
+__global__ void rc_levels_kernel(int L, unsigned long long *maxbits, int32_t *vrc, int64_t nvec, const int32_t *ff,
+                                 const WsHeader *ws)
 {
+    if (ff && ws->fix_any == 0) return;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += (int64_t)gridDim.x * blockDim.x) {
+        if (ff && ff[i] >= L) continue;
         const unsigned long long m = maxbits[i];
         int v = m ? ceil_log2_bits(m) : kZeroLevel;
         if (L > 0 && vrc[(L - 1) * nvec + i] == kZeroLevel) v = kZeroLevel;
         vrc[L * nvec + i] = v;
         maxbits[i] = 0;
+    }
+}
+
+// Speculative pass with per-vector levels: each element is split with its
+// vector's v0 (level 0 is literal) under the assumption v^(r) = v0 - 8r, as
+// in the whole-matrix speculative pass; the magnitudes |X^(r)| before levels
+// 1 .. 5 are reduced per vector into vmax[5][vectors] (32-bit: levels 1 and
+// 2 in units of 2^(F + 20) with a sticky last bit, levels 3 .. 5 exact in
+// units of 2^F, F = v0 - 50).
+__device__ __forceinline__ uint32_t jam20(unsigned long long m)
+{
+    return (uint32_t)(m >> 20) | ((m & 0xFFFFFull) != 0 ? 1u : 0u);
+}
+
+__device__ __forceinline__ void spec_element_mags(double x, int v0, uint32_t (&s)[6], uint32_t &badmask,
+                                                  uint32_t (&mag)[5])
+{
+    SpecState st;
+    spec_element(x, v0, v0 >= -78, s, st);
+    badmask |= st.badmask;
+    mag[0] = jam20(st.m1);
+    mag[1] = jam20(st.m2);
+    mag[2] = st.m[0];
+    mag[3] = st.m[1];
+    mag[4] = st.m[2];
+}
+
+// Row-major planes, levels per row: thread = 4 consecutive entries of a row.
+__global__ void __launch_bounds__(kThreads)
+rc_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                    uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, const int32_t *__restrict__ vrc,
+                    uint32_t *vmax, WsHeader *ws, int slot)
+{
+    const bool vin = ((ldx & 1) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
+    const bool vout = ((ldcomp & 3) == 0) && ((plane & 3) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 7u) == 0);
+    const int64_t j0 = ((int64_t)blockIdx.x * kThreads + threadIdx.x) * 4;
+    const bool full = j0 + 4 <= cols;
+    uint32_t badmask = 0;
+    for (int64_t i = blockIdx.y; i < rows; i += gridDim.y) {
+        const int v0 = vrc[i];
+        uint32_t mx[5] = {0, 0, 0, 0, 0};
+        if (j0 < cols) {
+            const double *src = X + i * ldx + j0;
+            double x[4];
+            if (vin && full) {
+                const double2 a = reinterpret_cast<const double2 *>(src)[0], c = reinterpret_cast<const double2 *>(src)[1];
+                x[0] = a.x; x[1] = a.y; x[2] = c.x; x[3] = c.y;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) x[e] = (j0 + e < cols) ? src[e] : 0.0;
+            }
+            uint32_t w[6][2] = {};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                uint32_t sl[6], mag[5];
+                spec_element_mags(x[e], v0, sl, badmask, mag);
+#pragma unroll
+                for (int r = 0; r < 5; ++r) mx[r] = mag[r] > mx[r] ? mag[r] : mx[r];
+#pragma unroll
+                for (int r = 0; r < 6; ++r) w[r][e >> 1] |= sl[r] << (16 * (e & 1));
+            }
+            uint16_t *dst = comps + i * ldcomp + j0;
+#pragma unroll
+            for (int r = 0; r < 6; ++r) {
+                if (vout && full) {
+                    *reinterpret_cast<uint2 *>(dst + r * plane) = make_uint2(w[r][0], w[r][1]);
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        if (j0 + e < cols) dst[r * plane + e] = (uint16_t)(w[r][e >> 1] >> (16 * (e & 1)));
+                }
+            }
+        }
+#pragma unroll
+        for (int r = 0; r < 5; ++r) {
+            const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, mx[r]);
+            if (lane_id() == 0 && m) atomicMax(&vmax[r * rows + i], m);
+        }
+    }
+    badmask = __reduce_or_sync(0xFFFFFFFFu, badmask);
+    if (badmask && lane_id() == 0) atomicOr(&ws->slice_bad[slot], badmask);
+}
+
+// Transposed planes, levels per column: the 64 x 64 tile of the whole-matrix
+// transposed pass; each warp reduces its 8 columns' magnitudes over its 64 rows.
+__global__ void __launch_bounds__(kThreads)
+rc_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                         uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane,
+                         const int32_t *__restrict__ vrc, uint32_t *vmax, WsHeader *ws, int slot)
+{
+    extern __shared__ __align__(16) uint32_t smw[];                  // [6][kTile][kTile / 2]
+    const bool vin = ((ldx & 1) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
+    const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
+    const int q = threadIdx.x >> 5, p = lane_id();
+    const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
+    uint32_t badmask = 0;
+    for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
+        const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
+        const int64_t gj = c0 + 8 * q;
+        double x[2][8];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int64_t gi = r0 + 2 * p + h;
+            const double *src = X + gi * ldx + gj;
+            if (gi < rows && vin && gj + 8 <= cols) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const double2 a = reinterpret_cast<const double2 *>(src)[k];
+                    x[h][2 * k] = a.x; x[h][2 * k + 1] = a.y;
+                }
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) x[h][e] = (gi < rows && gj + e < cols) ? src[e] : 0.0;
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int64_t col = gj + e;
+            const int v0 = col < cols ? vrc[col] : kZeroLevel;
+            uint32_t s0[6], s1[6], m0[5], m1[5];
+            spec_element_mags(x[0][e], v0, s0, badmask, m0);
+            spec_element_mags(x[1][e], v0, s1, badmask, m1);
+#pragma unroll
+            for (int r = 0; r < 6; ++r) smw[(r * kTile + 8 * q + e) * (kTile / 2) + p] = s0[r] | (s1[r] << 16);
+#pragma unroll
+            for (int r = 0; r < 5; ++r) {
+                const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, m0[r] > m1[r] ? m0[r] : m1[r]);
+                if (p == 0 && m && col < cols) atomicMax(&vmax[r * cols + col], m);
+            }
+        }
+        __syncthreads();
+#pragma unroll 4
+        for (int it = 0; it < 6 * kTile * 8 / kThreads; ++it) {
+            const int c = threadIdx.x + it * kThreads;
+            const int r = c >> 9, orow = (c >> 3) & 63, ch = c & 7;
+            const int64_t go = c0 + orow, gk = r0 + 8 * ch;
+            if (go < cols && gk < rows) {
+                const uint4 v = *reinterpret_cast<const uint4 *>(&smw[(r * kTile + orow) * (kTile / 2) + 4 * ch]);
+                uint16_t *dst = comps + r * plane + go * ldcomp + gk;
+                if (vout && gk + 8 <= rows) {
+                    *reinterpret_cast<uint4 *>(dst) = v;
+                } else {
+                    const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        if (gk + e < rows) dst[e] = (uint16_t)(wv[e >> 1] >> (16 * (e & 1)));
+                }
+            }
+        }
+        __syncthreads();
+    }
+    badmask = __reduce_or_sync(0xFFFFFFFFu, badmask);
+    if (badmask && lane_id() == 0) atomicOr(&ws->slice_bad[slot], badmask);
+}
+
+__device__ __forceinline__ int ceil_log2_u32(uint32_t m) { return m <= 1u ? 0 : 32 - __clz(m - 1u); }
+
+// One thread per vector: checks its speculative levels in order.  A level
+// that matches v0 - 8r is final (the 32-bit maxima decide matches exactly);
+// at the first mismatch r the literal passes redo levels r .. 5 (ff = r - 1:
+// levels up to ff are final).  A residual that became zero ends the vector
+// (literal as long as the levels before were right).  A slice outside the
+// BF16 range (or a non-finite input) anywhere in the operand sends every
+// vector to the literal passes, which flag such slices as Eq. (fp64split)
+// computes them.
+__global__ void rc_verify_kernel(const uint32_t *vmax, int32_t *vrc, int32_t *ff, int64_t nvec, WsHeader *ws, int slot)
+{
+    const bool fix_all = (ws->slice_bad[slot] & 0x3Fu) != 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += (int64_t)gridDim.x * blockDim.x) {
+        const int v0 = vrc[i];
+        int f = 6;
+        if (v0 == kZeroLevel) {
+            for (int r = 1; r < 6; ++r) vrc[r * nvec + i] = kZeroLevel;
+        } else if (fix_all) {
+            f = 0;
+        } else {
+            const int F = v0 - 50;
+            bool zero = false;
+            for (int r = 1; r < 6; ++r) {
+                if (zero) { vrc[r * nvec + i] = kZeroLevel; continue; }
+                const uint32_t m = vmax[(r - 1) * nvec + i];
+                if (m == 0) { vrc[r * nvec + i] = kZeroLevel; zero = true; continue; }
+                const int vr = ceil_log2_u32(m) + F + (r <= 2 ? 20 : 0);
+                if (vr != v0 - 8 * r) { f = r - 1; break; }
+                vrc[r * nvec + i] = vr;
+            }
+        }
+        ff[i] = f;
+        if (f < 6) atomicOr(&ws->fix_any, 1u);
     }
 }
 
@@ -1055,9 +1257,9 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
         f64_max_kernel<4><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
         f64_max_kernel<5><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
         if (transpose)
-            split_tile_kernel<double, 2, true><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, nullptr);
+            split_tile_kernel<double, 2, true><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, nullptr, nullptr);
         else
-            split_tile_kernel<double, 2, false><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, nullptr);
+            split_tile_kernel<double, 2, false><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, nullptr, nullptr);
     } else {
         f64_verify_kernel<<<1, 1, 0, st>>>(ws, slot);
     }
@@ -1066,51 +1268,71 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
 }
 
 cudaError_t launch_split_f64_rc(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
-                                uint16_t *comps, int64_t ldcomp, int32_t *v_out, unsigned long long *maxbits,
-                                WsHeader *ws, cudaStream_t st)
+                                uint16_t *comps, int64_t ldcomp, int32_t *v_out, void *scratch, WsHeader *ws,
+                                int slot, cudaStream_t st)
 {
     const int64_t nvec = transpose ? cols : rows;
     const int64_t plane = nvec * ldcomp;
+    // scratch: literal maxima [nvec] u64, speculative maxima [5][nvec] u32, ff [nvec] i32
+    auto *maxbits = static_cast<unsigned long long *>(scratch);
+    auto *vmax = reinterpret_cast<uint32_t *>(maxbits + nvec);
+    int32_t *ff = reinterpret_cast<int32_t *>(vmax + 5 * nvec);
+    if (nvec == 0) return cudaSuccess;
+    const int lgrid = grid_for((nvec + 255) / 256, 152 * 4);
+    cudaError_t e = cudaMemsetAsync(scratch, 0, (size_t)nvec * (8 + 20), st);
     if (rows == 0 || cols == 0) {
-        if (nvec == 0) return cudaSuccess;
         // an empty vector has no nonzero entry: every level is zero
-        cudaError_t e = cudaMemsetAsync(maxbits, 0, (size_t)nvec * 8, st);
         for (int L = 0; L < 6 && e == cudaSuccess; ++L) {
-            rc_levels_kernel<<<grid_for((nvec + 255) / 256, 152 * 4), 256, 0, st>>>(L, maxbits, v_out, nvec);
+            rc_levels_kernel<<<lgrid, 256, 0, st>>>(L, maxbits, v_out, nvec, nullptr, ws);
             e = cudaGetLastError();
         }
         return e;
     }
     const size_t sm = smem_bytes(6);
-    cudaError_t e = transpose
-        ? cudaFuncSetAttribute(split_tile_kernel<double, 3, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm)
-        : cudaFuncSetAttribute(split_tile_kernel<double, 3, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-    if (e == cudaSuccess) e = cudaMemsetAsync(maxbits, 0, (size_t)nvec * 8, st);
-    const int lgrid = grid_for((nvec + 255) / 256, 152 * 4);
-    for (int L = 0; L < 6 && e == cudaSuccess; ++L) {
-        if (transpose) {
-            // blocks of 256 columns, each over a range of rows: about eight blocks per SM
-            const int64_t bx = (cols + kThreads - 1) / kThreads;
-            int64_t by = (152 * 8 + bx - 1) / bx;
-            by = by < rows ? by : rows;
-            by = by < 65535 ? by : 65535;
-            const int64_t rpb = (rows + by - 1) / by;
-            rc_max_kernel<true><<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, L, v_out,
-                                                                                     maxbits, rpb, ws);
-        } else {
-            rc_max_kernel<false><<<grid_for((rows + 7) / 8, 152 * 8), kThreads, 0, st>>>(X, rows, cols, ldx, L, v_out,
-                                                                                        maxbits, 0, ws);
-        }
-        rc_levels_kernel<<<lgrid, 256, 0, st>>>(L, maxbits, v_out, nvec);
-        e = cudaGetLastError();
-    }
+    if (e == cudaSuccess)
+        e = transpose ? cudaFuncSetAttribute(split_tile_kernel<double, 3, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm)
+                      : cudaFuncSetAttribute(split_tile_kernel<double, 3, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e == cudaSuccess && transpose)
+        e = cudaFuncSetAttribute(rc_spec_transpose_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSpecTransposeSmem);
     if (e != cudaSuccess) return e;
+    // grids: transposed max passes use blocks of 256 columns over row ranges
+    const int64_t cbx = (cols + kThreads - 1) / kThreads;
+    int64_t cby = (152 * 8 + cbx - 1) / cbx;
+    cby = cby < rows ? cby : rows;
+    cby = cby < 65535 ? cby : 65535;
+    const int64_t rpb = (rows + cby - 1) / cby;
+    auto max_pass = [&](int L, const int32_t *gate) {
+        if (transpose)
+            rc_max_kernel<true><<<dim3((unsigned)cbx, (unsigned)cby), kThreads, 0, st>>>(X, rows, cols, ldx, L, v_out,
+                                                                                       maxbits, rpb, ws, gate);
+        else
+            rc_max_kernel<false><<<grid_for((rows + 7) / 8, 152 * 8), kThreads, 0, st>>>(X, rows, cols, ldx, L, v_out,
+                                                                                        maxbits, 0, ws, gate);
+        rc_levels_kernel<<<lgrid, 256, 0, st>>>(L, maxbits, v_out, nvec, gate, ws);
+    };
+    // level 0 literally, then all levels speculatively, verified per vector
+    max_pass(0, nullptr);
     const int64_t tiles = ((rows + kTile - 1) / kTile) * ((cols + kTile - 1) / kTile);
     const int gt = grid_for(tiles, 152 * 8);
+    if (transpose) {
+        rc_spec_transpose_kernel<<<gt, kThreads, kSpecTransposeSmem, st>>>(X, rows, cols, ldx, comps, ldcomp, plane,
+                                                                          v_out, vmax, ws, slot);
+    } else {
+        const int64_t bx = (cols + 4 * kThreads - 1) / (4 * kThreads);
+        const int64_t want = (152 * 8 + bx - 1) / bx;
+        const int64_t by = rows < want ? rows : (want < 65535 ? want : 65535);
+        rc_spec_rows_kernel<<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, comps, ldcomp,
+                                                                                  plane, v_out, vmax, ws, slot);
+    }
+    rc_verify_kernel<<<lgrid, 256, 0, st>>>(vmax, v_out, ff, nvec, ws, slot);
+    // literal passes for the vectors whose speculation failed (no-ops otherwise)
+    for (int L = 1; L < 6; ++L) max_pass(L, ff);
     if (transpose)
-        split_tile_kernel<double, 3, true><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, 0, v_out);
+        split_tile_kernel<double, 3, true><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot,
+                                                                     v_out, ff);
     else
-        split_tile_kernel<double, 3, false><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, 0, v_out);
+        split_tile_kernel<double, 3, false><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot,
+                                                                      v_out, ff);
     return cudaGetLastError();
 }
 

@@ -110,7 +110,8 @@ def test_prodsum_workspace_sizes_and_check(lib):
 
 def test_rowcol_argument_checks_need_no_gpu(lib):
     P = 16
-    assert emu.emu_split_f64_rowcol_workspace_bytes(100) == emu.emu_split_workspace_bytes(64) + 1024
+    # header plus 28 bytes per plane row (literal maxima, speculative maxima, fix marks), 256-byte rounded
+    assert emu.emu_split_f64_rowcol_workspace_bytes(100) == emu.emu_split_workspace_bytes(64) + 2816
     assert emu.emu_split_f64_rowcol(P, 100, 8, 8, 0, P, 8, P, P, 600, None) == 3           # workspace
     assert emu.emu_split_f64_rowcol(P, 100, 8, 8, 0, P, 8, 0, P, 1 << 20, None) == 1       # no v_out
     need = emu.emu_gemm_f64_rowcol_workspace_bytes(300, 200, 700)

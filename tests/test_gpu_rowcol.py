@@ -102,3 +102,19 @@ def test_gemm_rowcol_commutes_with_scaling_on_gpu(dev):
     # whole-matrix levels are not scale-invariant on such inputs
     Cg, _ = emu.gemm_f64(to_dev(A, dev), to_dev(B, dev), 21)
     assert not np.array_equal(Cg.cpu().numpy(), C0.cpu().numpy() * scale)
+
+
+@pytest.mark.parametrize("transpose", [False, True])
+def test_split_rowcol_some_vectors_fail_speculation(dev, transpose):
+    """Rows whose residual shrinks by far more than 2^-8 per level (integers at
+    three widely separated scales) fail the speculative levels and are redone
+    by the literal passes alone; uniform rows keep their speculative levels."""
+    rng = np.random.default_rng(48)
+    X = synth.uniform_f64(48, 0, (96, 130))
+    for i in (3, 17, 40, 95):
+        X[i] = (rng.integers(-127, 128, size=130) * 2.0 ** 10 + rng.integers(-127, 128, size=130) * 2.0 ** -20
+                + rng.integers(-127, 128, size=130) * 2.0 ** -50)
+        X[i, 0] = 127 * 2.0 ** 10
+    X = np.ascontiguousarray(X.T) if transpose else X
+    wv = _check_split(X, dev, transpose)
+    assert wv[3, 1] != wv[3, 0] - 8 and wv[4, 1] == wv[4, 0] - 8
