@@ -4,11 +4,13 @@
 // and the copy of C back to the host are pipelined over panels on internal
 // streams, so that the host link and the GPU work at the same time:
 //
-//   FP32: B arrives in K-panels, each split as soon as it lands; A arrives in
-//   row panels, each split and multiplied as soon as it lands; every finished
-//   row panel of C goes back while the next one is computed.  Row panels
-//   alternate between two compute streams so that one panel's last wave of
-//   CTAs overlaps the next panel's first.
+//   FP32: the first two row panels of A arrive, then B in column panels; as
+//   each column panel lands it is split and both leading row panels multiply
+//   it (one block of C each, on the two compute streams), so the GPU works
+//   while B streams in.  The remaining row panels of A then arrive, are split
+//   and multiplied with all of B.  Every finished row panel of C goes back
+//   while the next one is computed; row panels alternate between the two
+//   compute streams so that one panel's last wave of CTAs overlaps the next.
 //
 //   FP64: the split needs the maximum over the whole operand (Eq. (fp64split)),
 //   so A and B arrive whole; B's copy overlaps A's split, and C goes back in
@@ -26,8 +28,8 @@ namespace {
 
 constexpr int kMaxDevices = 64;
 constexpr int kPanelsM = 8;                         // row panels of C (at most)
-constexpr int kPanelsK = 4;                         // K-panels of B in FP32 mode (at most)
-constexpr int kEvents = 1 + 2 * kPanelsK + 4 * kPanelsM + 4;
+constexpr int kPanelsN = 4;                         // column panels of B in FP32 mode (at most)
+constexpr int kEvents = 2 * kPanelsN + 4 * kPanelsM + 8;
 constexpr int64_t kMaxDim = (int64_t)1 << 31;
 
 int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
@@ -63,36 +65,36 @@ cudaError_t device_ctx(HostCtx **out)
 }
 
 // Panel geometry: row panels of Mp rows (a multiple of the 128-row CTA tile),
-// K-panels of Kp (a multiple of the 256 K-chunk).
+// column panels of Nb columns (a multiple of the FP32 kernel's 256-column tile).
 struct Geometry {
-    int64_t ldk, Mp, PM, Kp, PK;
-    Geometry(int64_t M, int64_t K)
+    int64_t ldk, Mp, PM, Nb, PN;
+    Geometry(int64_t M, int64_t N, int64_t K)
     {
         ldk = round_up(K < 1 ? 1 : K, 8);
         Mp = round_up(ceil_div(M, kPanelsM), 128);
         if (Mp < 128) Mp = 128;
         PM = ceil_div(M, Mp);
-        Kp = round_up(ceil_div(K, kPanelsK), kKChunk);
-        if (Kp < kKChunk) Kp = kKChunk;
-        PK = ceil_div(K, Kp);
+        Nb = round_up(ceil_div(N, kPanelsN), 256);
+        if (Nb < 256) Nb = 256;
+        PN = ceil_div(N, Nb);
     }
 };
 
 // Workspace layout (each part 256-byte aligned): header, A planes [s][M][ldk],
 // B planes [s][N][ldk], A staging, B staging, C ring of two row panels, and in
 // FP64 mode one product-sum accumulator per ring slot.  FP32 stages two row
-// panels of A and two K-panels of B; FP64 stages A and B whole.
+// panels of A and two column panels of B; FP64 stages A and B whole.
 struct Layout {
     size_t ap, bp, ast, bst, cring, acc, total;
     Layout(int mode, int64_t M, int64_t N, int64_t K)
     {
-        const Geometry g(M, K);
+        const Geometry g(M, N, K);
         const int64_t s = mode == 64 ? 6 : 3, esz = mode == 64 ? 8 : 4;
         ap = kWsHeaderBytes;
         bp = ap + (size_t)round_up(s * M * g.ldk * 2, 256);
         ast = bp + (size_t)round_up(s * N * g.ldk * 2, 256);
         const int64_t a_stage = mode == 64 ? M * K : 2 * g.Mp * K;
-        const int64_t b_stage = mode == 64 ? K * N : 2 * g.Kp * N;
+        const int64_t b_stage = mode == 64 ? K * N : 2 * K * g.Nb;
         bst = ast + (size_t)round_up(a_stage * esz, 256);
         cring = bst + (size_t)round_up(b_stage * esz, 256);
         acc = cring + (size_t)round_up(2 * g.Mp * N * esz, 256);
@@ -185,7 +187,7 @@ emu_status emu_gemm_f32_host(int64_t M, int64_t N, int64_t K, const float *A, in
     std::lock_guard<std::mutex> lock(g_mutex);
     HostCtx *cx = nullptr;
     if (device_ctx(&cx) != cudaSuccess) return EMU_ERR_CUDA;
-    const Geometry g(M, K);
+    const Geometry g(M, N, K);
     const Layout L(32, M, N, K);
     unsigned char *w = static_cast<unsigned char *>(ws);
     uint16_t *Ap = reinterpret_cast<uint16_t *>(w + L.ap), *Bp = reinterpret_cast<uint16_t *>(w + L.bp);
@@ -194,30 +196,21 @@ emu_status emu_gemm_f32_host(int64_t M, int64_t N, int64_t K, const float *A, in
     const int64_t a_plane = M * g.ldk, b_plane = N * g.ldk;
     int ne = 0;
     cudaError_t e = begin(*cx, ne, h, st);
-
-    // B in K-panels: copy into one of two staging slots, split into planes
-    // columns k0 .. k0 + kp (comp[0]); comp[1] waits for the last split.
-    cudaEvent_t bsplit[kPanelsK] = {};
-    for (int64_t p = 0; p < g.PK && e == cudaSuccess; ++p) {
-        const int64_t k0 = p * g.Kp, kp = (K - k0 < g.Kp) ? K - k0 : g.Kp;
-        float *bs = Bst + (p & 1) * g.Kp * N;
-        if (p >= 2) e = cudaStreamWaitEvent(cx->cin, bsplit[p - 2], 0);       // staging slot consumed
-        if (e == cudaSuccess)
-            e = cudaMemcpy2DAsync(bs, (size_t)N * 4, B + k0 * ldb, (size_t)ldb * 4, (size_t)N * 4, (size_t)kp,
-                                  cudaMemcpyHostToDevice, cx->cin);
-        cudaEvent_t landed = cx->ev[ne++];
-        if (e == cudaSuccess) e = cudaEventRecord(landed, cx->cin);
-        if (e == cudaSuccess) e = cudaStreamWaitEvent(cx->comp[0], landed, 0);
-        if (e == cudaSuccess) e = launch_split_f32(bs, kp, N, N, true, Bp + k0, g.ldk, h, cx->comp[0], b_plane);
-        bsplit[p] = cx->ev[ne++];
-        if (e == cudaSuccess) e = cudaEventRecord(bsplit[p], cx->comp[0]);
+    if (K == 0) {                                     // C = 0, panel by panel
+        auto none = [](int64_t, int64_t, int64_t, cudaStream_t) -> cudaError_t { return cudaSuccess; };
+        auto zero = [&](int64_t, int64_t, int64_t mp, float *cr, cudaStream_t cs) -> cudaError_t {
+            return cudaMemsetAsync(cr, 0, (size_t)mp * N * 4, cs);
+        };
+        if (e == cudaSuccess) e = row_panels(*cx, ne, g, M, N, C, ldc, cring, none, zero);
+        if (e == cudaSuccess) e = finish(*cx, ne, st);
+        return e == cudaSuccess ? EMU_OK : EMU_ERR_CUDA;
     }
-    if (e == cudaSuccess && g.PK > 0) e = cudaStreamWaitEvent(cx->comp[1], bsplit[g.PK - 1], 0);
 
-    // A in row panels: copy, split into plane rows m0 .. m0 + mp, multiply.
+    // row panel i of A: copy into staging slot i & 1, split into plane rows
+    // m0 .. m0 + mp on stream cs
     cudaEvent_t asplit[kPanelsM] = {};
-    auto prepare = [&](int64_t i, int64_t m0, int64_t mp, cudaStream_t cs) -> cudaError_t {
-        if (K == 0) return cudaSuccess;
+    auto load_a = [&](int64_t i, cudaStream_t cs) -> cudaError_t {
+        const int64_t m0 = i * g.Mp, mp = (M - m0 < g.Mp) ? M - m0 : g.Mp;
         float *as = Ast + (i & 1) * g.Mp * K;
         cudaError_t r = (i >= 2) ? cudaStreamWaitEvent(cx->cin, asplit[i - 2], 0) : cudaSuccess;
         if (r == cudaSuccess)
@@ -231,11 +224,59 @@ emu_status emu_gemm_f32_host(int64_t M, int64_t N, int64_t K, const float *A, in
         if (r == cudaSuccess) r = cudaEventRecord(asplit[i], cs);
         return r;
     };
-    auto compute = [&](int64_t, int64_t m0, int64_t mp, float *cr, cudaStream_t cs) -> cudaError_t {
-        if (K == 0) return cudaMemsetAsync(cr, 0, (size_t)mp * N * 4, cs);
-        return launch_prodsum_f32(mp, N, K, Ap + m0 * g.ldk, Bp, g.ldk, cr, N, &h->flags, cs, a_plane);
+    // C row panel i goes back to the host once computed on stream cs
+    cudaEvent_t cdone[kPanelsM] = {};
+    auto store_c = [&](int64_t i, cudaStream_t cs) -> cudaError_t {
+        const int64_t m0 = i * g.Mp, mp = (M - m0 < g.Mp) ? M - m0 : g.Mp;
+        cudaEvent_t ready = cx->ev[ne++];
+        cudaError_t r = cudaEventRecord(ready, cs);
+        if (r == cudaSuccess) r = cudaStreamWaitEvent(cx->cout, ready, 0);
+        if (r == cudaSuccess)
+            r = cudaMemcpy2DAsync(C + m0 * ldc, (size_t)ldc * 4, cring + (i & 1) * g.Mp * N, (size_t)N * 4,
+                                  (size_t)N * 4, (size_t)mp, cudaMemcpyDeviceToHost, cx->cout);
+        cdone[i] = cx->ev[ne++];
+        if (r == cudaSuccess) r = cudaEventRecord(cdone[i], cx->cout);
+        return r;
     };
-    if (e == cudaSuccess) e = row_panels(*cx, ne, g, M, N, C, ldc, cring, prepare, compute);
+
+    // the leading row panels, then B column by column, each column panel
+    // multiplied by the leading row panels as soon as it is split
+    const int64_t lead = g.PM < 2 ? g.PM : 2;
+    for (int64_t i = 0; i < lead && e == cudaSuccess; ++i) e = load_a(i, cx->comp[i]);
+    cudaEvent_t bsplit[kPanelsN] = {};
+    for (int64_t j = 0; j < g.PN && e == cudaSuccess; ++j) {
+        const int64_t n0 = j * g.Nb, nb = (N - n0 < g.Nb) ? N - n0 : g.Nb;
+        float *bs = Bst + (j & 1) * K * g.Nb;
+        if (j >= 2) e = cudaStreamWaitEvent(cx->cin, bsplit[j - 2], 0);       // staging slot consumed
+        if (e == cudaSuccess)
+            e = cudaMemcpy2DAsync(bs, (size_t)nb * 4, B + n0, (size_t)ldb * 4, (size_t)nb * 4, (size_t)K,
+                                  cudaMemcpyHostToDevice, cx->cin);
+        cudaEvent_t landed = cx->ev[ne++];
+        if (e == cudaSuccess) e = cudaEventRecord(landed, cx->cin);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(cx->comp[0], landed, 0);
+        if (e == cudaSuccess) e = launch_split_f32(bs, K, nb, nb, true, Bp + n0 * g.ldk, g.ldk, h, cx->comp[0], b_plane);
+        bsplit[j] = cx->ev[ne++];
+        if (e == cudaSuccess) e = cudaEventRecord(bsplit[j], cx->comp[0]);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(cx->comp[1], bsplit[j], 0);
+        for (int64_t i = 0; i < lead && e == cudaSuccess; ++i) {
+            const int64_t m0 = i * g.Mp, mp = (M - m0 < g.Mp) ? M - m0 : g.Mp;
+            e = launch_prodsum_f32(mp, nb, K, Ap + m0 * g.ldk, Bp + n0 * g.ldk, g.ldk, cring + i * g.Mp * N + n0, N,
+                                   &h->flags, cx->comp[i], a_plane, b_plane);
+        }
+    }
+    for (int64_t i = 0; i < lead && e == cudaSuccess; ++i) e = store_c(i, cx->comp[i]);
+    // the remaining row panels against all of B (both compute streams have
+    // waited for every column panel's split)
+    for (int64_t i = lead; i < g.PM && e == cudaSuccess; ++i) {
+        const int64_t m0 = i * g.Mp, mp = (M - m0 < g.Mp) ? M - m0 : g.Mp;
+        cudaStream_t cs = cx->comp[i & 1];
+        e = load_a(i, cs);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, cdone[i - 2], 0);   // C ring slot copied out
+        if (e == cudaSuccess)
+            e = launch_prodsum_f32(mp, N, K, Ap + m0 * g.ldk, Bp, g.ldk, cring + (i & 1) * g.Mp * N, N, &h->flags, cs,
+                                   a_plane);
+        if (e == cudaSuccess) e = store_c(i, cs);
+    }
     if (e == cudaSuccess) e = finish(*cx, ne, st);
     return e == cudaSuccess ? EMU_OK : EMU_ERR_CUDA;
 }
@@ -254,7 +295,7 @@ emu_status emu_gemm_f64_host(int64_t M, int64_t N, int64_t K, const double *A, i
     std::lock_guard<std::mutex> lock(g_mutex);
     HostCtx *cx = nullptr;
     if (device_ctx(&cx) != cudaSuccess) return EMU_ERR_CUDA;
-    const Geometry g(M, K);
+    const Geometry g(M, N, K);
     const Layout L(64, M, N, K);
     unsigned char *w = static_cast<unsigned char *>(ws);
     uint16_t *Ap = reinterpret_cast<uint16_t *>(w + L.ap), *Bp = reinterpret_cast<uint16_t *>(w + L.bp);

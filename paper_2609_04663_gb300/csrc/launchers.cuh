@@ -27,12 +27,13 @@ cudaError_t launch_split_f64_rc(const double *X, int64_t rows, int64_t cols, int
                                 int slot, cudaStream_t st);
 inline size_t rc_scratch_bytes(int64_t plane_rows) { return (size_t)plane_rows * 28; }
 
-// Product-sums from K-major planes; a_plane: distance between the A planes in
-// elements (0 = dense: M * ldcomp), so that a row panel of a larger plane set
-// can be multiplied on its own.
+// Product-sums from K-major planes; a_plane / b_plane: distance between the A /
+// B planes in elements (0 = dense: M * ldcomp / N * ldcomp), so that a row
+// panel of A or a column panel of B in a larger plane set can be multiplied
+// on its own.
 cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
-                               int64_t a_plane = 0);
+                               int64_t a_plane = 0, int64_t b_plane = 0);
 // acc: FP64 accumulator scratch of f64_acc_bytes(M, N) bytes (16-byte aligned).
 // rowcol: vA / vB are levels per row of A ([6][M]) and per column of B ([6][N]).
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,

@@ -151,11 +151,12 @@ prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
 
 template <int BN, int KB, int STAGES>
 cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
-                    float *C, int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane)
+                    float *C, int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane, int64_t b_plane)
 {
     using Cfg = F32Cfg<BN, KB, STAGES>;
     CUtensorMap ta, tb;
-    if (!make_plane_map(&ta, Ap, K, M, 3, ldcomp, KB, kBM, a_plane) || !make_plane_map(&tb, Bp, K, N, 3, ldcomp, KB, BN))
+    if (!make_plane_map(&ta, Ap, K, M, 3, ldcomp, KB, kBM, a_plane) ||
+        !make_plane_map(&tb, Bp, K, N, 3, ldcomp, KB, BN, b_plane))
         return cudaErrorInvalidValue;
     auto kern = prodsum_f32_kernel<BN, KB, STAGES>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
@@ -172,14 +173,14 @@ cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
 // (128-byte swizzle, 2 stages).
 cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
-                               int64_t a_plane)
+                               int64_t a_plane, int64_t b_plane)
 {
     static const bool narrow = [] {
         const char *e = std::getenv("EMU_F32_TILE");
         return e && e[0] == '1' && e[1] == '2' && e[2] == '8' && e[3] == 'x' && e[4] == '1';
     }();
-    if (narrow) return run_f32<128, 64, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane);
-    return run_f32<256, 32, 3>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane);
+    if (narrow) return run_f32<128, 64, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
+    return run_f32<256, 32, 3>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
 }
 
 }  // namespace emu

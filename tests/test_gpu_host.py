@@ -42,8 +42,9 @@ def run_host(A, B, nprod=None, pinned=True, pads=(0, 0, 0)):
 
 
 @pytest.mark.parametrize("M,N,K,seed", [
-    (300, 200, 700, 21),     # 3 row panels, 3 K-panels, all ragged
-    (2048, 384, 2048, 22),   # 8 row panels and 4 K-panels: both rings reused
+    (300, 200, 700, 21),     # 3 row panels, 1 column panel, ragged
+    (2048, 384, 2048, 22),   # 8 row panels, 2 column panels: both rings reused
+    (1100, 2300, 520, 25),   # 5 row panels, 5 column panels, ragged edges
     (1, 1, 1, 23),
     (129, 257, 33, 24),
 ])
