@@ -176,7 +176,7 @@ class Case:
         self.name = name
         kind, M, N, K, seed, phi, nprods = workload(name)
         self.kind, self.M, self.N, self.K = kind, M, N, K
-        self.mode = 32 if kind == "f32" else 64
+        self.mode = 32 if kind.startswith("f32") else 64
         self.nprod = nprod or nprods[0]
         # each rank draws its own problem (replicas): offset the seed by the rank
         A, B = synth.gemm_inputs(kind, M, N, K, seed + 1000003 * rank, phi=phi)
@@ -329,14 +329,14 @@ class OracleSampler:
 
     def _split(self, X):
         import oracle
-        return oracle.split_f32(X)[0] if self.kind == "f32" else oracle.split_f64(X)[0]
+        return oracle.split_f32(X)[0] if self.kind.startswith("f32") else oracle.split_f64(X)[0]
 
     def sample(self, budget_s: float):
         import numpy as np
         import oracle
         M, N, K = self.M, self.N, self.K
         t0 = time.perf_counter()
-        if self.kind == "f32":
+        if self.kind.startswith("f32"):
             kb = min(K, 1024)
             self._split(self.B[:kb])
             t_b = (time.perf_counter() - t0) * K / kb
@@ -351,7 +351,7 @@ class OracleSampler:
         while True:
             sel = np.arange(self.rows)
             t0 = time.perf_counter()
-            if self.kind == "f32":
+            if self.kind.startswith("f32"):
                 oracle.prodsum_f32(self._split(self.A[sel]), self.Bp)
             else:
                 oracle.prodsum_f64(self.Ap[:, sel], self.Bp, self.nprod)
@@ -360,11 +360,11 @@ class OracleSampler:
                 break
             self.rows = min(M, self.rows * 2)
         share = self.rows / M
-        t = t_rows + t_b * share + (0.0 if self.kind == "f32" else t_a_full * share)
+        t = t_rows + t_b * share + (0.0 if self.kind.startswith("f32") else t_a_full * share)
         cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
         return {"value": 2.0 * self.rows * N * K / t / 1e12, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
                 "sample": f"{self.rows} of {M} output rows of {self.name} (nprod "
-                          f"{6 if self.kind == 'f32' else self.nprod}); operand splits timed and pro-rated to "
+                          f"{6 if self.kind.startswith('f32') else self.nprod}); operand splits timed and pro-rated to "
                           f"those rows; {t:.2f} s of CPU work"}
 
 
@@ -394,7 +394,7 @@ def reference_arm(args, rank, world):
         "impl": "reference", "metric": METRIC, "value": v, "unit": "TFLOP/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * wall / max(args.steps, 1),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "f32" if kind == "f32" else "f64", "data": "synthetic",
+        "dtype": "f32" if kind.startswith("f32") else "f64", "data": "synthetic",
         "config": {"workload": name, "M": M, "N": N, "K": K},
         "cpu_baseline": cpu,
         "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -461,7 +461,8 @@ def variants(args, rank, world, pk):
     todo = [("fp32_n8192", None), ("fp64_n4096", 6), ("fp64_n4096", 10), ("fp64_n4096", 15), ("fp64_n4096", 21)]
     if args.all_variants:
         todo += [("fp32_n1024", None), ("fp32_n2048", None), ("fp32_n4096", None), ("fp32_largek", None),
-                 ("fp64_scaled_phi4_n8192", 21), ("fp64_scaled_phi4_n8192", 10), ("fp64_largek", 21)]
+                 ("fp64_scaled_phi4_n8192", 21), ("fp64_scaled_phi4_n8192", 10), ("fp64_largek", 21),
+                 ("fp32_cancel_n4096", None), ("fp64_cancel_n4096", 21)]
     torch = __import__("torch")
     for name, nprod in todo:
         case = Case(name, rank, nprod)

@@ -110,6 +110,23 @@ def test_gemm_f64_scaled_bitexact(dev, phi, nprod):
     assert np.array_equal(C.cpu().numpy(), Co)
 
 
+@pytest.mark.parametrize("M,N,K,seed", [(150, 260, 513, 8), (64, 130, 2048, 9)])
+def test_cancel_class_parity(dev, M, N, K, seed):
+    """Cancellation-sensitive inputs (A = [P | P], B = [Q ; -Q + 2^-20 R]):
+    FP32 within the scaled bar, FP64 bit for bit, at a ragged odd K."""
+    A, B = synth.gemm_inputs("f32_cancel", M, N, K, seed)
+    C, ws = emu.gemm_f32(to_dev(A, dev), to_dev(B, dev))
+    assert emu.read_flags(ws) == 0
+    Co, _ = oracle.gemm_f32(A, B)
+    ok, worst = fp32_within_tolerance(C.cpu().numpy(), Co, A, B)
+    assert ok, worst
+    A, B = synth.gemm_inputs("f64_cancel", M, N, K, seed)
+    for nprod in (6, 21):
+        C, ws = emu.gemm_f64(to_dev(A, dev), to_dev(B, dev), nprod)
+        assert emu.read_flags(ws) == 0
+        assert np.array_equal(C.cpu().numpy(), oracle.gemm_f64(A, B, nprod)[0]), nprod
+
+
 def test_gemm_f64_partials_at_the_2pow24_edge(dev):
     """Chunk partials needing all 24 FP32 bits must come out of the tensor
     cores exact (the oracle pin's input, widened to a full tile)."""
@@ -265,6 +282,28 @@ def test_fullsize_fp64_scaled_n8192_sampled(dev, phi, seed):
         Cg = C.cpu().numpy()[rows]
         Co = oracle.prodsum_f64(Ap[:, rows], Bp, nprod)
         assert np.array_equal(Cg, Co)
+        del C, ws
+
+
+def test_fullsize_cancel_n4096_sampled(dev):
+    n = 4096
+    A, B = synth.gemm_inputs("f32_cancel", n, n, n, 6)
+    C, ws = emu.gemm_f32(to_dev(A, dev), to_dev(B, dev))
+    assert emu.read_flags(ws) == 0
+    rows = sample_rows(n, 2, 6)
+    Cg = C.cpu().numpy()[rows]
+    del C, ws
+    Co = oracle.prodsum_f32(oracle.split_f32(A[rows])[0], oracle.split_f32(B)[0])
+    ok, worst = fp32_within_tolerance(Cg, Co, A[rows], B)
+    assert ok, worst
+    A, B = synth.gemm_inputs("f64_cancel", n, n, n, 7)
+    Ap, _, _ = oracle.split_f64(A)
+    Bp, _, _ = oracle.split_f64(B)
+    for nprod in (21, 10):
+        C, ws = emu.gemm_f64(to_dev(A, dev), to_dev(B, dev), nprod)
+        assert emu.read_flags(ws) == 0
+        Cg = C.cpu().numpy()[rows]
+        assert np.array_equal(Cg, oracle.prodsum_f64(Ap[:, rows], Bp, nprod)), nprod
         del C, ws
 
 
