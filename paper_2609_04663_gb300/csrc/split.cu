@@ -725,29 +725,31 @@ f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t co
     for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
         const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
         const int64_t gj = c0 + 8 * q;
-        double x[2][8];
+        // two adjacent columns per step (one 16-byte load per row), so that
+        // the element body appears four times in the loop, not sixteen
+#pragma unroll 1
+        for (int k = 0; k < 8; k += 2) {
+            double x[2][2];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int64_t gi = r0 + 2 * p + h;
-            const double *src = X + gi * ldx + gj;
-            if (gi < rows && vin && gj + 8 <= cols) {
+            for (int h = 0; h < 2; ++h) {
+                const int64_t gi = r0 + 2 * p + h;
+                const double *src = X + gi * ldx + gj + k;
+                if (gi < rows && vin && gj + 8 <= cols) {
+                    const double2 a = *reinterpret_cast<const double2 *>(src);
+                    x[h][0] = a.x; x[h][1] = a.y;
+                } else {
 #pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    const double2 a = reinterpret_cast<const double2 *>(src)[k];
-                    x[h][2 * k] = a.x; x[h][2 * k + 1] = a.y;
+                    for (int e = 0; e < 2; ++e) x[h][e] = (gi < rows && gj + k + e < cols) ? src[e] : 0.0;
                 }
-            } else {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) x[h][e] = (gi < rows && gj + e < cols) ? src[e] : 0.0;
             }
-        }
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            uint32_t s0[6], s1[6];
-            spec_element(x[0][e], v0, fast, s0, st);
-            spec_element(x[1][e], v0, fast, s1, st);
+            for (int e = 0; e < 2; ++e) {
+                uint32_t s0[6], s1[6];
+                spec_element(x[0][e], v0, fast, s0, st);
+                spec_element(x[1][e], v0, fast, s1, st);
 #pragma unroll
-            for (int r = 0; r < 6; ++r) smw[(r * kTile + 8 * q + e) * (kTile / 2) + p] = s0[r] | (s1[r] << 16);
+                for (int r = 0; r < 6; ++r) smw[(r * kTile + 8 * q + k + e) * (kTile / 2) + p] = s0[r] | (s1[r] << 16);
+            }
         }
         __syncthreads();
 #pragma unroll 4
@@ -1094,35 +1096,37 @@ rc_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t col
     for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
         const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
         const int64_t gj = c0 + 8 * q;
-        double x[2][8];
+        // two adjacent columns per step (one 16-byte load per row), so that
+        // the element body appears four times in the loop, not sixteen
+#pragma unroll 1
+        for (int k = 0; k < 8; k += 2) {
+            double x[2][2];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int64_t gi = r0 + 2 * p + h;
-            const double *src = X + gi * ldx + gj;
-            if (gi < rows && vin && gj + 8 <= cols) {
+            for (int h = 0; h < 2; ++h) {
+                const int64_t gi = r0 + 2 * p + h;
+                const double *src = X + gi * ldx + gj + k;
+                if (gi < rows && vin && gj + 8 <= cols) {
+                    const double2 a = *reinterpret_cast<const double2 *>(src);
+                    x[h][0] = a.x; x[h][1] = a.y;
+                } else {
 #pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    const double2 a = reinterpret_cast<const double2 *>(src)[k];
-                    x[h][2 * k] = a.x; x[h][2 * k + 1] = a.y;
+                    for (int e = 0; e < 2; ++e) x[h][e] = (gi < rows && gj + k + e < cols) ? src[e] : 0.0;
                 }
-            } else {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) x[h][e] = (gi < rows && gj + e < cols) ? src[e] : 0.0;
             }
-        }
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            const int64_t col = gj + e;
-            const int v0 = col < cols ? vrc[col] : kZeroLevel;
-            uint32_t s0[6], s1[6], m0[5], m1[5];
-            spec_element_mags(x[0][e], v0, s0, badmask, m0);
-            spec_element_mags(x[1][e], v0, s1, badmask, m1);
+            for (int e = 0; e < 2; ++e) {
+                const int64_t col = gj + k + e;
+                const int v0 = col < cols ? vrc[col] : kZeroLevel;
+                uint32_t s0[6], s1[6], m0[5], m1[5];
+                spec_element_mags(x[0][e], v0, s0, badmask, m0);
+                spec_element_mags(x[1][e], v0, s1, badmask, m1);
 #pragma unroll
-            for (int r = 0; r < 6; ++r) smw[(r * kTile + 8 * q + e) * (kTile / 2) + p] = s0[r] | (s1[r] << 16);
+                for (int r = 0; r < 6; ++r) smw[(r * kTile + 8 * q + k + e) * (kTile / 2) + p] = s0[r] | (s1[r] << 16);
 #pragma unroll
-            for (int r = 0; r < 5; ++r) {
-                const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, m0[r] > m1[r] ? m0[r] : m1[r]);
-                if (p == 0 && m && col < cols) atomicMax(&vmax[r * cols + col], m);
+                for (int r = 0; r < 5; ++r) {
+                    const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, m0[r] > m1[r] ? m0[r] : m1[r]);
+                    if (p == 0 && m && col < cols) atomicMax(&vmax[r * cols + col], m);
+                }
             }
         }
         __syncthreads();
