@@ -24,6 +24,7 @@ struct WsHeader {
     int32_t fix_from[2];                  // first level the fix passes redo (6 = none)
     uint32_t slice_bad[2];                // spec pass: bit r set = slice violation at level r
     int32_t vout[2][6];                   // final level exponents as published by the split
+    uint32_t bar_count[2], bar_gen[2];    // grid barrier of the FP64 split's fix passes (per operand)
 };
 constexpr size_t kWsHeaderBytes = 512;
 static_assert(sizeof(WsHeader) <= kWsHeaderBytes, "workspace header too large");

@@ -283,14 +283,14 @@ __device__ __forceinline__ void block_max_to(unsigned long long x, unsigned long
 // per plane row (per input row, or per input column when transposed), read
 // from vrc[6][plane rows].
 template <typename T, int MODE, bool TRANSPOSE>
-__global__ void __launch_bounds__(kThreads)
-split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
-                  uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot,
-                  const int32_t *__restrict__ vrc, const int32_t *__restrict__ ff)
+__device__ __forceinline__ void
+split_tile_pass(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot,
+                const int32_t *__restrict__ vrc, const int32_t *__restrict__ ff, int64_t bid, int64_t nblk,
+                uint16_t *smdyn)
 {
     static_assert(MODE == 2 || MODE == 3, "literal FP64 split modes only");
     constexpr int NS = 6;
-    extern __shared__ __align__(16) uint16_t smdyn[];    // [NS][kTile][kSRow]
     auto sm = [&](int r, int row, int col) -> uint16_t & {
         return smdyn[((size_t)r * kTile + row) * kSRow + col];
     };
@@ -309,7 +309,7 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
     const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;   // 16 x 16 threads
 
-    for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
+    for (int64_t t = bid; t < tiles_r * tiles_c; t += nblk) {
         const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
         // ---- load, split, stage: thread (ty, tx) owns rows ty + 16p, columns 4tx..4tx+3
 #pragma unroll
@@ -389,16 +389,27 @@ split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t l
     }
 }
 
+// The pass above as a kernel of its own (smdyn: [NS][kTile][kSRow]).
+template <typename T, int MODE, bool TRANSPOSE>
+__global__ void __launch_bounds__(kThreads)
+split_tile_kernel(const T *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                  uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot,
+                  const int32_t *__restrict__ vrc, const int32_t *__restrict__ ff)
+{
+    extern __shared__ __align__(16) uint16_t smdyn[];
+    split_tile_pass<T, MODE, TRANSPOSE>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, vrc, ff, blockIdx.x,
+                                        gridDim.x, smdyn);
+}
+
 // --------------------------------------------- row-segment FP64 passes
 // LEVEL = 0: max |x| and the input-domain checks of Eq. (bf16rangefp64).
 // LEVEL = L in 1..5: max |A^(L)| recomputed literally from x with the final
 // levels 0..L-1 (only when the trusted speculative levels end before L).
 template <int LEVEL>
-__global__ void __launch_bounds__(kThreads)
-f64_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, WsHeader *ws,
-               int slot)
+__device__ __forceinline__ void f64_max_pass(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                                             WsHeader *ws, int slot, int64_t bid, int64_t nblk,
+                                             unsigned long long *red)
 {
-    __shared__ unsigned long long red[kThreads / 32];
     int v[6] = {0, 0, 0, 0, 0, 0};
     if constexpr (LEVEL > 0) {
         if (ws->fix_from[slot] >= LEVEL) return;
@@ -411,7 +422,7 @@ f64_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t
     unsigned long long m = 0;
     uint32_t flagbits = 0;
     const int64_t segs = (cols + 4 * kThreads - 1) / (4 * kThreads);
-    for (int64_t it = blockIdx.x; it < rows * segs; it += gridDim.x) {
+    for (int64_t it = bid; it < rows * segs; it += nblk) {
         const int64_t i = it / segs, j0 = (it % segs) * (4 * kThreads) + 4 * threadIdx.x;
         const double *src = X + i * ldx + j0;
         double x[4];
@@ -450,6 +461,14 @@ f64_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t
     }
 }
 
+template <int LEVEL>
+__global__ void __launch_bounds__(kThreads)
+f64_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, WsHeader *ws, int slot)
+{
+    __shared__ unsigned long long red[kThreads / 32];
+    f64_max_pass<LEVEL>(X, rows, cols, ldx, ws, slot, blockIdx.x, gridDim.x, red);
+}
+
 // One thread: checks the speculative levels in order.  Level r's max from
 // the fused pass is literal as long as levels < r were right, so the first
 // mismatch r gives the true v^(r) directly; levels after r are redone.  A
@@ -457,33 +476,34 @@ f64_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t
 // the finalizer flags) also ends the trusted levels at r: the fused pass
 // subtracts the exact projection Z there, while Eq. (fp64split) subtracts
 // fl_BF16(Z), so the literal passes redo the levels after r.
-__global__ void f64_verify_kernel(WsHeader *ws, int slot)
+__device__ __forceinline__ int f64_verify_levels(const WsHeader *ws, int slot, int (&v)[6])
 {
     int ff = 6;
     const uint32_t sb = ws->slice_bad[slot] & 0x3Fu;
     const int badlvl = (sb && !(ws->flags & EMU_FLAG_NONFINITE)) ? __ffs(sb) - 1 : 6;
     const unsigned long long m0 = ws->maxbits[slot][0];
+    for (int r = 0; r < 6; ++r) v[r] = 0;
     if (m0 == 0) {
-        for (int r = 0; r < 6; ++r) ws->v[slot][r] = kZeroLevel;
+        for (int r = 0; r < 6; ++r) v[r] = kZeroLevel;
     } else {
         const int v0 = ceil_log2_bits(m0);
-        ws->v[slot][0] = v0;
+        v[0] = v0;
         if (badlvl == 0) ff = 0;
         bool zero = false;
         for (int r = 1; r < 6 && ff == 6; ++r) {
-            if (zero) { ws->v[slot][r] = kZeroLevel; continue; }
+            if (zero) { v[r] = kZeroLevel; continue; }
             const unsigned long long m = ws->maxbits[slot][r];
-            if (m == 0) { ws->v[slot][r] = kZeroLevel; zero = true; continue; }
+            if (m == 0) { v[r] = kZeroLevel; zero = true; continue; }
             const int vr = ceil_log2_bits(m);
-            ws->v[slot][r] = vr;
+            v[r] = vr;
             if (vr != v0 - 8 * r || r == badlvl) ff = r;
         }
     }
-    ws->fix_from[slot] = ff;
+    return ff;
 }
 
 // One thread: publishes v_out and the slice flag of the levels actually used.
-__global__ void f64_finalize_kernel(WsHeader *ws, int slot, int32_t *v_out)
+__device__ __forceinline__ void f64_finalize(WsHeader *ws, int slot, int32_t *v_out)
 {
     int v[6];
     final_levels(ws, slot, 6, v);
@@ -494,6 +514,80 @@ __global__ void f64_finalize_kernel(WsHeader *ws, int slot, int32_t *v_out)
     const uint32_t sb = ws->slice_bad[slot];
     const uint32_t bad = (sb & keep & 0x3Fu) | ((sb >> 8) & ~keep & 0x3Fu);
     if (bad) atomicOr(&ws->flags, (uint32_t)EMU_FLAG_SLICE);
+}
+
+// Bounded barrier over all blocks of a cooperative launch (ws->bar_*[slot]
+// start at zero; the last block to arrive resets the count and opens the next
+// generation).  After kWaitLimitNs a waiting block sets EMU_FLAG_TIMEOUT and
+// goes on; the results of that call are then void, as the flag says.
+__device__ __forceinline__ void grid_sync(WsHeader *ws, int slot)
+{
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        volatile uint32_t *gen = &ws->bar_gen[slot];
+        const uint32_t g = *gen;
+        __threadfence();
+        if (atomicAdd(&ws->bar_count[slot], 1u) == gridDim.x - 1) {
+            ws->bar_count[slot] = 0;
+            __threadfence();
+            atomicAdd(&ws->bar_gen[slot], 1u);
+        } else {
+            const unsigned long long t0 = globaltimer_ns();
+            for (uint32_t it = 0; *gen == g; ++it) {
+                if ((it & 63u) == 63u && globaltimer_ns() - t0 > kWaitLimitNs) {
+                    atomicOr(&ws->flags, (uint32_t)EMU_FLAG_TIMEOUT);
+                    break;
+                }
+            }
+        }
+        __threadfence();
+    }
+    __syncthreads();
+}
+
+// Everything after the fused pass, in one cooperative launch: every block
+// checks the speculative levels from the pass's maxima (the same answer in
+// each block).  When they held -- the usual case -- block 0 publishes them
+// and the launch ends, no block waiting on another.  Otherwise the literal
+// passes redo the levels from the first wrong one: the maxima of levels
+// fix_from + 1 .. 5 one pass each, then the rewrite of the planes with the
+// final levels, the grid synchronised between passes.
+template <bool TRANSPOSE>
+__global__ void __launch_bounds__(kThreads)
+f64_fix_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, uint16_t *__restrict__ comps,
+               int64_t ldcomp, int64_t plane, WsHeader *ws, int slot, int32_t *v_out)
+{
+    extern __shared__ __align__(16) uint16_t smdyn[];
+    __shared__ unsigned long long red[kThreads / 32];
+    int v[6];
+    const int ff = f64_verify_levels(ws, slot, v);
+    if (ff == 6) {
+        if (blockIdx.x == 0 && threadIdx.x == 0) {
+            for (int r = 0; r < 6; ++r) ws->v[slot][r] = v[r];
+            ws->fix_from[slot] = 6;
+            f64_finalize(ws, slot, v_out);
+        }
+        return;
+    }
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        for (int r = 0; r < 6; ++r) ws->v[slot][r] = v[r];
+        ws->fix_from[slot] = ff;
+    }
+    grid_sync(ws, slot);
+    f64_max_pass<1>(X, rows, cols, ldx, ws, slot, blockIdx.x, gridDim.x, red);
+    grid_sync(ws, slot);
+    f64_max_pass<2>(X, rows, cols, ldx, ws, slot, blockIdx.x, gridDim.x, red);
+    grid_sync(ws, slot);
+    f64_max_pass<3>(X, rows, cols, ldx, ws, slot, blockIdx.x, gridDim.x, red);
+    grid_sync(ws, slot);
+    f64_max_pass<4>(X, rows, cols, ldx, ws, slot, blockIdx.x, gridDim.x, red);
+    grid_sync(ws, slot);
+    f64_max_pass<5>(X, rows, cols, ldx, ws, slot, blockIdx.x, gridDim.x, red);
+    grid_sync(ws, slot);
+    split_tile_pass<double, 2, TRANSPOSE>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, nullptr, nullptr,
+                                          blockIdx.x, gridDim.x, smdyn);
+    grid_sync(ws, slot);
+    if (blockIdx.x == 0 && threadIdx.x == 0) f64_finalize(ws, slot, v_out);
 }
 
 // ------------------------------------------ FP64 speculative pass kernels
@@ -1222,6 +1316,42 @@ cudaError_t launch_split_f32(const float *X, int64_t rows, int64_t cols, int64_t
     return cudaGetLastError();
 }
 
+namespace {
+
+// Cooperative launch of f64_fix_kernel: as many blocks as fit on the device
+// at once (at most 152 x 8), found once per device.
+template <bool TRANSPOSE>
+cudaError_t launch_f64_fix(const double *X, int64_t rows, int64_t cols, int64_t ldx, uint16_t *comps,
+                           int64_t ldcomp, int64_t plane, WsHeader *ws, int slot, int32_t *v_out, cudaStream_t st)
+{
+    constexpr int kMaxDev = 64;
+    static int grid_of[kMaxDev] = {};
+    const size_t sm = smem_bytes(6);
+    auto kern = f64_fix_kernel<TRANSPOSE>;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDev) return cudaErrorInvalidDevice;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    int grid = grid_of[dev];
+    if (grid == 0) {
+        int sms = 0, per = 0;
+        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, kern, kThreads, sm);
+        if (e != cudaSuccess) return e;
+        grid = per * sms;
+        if (grid > 152 * 8) grid = 152 * 8;
+        if (grid < 1) return cudaErrorInvalidConfiguration;
+        grid_of[dev] = grid;
+    }
+    void *args[] = {(void *)&X, (void *)&rows, (void *)&cols, (void *)&ldx, (void *)&comps, (void *)&ldcomp,
+                    (void *)&plane, (void *)&ws, (void *)&slot, (void *)&v_out};
+    return cudaLaunchCooperativeKernel((const void *)kern, dim3((unsigned)grid), dim3(kThreads), args, sm, st);
+}
+
+}  // namespace
+
 cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
                              uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
                              cudaStream_t st)
@@ -1232,14 +1362,10 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
         const int gmax = grid_for(segs, 152 * 8);
         const int64_t tiles = ((rows + kTile - 1) / kTile) * ((cols + kTile - 1) / kTile);
         const int gt = grid_for(tiles, 152 * 8);
-        const size_t sm = smem_bytes(6);
         cudaError_t e = cudaSuccess;
         if (transpose) {
             e = cudaFuncSetAttribute(f64_spec_transpose_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)kSpecTransposeSmem);
-            if (e == cudaSuccess) e = cudaFuncSetAttribute(split_tile_kernel<double, 2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-        } else {
-            e = cudaFuncSetAttribute(split_tile_kernel<double, 2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
         }
         if (e != cudaSuccess) return e;
         f64_max_kernel<0><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
@@ -1254,20 +1380,14 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
             f64_spec_rows_kernel<<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, comps,
                                                                                        ldcomp, plane, ws, slot);
         }
-        f64_verify_kernel<<<1, 1, 0, st>>>(ws, slot);
-        f64_max_kernel<1><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
-        f64_max_kernel<2><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
-        f64_max_kernel<3><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
-        f64_max_kernel<4><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
-        f64_max_kernel<5><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
-        if (transpose)
-            split_tile_kernel<double, 2, true><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, nullptr, nullptr);
-        else
-            split_tile_kernel<double, 2, false><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, nullptr, nullptr);
-    } else {
-        f64_verify_kernel<<<1, 1, 0, st>>>(ws, slot);
+        if (e == cudaSuccess) e = cudaGetLastError();
+        if (e == cudaSuccess)
+            e = transpose ? launch_f64_fix<true>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, v_out, st)
+                          : launch_f64_fix<false>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, v_out, st);
+        return e;
     }
-    f64_finalize_kernel<<<1, 1, 0, st>>>(ws, slot, v_out);
+    // an empty matrix: all levels zero, nothing to fix
+    f64_fix_kernel<false><<<1, kThreads, 0, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, v_out);
     return cudaGetLastError();
 }
 

@@ -110,6 +110,19 @@ def test_split_f64_fix_path_levels(dev, transpose):
     _check_f64(np.zeros((20, 30)), dev, transpose)
 
 
+@pytest.mark.parametrize("transpose", [False, True])
+def test_split_f64_fix_path_large(dev, transpose):
+    """The fix path on a matrix that spans every block of its launch: the
+    literal passes run across the whole grid with barriers between them."""
+    rng = np.random.default_rng(10)
+    shape = (1500, 1300)
+    X = (rng.integers(-127, 128, size=shape) * 2.0**10 + rng.integers(-127, 128, size=shape) * 2.0**-20
+         + rng.integers(-127, 128, size=shape) * 2.0**-50)
+    X[0, 0] = 127 * 2.0**10
+    wv = _check_f64(X, dev, transpose)
+    assert wv[1] != wv[0] - 8
+
+
 def test_split_f64_flags(dev):
     X = synth.uniform_f64(3, 0, (33, 47))
     for val in (np.nan, np.inf, 2.0**-127, 2.0**129):
