@@ -601,27 +601,41 @@ f64_fix_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t
 // remainder with the opposite sign.  No range check is needed when
 // v0 >= -78: every nonzero slice then lies between 2^(v0 - 48) >= 2^-126 and
 // 2^v0 <= 2^127.  Results are bit-identical to spec_levels.
-// BF16 bits of (-1)^sg * n * 2^e for an integer 0 <= n <= 256 whose value is
-// a normal BF16 (guaranteed on the fast path): n is converted exactly to FP32
-// (2^23 + n by bits, minus 2^23), whose upper half is the BF16 of n; adding e
-// to the exponent field and the sign gives the slice.
-__device__ __forceinline__ uint32_t bf16_of_level(uint32_t n, uint32_t sg, int e)
+// Slices are returned as 32-bit words holding the FP32 value of the slice,
+// whose upper 16 bits are its BF16 bits (the value has at most 8 significant
+// bits, so the lower 16 are zero); two words pack into one plane word with a
+// byte permutation.  The arithmetic runs on the FP32 pipe: n (an integer
+// <= 256) is converted exactly (2^23 + n by bits, minus 2^23) and scaled by
+// the level's unit, a power of two, with the sign of the residual (whose grid
+// is half as coarse when negative: -1/2).  All values are normal floats on
+// the fast path.  The FMA with +0 keeps a zero slice +0.
+__device__ __forceinline__ uint32_t slice_word(uint32_t n, uint32_t sg, float unit)
 {
-    const float fn = __fsub_rn(__uint_as_float(0x4B000000u | n), 8388608.0f);
-    const uint32_t out = (__float_as_uint(fn) >> 16) + ((uint32_t)e << 7) + (sg << 15);
-    return n ? out : 0u;
+    const float fn = __fsub_rn(__uint_as_float(0x4B000000u + n), 8388608.0f);
+    const float us = __fmul_rn(unit, __uint_as_float(0x3F800000u + sg * 0x7F800000u));   // +1 or -1/2
+    return __float_as_uint(__fmaf_rn(fn, us, 0.0f));
 }
 
-// BF16 bits of an FP32 value z (a multiple of the level's grid with at most
-// nine significant bits, or zero) scaled by 2^F.
-__device__ __forceinline__ uint32_t bf16_of_scaled(float z, int F)
+// Slice word of an FP32 value z (a multiple of the level's grid 2^c or 2^(c-1)
+// units, at most nine significant bits) in units of 2^F: z * 2^-c * 2^(F + c),
+// both steps exact; a zero z gives +0.
+__device__ __forceinline__ uint32_t slice_word_scaled(float z, float inv_grid, float unit)
 {
-    const uint32_t zb = __float_as_uint(z);
-    return (zb & 0x7FFFFFFFu) ? (zb >> 16) + ((uint32_t)F << 7) : 0u;
+    return __float_as_uint(__fmul_rn(__fmul_rn(z, inv_grid), unit));
 }
 
-__device__ __forceinline__ void spec_levels_fast(double x, int F, uint32_t (&s)[6], uint32_t &badmask,
-                                                 unsigned long long &m1, unsigned long long &m2, uint32_t (&m)[3])
+// Units of the six levels of the fast path: 2^(F + 43 - 8r), r = 0..5 (the
+// grid of a non-negative residual at level r, in value).
+__device__ __forceinline__ void spec_units(int F, float (&P)[6])
+{
+    P[0] = __int_as_float((F + 43 + 127) << 23);
+#pragma unroll
+    for (int r = 1; r < 6; ++r) P[r] = __fmul_rn(P[r - 1], 0.00390625f);          // 2^-8
+}
+
+__device__ __forceinline__ void spec_levels_fast(double x, int F, const float (&P)[6], uint32_t (&s)[6],
+                                                 uint32_t &badmask, unsigned long long &m1, unsigned long long &m2,
+                                                 uint32_t (&m)[3])
 {
     const uint64_t b = (uint64_t)__double_as_longlong(x);
     uint32_t sg = (uint32_t)(b >> 63);
@@ -648,7 +662,7 @@ __device__ __forceinline__ void spec_levels_fast(double x, int F, uint32_t (&s)[
         const uint32_t t = H >> gh, rh = H & ((1u << gh) - 1u), hh = 1u << (gh - 1);
         const uint32_t lnz = (uint32_t)(L != 0u);
         const uint32_t up = (uint32_t)(rh > hh) | ((uint32_t)(rh == hh) & (lnz | (t & 1u)));
-        s[r] = bf16_of_level(t + up, sg, F + 32 + gh);
+        s[r] = slice_word(t + up, sg, P[r]);
         H = up ? (1u << gh) - rh - lnz : rh;
         L = up ? 0u - L : L;
         sg ^= up;
@@ -661,7 +675,7 @@ __device__ __forceinline__ void spec_levels_fast(double x, int F, uint32_t (&s)[
         const int g = 27 - (int)sg;
         const uint32_t t = (H << (32 - g)) | (L >> g), rem = L & ((1u << g) - 1u), half = 1u << (g - 1);
         const uint32_t up = (uint32_t)(rem > half) | ((uint32_t)(rem == half) & t & 1u);
-        s[2] = bf16_of_level(t + up, sg, F + g);
+        s[2] = slice_word(t + up, sg, P[2]);
         Y = up ? (1u << g) - rem : rem;
         sg ^= up;
     }
@@ -671,7 +685,7 @@ __device__ __forceinline__ void spec_levels_fast(double x, int F, uint32_t (&s)[
         const int g = 19 - (int)sg;
         const uint32_t t = Y >> g, rem = Y & ((1u << g) - 1u), half = 1u << (g - 1);
         const uint32_t up = (uint32_t)(rem > half) | ((uint32_t)(rem == half) & t & 1u);
-        s[3] = bf16_of_level(t + up, sg, F + g);
+        s[3] = slice_word(t + up, sg, P[3]);
         Y = up ? (1u << g) - rem : rem;
         sg ^= up;
     }
@@ -686,7 +700,7 @@ __device__ __forceinline__ void spec_levels_fast(double x, int F, uint32_t (&s)[
         const float C = (y < 0.0f) ? (r == 4 ? 12884901888.0f : 50331648.0f)      // 1.5 * 2^33, 1.5 * 2^25
                                    : (r == 4 ? 25769803776.0f : 100663296.0f);    // 1.5 * 2^34, 1.5 * 2^26
         const float z = __fsub_rn(__fadd_rn(y, C), C);
-        s[r] = bf16_of_scaled(z, F);
+        s[r] = slice_word_scaled(z, r == 4 ? 0.00048828125f : 0.125f, P[r]);     // 2^-11, 2^-3
         y = __fsub_rn(y, z);
     }
 }
@@ -698,13 +712,14 @@ struct SpecState {
     uint32_t badmask = 0;
 };
 
-__device__ __forceinline__ void spec_element(double x, int v0, bool fast, uint32_t (&s)[6], SpecState &st)
+__device__ __forceinline__ void spec_element(double x, int v0, bool fast, const float (&P)[6], uint32_t (&s)[6],
+                                             SpecState &st)
 {
     if (v0 == kZeroLevel) {
 #pragma unroll
         for (int r = 0; r < 6; ++r) s[r] = 0;
     } else if (fast) {
-        spec_levels_fast(x, v0 - 50, s, st.badmask, st.m1, st.m2, st.m);
+        spec_levels_fast(x, v0 - 50, P, s, st.badmask, st.m1, st.m2, st.m);
     } else {                                          // tiny matrices: the checked general form
         uint16_t t[6];
         unsigned long long mx[5] = {st.m1, st.m2, st.m[0], st.m[1], st.m[2]};
@@ -712,9 +727,12 @@ __device__ __forceinline__ void spec_element(double x, int v0, bool fast, uint32
         st.m1 = mx[0]; st.m2 = mx[1];
         st.m[0] = (uint32_t)mx[2]; st.m[1] = (uint32_t)mx[3]; st.m[2] = (uint32_t)mx[4];
 #pragma unroll
-        for (int r = 0; r < 6; ++r) s[r] = t[r];
+        for (int r = 0; r < 6; ++r) s[r] = (uint32_t)t[r] << 16;
     }
 }
+
+// Plane word of two slice words (element e in the lower half, e + 1 in the upper).
+__device__ __forceinline__ uint32_t pack2(uint32_t lo, uint32_t hi) { return __byte_perm(lo, hi, 0x7632); }
 
 // Block-wide publication of the slice flags and the level maxima (as FP64
 // bit patterns of |A^(r)|, r = 1..5).  Every thread of the block calls it.
@@ -759,6 +777,8 @@ f64_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, i
     __shared__ unsigned long long red[5 * (kThreads / 32)];
     const int v0 = spec_v0(ws, slot);
     const bool fast = v0 >= -78;
+    float P[6] = {};
+    if (fast) spec_units(v0 - 50, P);
     const bool vin = ((ldx & 1) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
     const bool vout = ((ldcomp & 3) == 0) && ((plane & 3) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 7u) == 0);
     const int64_t j0 = ((int64_t)blockIdx.x * kThreads + threadIdx.x) * 4;
@@ -775,13 +795,14 @@ f64_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, i
 #pragma unroll
                 for (int e = 0; e < 4; ++e) x[e] = (j0 + e < cols) ? src[e] : 0.0;
             }
-            uint32_t w[6][2] = {};
+            uint32_t w[6][2];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                uint32_t sl[6];
-                spec_element(x[e], v0, fast, sl, st);
+            for (int e = 0; e < 4; e += 2) {
+                uint32_t sa[6], sb[6];
+                spec_element(x[e], v0, fast, P, sa, st);
+                spec_element(x[e + 1], v0, fast, P, sb, st);
 #pragma unroll
-                for (int r = 0; r < 6; ++r) w[r][e >> 1] |= sl[r] << (16 * (e & 1));
+                for (int r = 0; r < 6; ++r) w[r][e >> 1] = pack2(sa[r], sb[r]);
             }
             uint16_t *dst = comps + i * ldcomp + j0;
 #pragma unroll
@@ -811,6 +832,8 @@ f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t co
     __shared__ unsigned long long red[5 * (kThreads / 32)];
     const int v0 = spec_v0(ws, slot);
     const bool fast = v0 >= -78;
+    float P[6] = {};
+    if (fast) spec_units(v0 - 50, P);
     const bool vin = ((ldx & 1) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
     const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
     const int q = threadIdx.x >> 5, p = lane_id();
@@ -839,10 +862,10 @@ f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t co
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
                 uint32_t s0[6], s1[6];
-                spec_element(x[0][e], v0, fast, s0, st);
-                spec_element(x[1][e], v0, fast, s1, st);
+                spec_element(x[0][e], v0, fast, P, s0, st);
+                spec_element(x[1][e], v0, fast, P, s1, st);
 #pragma unroll
-                for (int r = 0; r < 6; ++r) smw[(r * kTile + 8 * q + k + e) * (kTile / 2) + p] = s0[r] | (s1[r] << 16);
+                for (int r = 0; r < 6; ++r) smw[(r * kTile + 8 * q + k + e) * (kTile / 2) + p] = pack2(s0[r], s1[r]);
             }
         }
         __syncthreads();
@@ -1105,11 +1128,11 @@ __device__ __forceinline__ uint32_t jam20(unsigned long long m)
     return (uint32_t)(m >> 20) | ((m & 0xFFFFFull) != 0 ? 1u : 0u);
 }
 
-__device__ __forceinline__ void spec_element_mags(double x, int v0, uint32_t (&s)[6], uint32_t &badmask,
-                                                  uint32_t (&mag)[5])
+__device__ __forceinline__ void spec_element_mags(double x, int v0, const float (&P)[6], uint32_t (&s)[6],
+                                                  uint32_t &badmask, uint32_t (&mag)[5])
 {
     SpecState st;
-    spec_element(x, v0, v0 >= -78, s, st);
+    spec_element(x, v0, v0 >= -78, P, s, st);
     badmask |= st.badmask;
     mag[0] = jam20(st.m1);
     mag[1] = jam20(st.m2);
@@ -1142,15 +1165,21 @@ rc_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, in
 #pragma unroll
                 for (int e = 0; e < 4; ++e) x[e] = (j0 + e < cols) ? src[e] : 0.0;
             }
-            uint32_t w[6][2] = {};
+            float P[6] = {};
+            if (v0 >= -78) spec_units(v0 - 50, P);
+            uint32_t w[6][2];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                uint32_t sl[6], mag[5];
-                spec_element_mags(x[e], v0, sl, badmask, mag);
+            for (int e = 0; e < 4; e += 2) {
+                uint32_t sa[6], sb[6], ma[5], mb[5];
+                spec_element_mags(x[e], v0, P, sa, badmask, ma);
+                spec_element_mags(x[e + 1], v0, P, sb, badmask, mb);
 #pragma unroll
-                for (int r = 0; r < 5; ++r) mx[r] = mag[r] > mx[r] ? mag[r] : mx[r];
+                for (int r = 0; r < 5; ++r) {
+                    const uint32_t mm = ma[r] > mb[r] ? ma[r] : mb[r];
+                    mx[r] = mm > mx[r] ? mm : mx[r];
+                }
 #pragma unroll
-                for (int r = 0; r < 6; ++r) w[r][e >> 1] |= sl[r] << (16 * (e & 1));
+                for (int r = 0; r < 6; ++r) w[r][e >> 1] = pack2(sa[r], sb[r]);
             }
             uint16_t *dst = comps + i * ldcomp + j0;
 #pragma unroll
@@ -1211,11 +1240,13 @@ rc_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t col
             for (int e = 0; e < 2; ++e) {
                 const int64_t col = gj + k + e;
                 const int v0 = col < cols ? vrc[col] : kZeroLevel;
+                float P[6] = {};
+                if (v0 >= -78) spec_units(v0 - 50, P);
                 uint32_t s0[6], s1[6], m0[5], m1[5];
-                spec_element_mags(x[0][e], v0, s0, badmask, m0);
-                spec_element_mags(x[1][e], v0, s1, badmask, m1);
+                spec_element_mags(x[0][e], v0, P, s0, badmask, m0);
+                spec_element_mags(x[1][e], v0, P, s1, badmask, m1);
 #pragma unroll
-                for (int r = 0; r < 6; ++r) smw[(r * kTile + 8 * q + k + e) * (kTile / 2) + p] = s0[r] | (s1[r] << 16);
+                for (int r = 0; r < 6; ++r) smw[(r * kTile + 8 * q + k + e) * (kTile / 2) + p] = pack2(s0[r], s1[r]);
 #pragma unroll
                 for (int r = 0; r < 5; ++r) {
                     const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, m0[r] > m1[r] ? m0[r] : m1[r]);
