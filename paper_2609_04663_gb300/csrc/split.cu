@@ -651,6 +651,12 @@ __device__ __forceinline__ void spec_levels_fast(double x, int F, const float (&
     else if (sh0 > -64) a = (M >> (-sh0)) | ((M << (64 + sh0)) != 0 ? 1ull : 0ull);
     else a = 1;
     uint32_t H = (uint32_t)(a >> 32), L = (uint32_t)a;
+    // At every level the rounding is written as multiply-adds where it can
+    // be: with the grid 2^g (g one lower for a negative residual), t the
+    // truncated quotient, rem = X - t 2^g and b the bits below the grid word
+    // (a sticky bit for levels 0 and 1), rounding up happens exactly when
+    // 2 rem + b + (t & 1) > 2^g (above half, or a tie with t odd); then the new
+    // residual is 2^g - rem - b with the opposite sign.
     // levels 0, 1: grid 2^(32 + gh) units, gh = 11 / 10 and 3 / 2
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
@@ -658,13 +664,17 @@ __device__ __forceinline__ void spec_levels_fast(double x, int F, const float (&
             const unsigned long long cur = ((unsigned long long)H << 32) | L;
             m1 = cur > m1 ? cur : m1;
         }
-        const int gh = 11 - 8 * r - (int)sg;
-        const uint32_t t = H >> gh, rh = H & ((1u << gh) - 1u), hh = 1u << (gh - 1);
-        const uint32_t lnz = (uint32_t)(L != 0u);
-        const uint32_t up = (uint32_t)(rh > hh) | ((uint32_t)(rh == hh) & (lnz | (t & 1u)));
+        constexpr uint32_t kG[2] = {1u << 11, 1u << 3};
+        const uint32_t grid = kG[r] - sg * (kG[r] >> 1);
+        const uint32_t t = H >> ((11 - 8 * r) - (int)sg);
+        const uint32_t rh = H - t * grid;
+        const uint32_t lnz = min(L, 1u);
+        const uint32_t lsb = t & 1u;
+        const int32_t d = (int32_t)(grid - 2u * rh - lnz - lsb);
+        const uint32_t up = (uint32_t)d >> 31;
         s[r] = slice_word(t + up, sg, P[r]);
-        H = up ? (1u << gh) - rh - lnz : rh;
-        L = up ? 0u - L : L;
+        H = rh + up * ((uint32_t)d + lsb);
+        L = L * (1u - 2u * up);
         sg ^= up;
     }
     // level 2: |X| < 2^35, grid 2^27 / 2^26
@@ -672,21 +682,27 @@ __device__ __forceinline__ void spec_levels_fast(double x, int F, const float (&
     {
         const unsigned long long cur = ((unsigned long long)H << 32) | L;
         m2 = cur > m2 ? cur : m2;
-        const int g = 27 - (int)sg;
-        const uint32_t t = (H << (32 - g)) | (L >> g), rem = L & ((1u << g) - 1u), half = 1u << (g - 1);
-        const uint32_t up = (uint32_t)(rem > half) | ((uint32_t)(rem == half) & t & 1u);
+        const uint32_t grid = (1u << 27) - sg * (1u << 26);
+        const uint32_t t = __funnelshift_r(L, H, 27 - (int)sg);
+        const uint32_t rem = L - t * grid;
+        const uint32_t lsb = t & 1u;
+        const int32_t d = (int32_t)(grid - 2u * rem - lsb);
+        const uint32_t up = (uint32_t)d >> 31;
         s[2] = slice_word(t + up, sg, P[2]);
-        Y = up ? (1u << g) - rem : rem;
+        Y = rem + up * ((uint32_t)d + lsb);
         sg ^= up;
     }
     // level 3: |X| <= 2^26, grid 2^19 / 2^18
     {
         m[0] = Y > m[0] ? Y : m[0];
-        const int g = 19 - (int)sg;
-        const uint32_t t = Y >> g, rem = Y & ((1u << g) - 1u), half = 1u << (g - 1);
-        const uint32_t up = (uint32_t)(rem > half) | ((uint32_t)(rem == half) & t & 1u);
+        const uint32_t grid = (1u << 19) - sg * (1u << 18);
+        const uint32_t t = Y >> (19 - (int)sg);
+        const uint32_t rem = Y - t * grid;
+        const uint32_t lsb = t & 1u;
+        const int32_t d = (int32_t)(grid - 2u * rem - lsb);
+        const uint32_t up = (uint32_t)d >> 31;
         s[3] = slice_word(t + up, sg, P[3]);
-        Y = up ? (1u << g) - rem : rem;
+        Y = rem + up * ((uint32_t)d + lsb);
         sg ^= up;
     }
     // levels 4, 5: |X| <= 2^18, exact in FP32; the add-subtract projection
