@@ -1066,15 +1066,15 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
 // along it.  Transposed: one thread per column over a range of rows, the
 // block's columns contiguous, maxima merged with atomicMax.  Level 0 also
 // checks the input domain of Eq. (bf16rangefp64).
+// Maxima of |X^(L)| per vector.  Transposed: work item = (block of 256
+// columns, range of rows_per_block rows), column_blocks of them per row range;
+// by rows: one warp per row.  Items are spread over nblk blocks.
 template <bool TRANSPOSE>
-__global__ void __launch_bounds__(kThreads)
-rc_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, int L,
-              const int32_t *__restrict__ vrc, unsigned long long *maxbits, int64_t rows_per_block, WsHeader *ws,
-              const int32_t *__restrict__ ff)
+__device__ __forceinline__ void
+rc_max_pass(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, int L,
+            const int32_t *__restrict__ vrc, unsigned long long *maxbits, int64_t rows_per_block, WsHeader *ws,
+            const int32_t *__restrict__ ff, int64_t bid, int64_t nblk)
 {
-    // ff (fix passes only): levels <= ff[vector] are final; nothing to do for
-    // vectors with ff >= L, and nothing at all unless some vector failed
-    if (ff && ws->fix_any == 0) return;
     constexpr unsigned long long kLo = 0x3810000000000000ull, kHi = 0x47EFE00000000000ull;
     constexpr unsigned long long kInf = 0x7FF0000000000000ull;
     const int64_t nvec = TRANSPOSE ? cols : rows;
@@ -1093,8 +1093,8 @@ rc_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t 
     };
     int v[6] = {0, 0, 0, 0, 0, 0};
     if (!TRANSPOSE) {
-        const int64_t nwarps = (int64_t)gridDim.x * (kThreads / 32);
-        for (int64_t i = (int64_t)blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5); i < rows; i += nwarps) {
+        const int64_t nwarps = nblk * (kThreads / 32);
+        for (int64_t i = bid * (kThreads / 32) + (threadIdx.x >> 5); i < rows; i += nwarps) {
             if (ff && ff[i] >= L) continue;
             for (int l = 0; l < L; ++l) v[l] = vrc[l * nvec + i];
             unsigned long long m = 0;
@@ -1103,27 +1103,43 @@ rc_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t 
             if (lane_id() == 0) maxbits[i] = m;
         }
     } else {
-        const int64_t j = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-        const int64_t i0 = (int64_t)blockIdx.y * rows_per_block;
-        const int64_t i1 = i0 + rows_per_block < rows ? i0 + rows_per_block : rows;
-        if (j < cols && !(ff && ff[j] >= L)) {
-            for (int l = 0; l < L; ++l) v[l] = vrc[l * nvec + j];
-            unsigned long long m = 0;
-            for (int64_t i = i0; i < i1; ++i) take(X[i * ldx + j], v, m);
-            if (m) atomicMax(&maxbits[j], m);
+        const int64_t cblocks = (cols + kThreads - 1) / kThreads;
+        const int64_t ranges = (rows + rows_per_block - 1) / rows_per_block;
+        for (int64_t it = bid; it < cblocks * ranges; it += nblk) {
+            const int64_t j = (it % cblocks) * kThreads + threadIdx.x;
+            const int64_t i0 = (it / cblocks) * rows_per_block;
+            const int64_t i1 = i0 + rows_per_block < rows ? i0 + rows_per_block : rows;
+            if (j < cols && !(ff && ff[j] >= L)) {
+                for (int l = 0; l < L; ++l) v[l] = vrc[l * nvec + j];
+                unsigned long long m = 0;
+                for (int64_t i = i0; i < i1; ++i) take(X[i * ldx + j], v, m);
+                if (m) atomicMax(&maxbits[j], m);
+            }
         }
     }
     flagbits = __reduce_or_sync(0xFFFFFFFFu, flagbits);
     if (flagbits && lane_id() == 0) atomicOr(&ws->flags, flagbits);
 }
 
-// v[L][vector] from the maxima of level L; a vector whose previous level was
-// already zero stays zero (Section 4.3's early stop).  Clears the maxima.
-__global__ void rc_levels_kernel(int L, unsigned long long *maxbits, int32_t *vrc, int64_t nvec, const int32_t *ff,
-                                 const WsHeader *ws)
+// The pass as a kernel: ff (fix passes only): levels <= ff[vector] are final;
+// nothing to do for vectors with ff >= L, and nothing at all unless some
+// vector failed.
+template <bool TRANSPOSE>
+__global__ void __launch_bounds__(kThreads)
+rc_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, int L,
+              const int32_t *__restrict__ vrc, unsigned long long *maxbits, int64_t rows_per_block, WsHeader *ws,
+              const int32_t *__restrict__ ff)
 {
     if (ff && ws->fix_any == 0) return;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += (int64_t)gridDim.x * blockDim.x) {
+    rc_max_pass<TRANSPOSE>(X, rows, cols, ldx, L, vrc, maxbits, rows_per_block, ws, ff, blockIdx.x, gridDim.x);
+}
+
+// v[L][vector] from the maxima of level L; a vector whose previous level was
+// already zero stays zero (Section 4.3's early stop).  Clears the maxima.
+__device__ __forceinline__ void rc_levels_pass(int L, unsigned long long *maxbits, int32_t *vrc, int64_t nvec,
+                                               const int32_t *ff, int64_t tid, int64_t nthreads)
+{
+    for (int64_t i = tid; i < nvec; i += nthreads) {
         if (ff && ff[i] >= L) continue;
         const unsigned long long m = maxbits[i];
         int v = m ? ceil_log2_bits(m) : kZeroLevel;
@@ -1131,6 +1147,14 @@ __global__ void rc_levels_kernel(int L, unsigned long long *maxbits, int32_t *vr
         vrc[L * nvec + i] = v;
         maxbits[i] = 0;
     }
+}
+
+__global__ void rc_levels_kernel(int L, unsigned long long *maxbits, int32_t *vrc, int64_t nvec, const int32_t *ff,
+                                 const WsHeader *ws)
+{
+    if (ff && ws->fix_any == 0) return;
+    rc_levels_pass(L, maxbits, vrc, nvec, ff, (int64_t)blockIdx.x * blockDim.x + threadIdx.x,
+                   (int64_t)gridDim.x * blockDim.x);
 }
 
 // Speculative pass with per-vector levels: each element is split with its
@@ -1305,10 +1329,11 @@ __device__ __forceinline__ int ceil_log2_u32(uint32_t m) { return m <= 1u ? 0 : 
 // BF16 range (or a non-finite input) anywhere in the operand sends every
 // vector to the literal passes, which flag such slices as Eq. (fp64split)
 // computes them.
-__global__ void rc_verify_kernel(const uint32_t *vmax, int32_t *vrc, int32_t *ff, int64_t nvec, WsHeader *ws, int slot)
+__device__ __forceinline__ void rc_verify_pass(const uint32_t *vmax, int32_t *vrc, int32_t *ff, int64_t nvec,
+                                               WsHeader *ws, int slot, int64_t tid, int64_t nthreads)
 {
     const bool fix_all = (ws->slice_bad[slot] & 0x3Fu) != 0;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += (int64_t)gridDim.x * blockDim.x) {
+    for (int64_t i = tid; i < nvec; i += nthreads) {
         const int v0 = vrc[i];
         int f = 6;
         if (v0 == kZeroLevel) {
@@ -1330,6 +1355,34 @@ __global__ void rc_verify_kernel(const uint32_t *vmax, int32_t *vrc, int32_t *ff
         ff[i] = f;
         if (f < 6) atomicOr(&ws->fix_any, 1u);
     }
+}
+
+// Everything after the per-vector speculative pass, in one cooperative
+// launch: every vector is verified; after a grid barrier each block reads
+// whether any vector failed (the same answer everywhere) and, if none did --
+// the usual case -- the launch ends.  Otherwise levels 1 .. 5 are redone
+// literally for the failed vectors (maxima, then levels, the grid
+// synchronised between the steps) and their planes rewritten.
+template <bool TRANSPOSE>
+__global__ void __launch_bounds__(kThreads)
+rc_fix_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, uint16_t *__restrict__ comps,
+              int64_t ldcomp, int64_t plane, const uint32_t *vmax, int32_t *vrc, int32_t *ff,
+              unsigned long long *maxbits, int64_t rows_per_block, WsHeader *ws, int slot)
+{
+    extern __shared__ __align__(16) uint16_t smdyn[];
+    const int64_t nvec = TRANSPOSE ? cols : rows;
+    const int64_t tid = (int64_t)blockIdx.x * kThreads + threadIdx.x, nthreads = (int64_t)gridDim.x * kThreads;
+    rc_verify_pass(vmax, vrc, ff, nvec, ws, slot, tid, nthreads);
+    grid_sync(ws, slot);
+    if (*reinterpret_cast<volatile uint32_t *>(&ws->fix_any) == 0) return;
+    for (int L = 1; L < 6; ++L) {
+        rc_max_pass<TRANSPOSE>(X, rows, cols, ldx, L, vrc, maxbits, rows_per_block, ws, ff, blockIdx.x, gridDim.x);
+        grid_sync(ws, slot);
+        rc_levels_pass(L, maxbits, vrc, nvec, ff, tid, nthreads);
+        grid_sync(ws, slot);
+    }
+    split_tile_pass<double, 3, TRANSPOSE>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, vrc, ff, blockIdx.x,
+                                          gridDim.x, smdyn);
 }
 
 constexpr size_t kSpecTransposeSmem = 6 * kTile * (kTile / 2) * sizeof(uint32_t);
@@ -1438,6 +1491,44 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
     return cudaGetLastError();
 }
 
+namespace {
+
+// Cooperative launch of rc_fix_kernel with as many blocks as fit at once
+// (at most 152 x 8), found once per device.
+template <bool TRANSPOSE>
+cudaError_t launch_rc_fix(const double *X, int64_t rows, int64_t cols, int64_t ldx, uint16_t *comps, int64_t ldcomp,
+                          int64_t plane, const uint32_t *vmax, int32_t *vrc, int32_t *ff, unsigned long long *maxbits,
+                          int64_t rows_per_block, WsHeader *ws, int slot, cudaStream_t st)
+{
+    constexpr int kMaxDev = 64;
+    static int grid_of[kMaxDev] = {};
+    const size_t sm = smem_bytes(6);
+    auto kern = rc_fix_kernel<TRANSPOSE>;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDev) return cudaErrorInvalidDevice;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    int grid = grid_of[dev];
+    if (grid == 0) {
+        int sms = 0, per = 0;
+        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, kern, kThreads, sm);
+        if (e != cudaSuccess) return e;
+        grid = per * sms;
+        if (grid > 152 * 8) grid = 152 * 8;
+        if (grid < 1) return cudaErrorInvalidConfiguration;
+        grid_of[dev] = grid;
+    }
+    void *args[] = {(void *)&X,    (void *)&rows,  (void *)&cols,    (void *)&ldx,           (void *)&comps,
+                    (void *)&ldcomp, (void *)&plane, (void *)&vmax, (void *)&vrc, (void *)&ff,
+                    (void *)&maxbits, (void *)&rows_per_block, (void *)&ws, (void *)&slot};
+    return cudaLaunchCooperativeKernel((const void *)kern, dim3((unsigned)grid), dim3(kThreads), args, sm, st);
+}
+
+}  // namespace
+
 cudaError_t launch_split_f64_rc(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
                                 uint16_t *comps, int64_t ldcomp, int32_t *v_out, void *scratch, WsHeader *ws,
                                 int slot, cudaStream_t st)
@@ -1459,14 +1550,10 @@ cudaError_t launch_split_f64_rc(const double *X, int64_t rows, int64_t cols, int
         }
         return e;
     }
-    const size_t sm = smem_bytes(6);
-    if (e == cudaSuccess)
-        e = transpose ? cudaFuncSetAttribute(split_tile_kernel<double, 3, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm)
-                      : cudaFuncSetAttribute(split_tile_kernel<double, 3, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e == cudaSuccess && transpose)
         e = cudaFuncSetAttribute(rc_spec_transpose_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSpecTransposeSmem);
     if (e != cudaSuccess) return e;
-    // grids: transposed max passes use blocks of 256 columns over row ranges
+    // transposed max passes: work items of 256 columns by rpb rows, one block each
     const int64_t cbx = (cols + kThreads - 1) / kThreads;
     int64_t cby = (152 * 8 + cbx - 1) / cbx;
     cby = cby < rows ? cby : rows;
@@ -1474,8 +1561,8 @@ cudaError_t launch_split_f64_rc(const double *X, int64_t rows, int64_t cols, int
     const int64_t rpb = (rows + cby - 1) / cby;
     auto max_pass = [&](int L, const int32_t *gate) {
         if (transpose)
-            rc_max_kernel<true><<<dim3((unsigned)cbx, (unsigned)cby), kThreads, 0, st>>>(X, rows, cols, ldx, L, v_out,
-                                                                                       maxbits, rpb, ws, gate);
+            rc_max_kernel<true><<<(unsigned)(cbx * cby), kThreads, 0, st>>>(X, rows, cols, ldx, L, v_out, maxbits, rpb,
+                                                                            ws, gate);
         else
             rc_max_kernel<false><<<grid_for((rows + 7) / 8, 152 * 8), kThreads, 0, st>>>(X, rows, cols, ldx, L, v_out,
                                                                                         maxbits, 0, ws, gate);
@@ -1495,16 +1582,15 @@ cudaError_t launch_split_f64_rc(const double *X, int64_t rows, int64_t cols, int
         rc_spec_rows_kernel<<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, comps, ldcomp,
                                                                                   plane, v_out, vmax, ws, slot);
     }
-    rc_verify_kernel<<<lgrid, 256, 0, st>>>(vmax, v_out, ff, nvec, ws, slot);
-    // literal passes for the vectors whose speculation failed (no-ops otherwise)
-    for (int L = 1; L < 6; ++L) max_pass(L, ff);
-    if (transpose)
-        split_tile_kernel<double, 3, true><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot,
-                                                                     v_out, ff);
-    else
-        split_tile_kernel<double, 3, false><<<gt, kThreads, sm, st>>>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot,
-                                                                      v_out, ff);
-    return cudaGetLastError();
+    // verification and the literal passes for the vectors whose speculation
+    // failed, in one cooperative launch
+    e = cudaGetLastError();
+    if (e == cudaSuccess)
+        e = transpose ? launch_rc_fix<true>(X, rows, cols, ldx, comps, ldcomp, plane, vmax, v_out, ff, maxbits, rpb, ws,
+                                            slot, st)
+                      : launch_rc_fix<false>(X, rows, cols, ldx, comps, ldcomp, plane, vmax, v_out, ff, maxbits, rpb,
+                                             ws, slot, st);
+    return e;
 }
 
 }  // namespace emu

@@ -118,3 +118,20 @@ def test_split_rowcol_some_vectors_fail_speculation(dev, transpose):
     X = np.ascontiguousarray(X.T) if transpose else X
     wv = _check_split(X, dev, transpose)
     assert wv[3, 1] != wv[3, 0] - 8 and wv[4, 1] == wv[4, 0] - 8
+
+
+@pytest.mark.parametrize("transpose", [False, True])
+def test_split_rowcol_fix_path_large(dev, transpose):
+    """Failed vectors spread over a matrix that spans every block of the
+    launch: the literal passes run across the whole grid with barriers."""
+    rng = np.random.default_rng(49)
+    X = synth.uniform_f64(49, 0, (1500, 1100))
+    bad = rng.choice(1500, size=60, replace=False)
+    for i in bad:
+        X[i] = (rng.integers(-127, 128, size=1100) * 2.0 ** 10 + rng.integers(-127, 128, size=1100) * 2.0 ** -20
+                + rng.integers(-127, 128, size=1100) * 2.0 ** -50)
+        X[i, 0] = 127 * 2.0 ** 10
+    X = np.ascontiguousarray(X.T) if transpose else X
+    wv = _check_split(X, dev, transpose)
+    good = next(i for i in range(1500) if i not in set(bad))
+    assert wv[bad[0], 1] != wv[bad[0], 0] - 8 and wv[good, 1] == wv[good, 0] - 8
