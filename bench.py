@@ -18,6 +18,7 @@ Rank 0 prints one JSON line.
 from __future__ import annotations
 
 import argparse
+import datetime
 import hashlib
 import json
 import os
@@ -75,7 +76,7 @@ def job_throughput(flop_per_rank_step: float, steps: int, world: int, t_max_s: f
 
 # ------------------------------------------------------------ clock sampler
 class ClockSampler:
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
               "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
               "clocks_event_reasons.sw_power_cap")
     NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
@@ -87,12 +88,15 @@ class ClockSampler:
     def start(self):
         try:
             self.proc = subprocess.Popen(
-                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "50",
                  "-i", str(self.gpu)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
 
-    def stop(self):
+    def stop(self, window=None):
+        """Median SM clock, max clock and throttle reasons of the samples taken
+        inside window = (t0, t1) (epoch seconds; all samples if None or if the
+        window caught none)."""
         if self.proc is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
         self.proc.terminate()
@@ -101,21 +105,24 @@ class ClockSampler:
         except subprocess.TimeoutExpired:
             self.proc.kill()
             out, _ = self.proc.communicate()
-        sm, mx, reasons = [], [], set()
+        rows = []
         for line in out.splitlines():
             f = [t.strip() for t in line.split(",")]
-            if len(f) < 8:
+            if len(f) < 9:
                 continue
             try:
-                sm.append(float(f[1]))
-                mx.append(float(f[2]))
+                ts = datetime.datetime.strptime(f[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                rows.append((ts, float(f[2]), float(f[3]), f[5:9]))
             except ValueError:
                 continue
-            for name, val in zip(self.NAMES, f[4:8]):
-                if val.lower().startswith("active"):
-                    reasons.add(name)
+        inside = [r for r in rows if window and window[0] <= r[0] <= window[1]]
+        used = inside if inside else rows
+        sm = [r[1] for r in used]
+        mx = [r[2] for r in used]
+        reasons = {name for r in used for name, val in zip(self.NAMES, r[3]) if val.lower().startswith("active")}
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
-                "reasons": sorted(reasons), "samples": len(sm)}
+                "reasons": sorted(reasons), "samples": len(sm),
+                "window": "timed region" if inside else "whole run (no sample inside the timed region)"}
 
 
 # ------------------------------------------------------------ workloads
@@ -245,6 +252,7 @@ def time_device(case: Case, steps: int, warmup: int, world: int, flush: bool):
     barrier(world)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
+    epoch0 = time.time()
     for i in range(steps):
         if flush:
             scratch.fill_(i & 0xFF)              # evict the previous step from L2 (not timed)
@@ -257,10 +265,11 @@ def time_device(case: Case, steps: int, warmup: int, world: int, flush: bool):
     barrier(world)
     torch.cuda.synchronize()
     wall = time.perf_counter() - t0
+    window = (epoch0, time.time())
     split_ms = [a.elapsed_time(b) for a, b, _ in ev]
     prod_ms = [b.elapsed_time(c) for _, b, c in ev]
     step_ms = [a.elapsed_time(c) for a, _, c in ev]
-    return {"step_ms": step_ms, "split_ms": split_ms, "prodsum_ms": prod_ms, "wall_s": wall}
+    return {"step_ms": step_ms, "split_ms": split_ms, "prodsum_ms": prod_ms, "wall_s": wall, "window": window}
 
 
 def time_e2e(case: Case, steps: int, warmup: int, world: int):
@@ -414,7 +423,7 @@ def gpu_arm(args, rank, world, local):
     clocks = ClockSampler(local)
     clocks.start()
     res = time_device(case, args.steps, args.warmup, world, flush=False)
-    clk = clocks.stop()
+    clk = clocks.stop(res["window"])
     t_job = max_over_ranks(sum(res["step_ms"]) / 1e3, world)
     value = job_throughput(case.flop, args.steps, world, t_job)
     prod_ms = statistics.mean(res["prodsum_ms"])

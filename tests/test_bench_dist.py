@@ -62,3 +62,34 @@ def test_torchrun_reference_arm_prints_one_line():
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_clock_sampler_keeps_the_timed_window():
+    """Only samples stamped inside the timed region count; throttle reasons
+    are those seen there."""
+    import datetime
+    import bench
+
+    class FakeProc:
+        def __init__(self, out):
+            self.out = out
+
+        def terminate(self):
+            pass
+
+        def communicate(self, timeout=None):
+            return self.out, ""
+
+    def line(t, mhz, power_cap):
+        ts = datetime.datetime.fromtimestamp(t).strftime("%Y/%m/%d %H:%M:%S.%f")[:-3]
+        return f"{ts}, 0, {mhz}, 2070, 900.0, Not Active, Not Active, Not Active, {'Active' if power_cap else 'Not Active'}"
+
+    t0 = 1_800_000_000.0
+    out = "\n".join([line(t0 - 1.0, 300, True), line(t0 + 0.1, 1900, False), line(t0 + 0.2, 1950, False),
+                     line(t0 + 5.0, 400, True)])
+    s = bench.ClockSampler(0)
+    s.proc = FakeProc(out)
+    clk = s.stop((t0, t0 + 1.0))
+    assert clk["samples"] == 2 and clk["sm_mhz"] == 1925 and clk["reasons"] == [] and clk["sm_max_mhz"] == 2070
+    s.proc = FakeProc(out)
+    assert s.stop((t0 + 10, t0 + 11))["samples"] == 4             # nothing inside: every sample
