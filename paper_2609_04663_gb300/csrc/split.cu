@@ -1002,11 +1002,10 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
     const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
     const int q = threadIdx.x >> 5, p = lane_id();
     const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
-    uint32_t amax = 0;
-    for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
-        const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
-        const int64_t gj = c0 + 8 * q;
-        float x[2][8];
+    // the next tile's rows are loaded before this tile is split and stored,
+    // so that the loads of a block overlap its own stores
+    auto load_tile = [&](int64_t t, float (&x)[2][8]) {
+        const int64_t r0 = (t / tiles_c) * kTile, gj = (t % tiles_c) * kTile + 8 * q;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
             const int64_t gi = r0 + 2 * p + h;
@@ -1020,6 +1019,14 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
                 for (int e = 0; e < 8; ++e) x[h][e] = (gi < rows && gj + e < cols) ? src[e] : 0.0f;
             }
         }
+    };
+    uint32_t amax = 0;
+    float x[2][8];
+    if ((int64_t)blockIdx.x < tiles_r * tiles_c) load_tile(blockIdx.x, x);
+    for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
+        const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
+        float xn[2][8];
+        if (t + gridDim.x < tiles_r * tiles_c) load_tile(t + gridDim.x, xn);
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
             amax = max(amax, max(__float_as_uint(x[0][e]) & 0x7FFFFFFFu, __float_as_uint(x[1][e]) & 0x7FFFFFFFu));
@@ -1050,6 +1057,10 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
             }
         }
         __syncthreads();
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int e = 0; e < 8; ++e) x[h][e] = xn[h][e];
     }
     publish_f32_flags(amax, ws);
 }
