@@ -165,3 +165,19 @@ def test_split_f64_scales_bitexact(dev, scale_exp, transpose):
     BF16 normal range and are flagged); both must match the oracle."""
     X = synth.uniform_f64(7, 0, (130, 75)) * 2.0**scale_exp
     _check_f64(X, dev, transpose, pad=3)
+
+
+@pytest.mark.parametrize("shape", [(0, 5), (7, 0), (0, 0)])
+@pytest.mark.parametrize("transpose", [False, True])
+def test_split_f64_empty_operands(dev, shape, transpose):
+    """An empty operand has no nonzero entry: all six levels are zero and no
+    flag is raised, through the whole-matrix and the per-vector splits."""
+    torch = emu._torch()
+    X = torch.zeros(shape, dtype=torch.float64, device=dev)
+    planes, v, ws = emu.split_f64(X, transpose=transpose, ldcomp=8)
+    assert emu.read_flags(ws) == 0
+    assert v.cpu().tolist() == [oracle.ZERO_LEVEL] * 6
+    if (shape[1] if transpose else shape[0]) > 0:
+        planes, v, ws = emu.split_f64_rowcol(X, transpose=transpose, ldcomp=8)
+        assert emu.read_flags(ws) == 0
+        assert (v.cpu().numpy() == oracle.ZERO_LEVEL).all()
