@@ -22,6 +22,12 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
 // input column when transposed): v_out[6][plane rows] (level-major);
 // scratch: rc_scratch_bytes(plane rows) bytes, 8-byte aligned; slot: the
 // header's per-operand state (0 = A, 1 = B).
+// The whole-matrix FP64 split's verifier and literal fix passes (one
+// cooperative launch after the speculative pass), and its form for an empty
+// matrix.
+cudaError_t launch_f64_fix(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose, uint16_t *comps,
+                           int64_t ldcomp, int64_t plane, WsHeader *ws, int slot, int32_t *v_out, cudaStream_t st);
+cudaError_t launch_f64_fix_empty(WsHeader *ws, int slot, int32_t *v_out, cudaStream_t st);
 cudaError_t launch_split_f64_rc(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
                                 uint16_t *comps, int64_t ldcomp, int32_t *v_out, void *scratch, WsHeader *ws,
                                 int slot, cudaStream_t st);

@@ -1,0 +1,188 @@
+// FP32 three-slice residual split, Eq. (fp32split): element pairs rounded by
+// the hardware BF16x2 conversion; row-major planes straight from registers,
+// transposed (K-major) planes through a conflict-free shared-memory tile.
+#include "split_common.cuh"
+
+namespace emu {
+
+namespace {
+
+// ------------------------------------------------------ FP32 split kernels
+// Eq. (fp32split) on pairs of elements: the hardware conversion
+// cvt.rn.bf16x2.f32 rounds two FP32 values to BF16 (round to nearest, ties
+// to even, subnormals kept) and packs them into one 32-bit word, low element
+// in the low half.  The residual of each is an exact FP32 subtraction of its
+// slice, whose FP32 value is the BF16 bits shifted into the upper half.
+__device__ __forceinline__ uint32_t bf16x2_rn(float lo, float hi)
+{
+    uint32_t d;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+    return d;
+}
+
+// Three slice words (planes 0, 1, 2) of the element pair (x0, x1).
+__device__ __forceinline__ void split_pair(float x0, float x1, uint32_t &w0, uint32_t &w1, uint32_t &w2)
+{
+    w0 = bf16x2_rn(x0, x1);
+    const float r0 = __fsub_rn(x0, __uint_as_float(w0 << 16)), r1 = __fsub_rn(x1, __uint_as_float(w0 & 0xFFFF0000u));
+    w1 = bf16x2_rn(r0, r1);
+    const float q0 = __fsub_rn(r0, __uint_as_float(w1 << 16)), q1 = __fsub_rn(r1, __uint_as_float(w1 & 0xFFFF0000u));
+    w2 = bf16x2_rn(q0, q1);
+}
+
+// Flags of Eq. (fp32split)'s domain from the largest |x| bit pattern seen:
+// a non-finite input, and a slice that is not finite.  For a finite x the
+// only non-finite slice is slice 0 rounding up to infinity, which happens
+// exactly when |x| >= 0x7F7F8000 (half a BF16 ulp above the largest BF16).
+__device__ __forceinline__ void publish_f32_flags(uint32_t amax, WsHeader *ws)
+{
+    uint32_t f = (amax >= 0x7F800000u ? (uint32_t)EMU_FLAG_NONFINITE : 0u) |
+                 (amax >= 0x7F7F8000u ? (uint32_t)EMU_FLAG_SLICE : 0u);
+    f = __reduce_or_sync(0xFFFFFFFFu, f);
+    if (f && lane_id() == 0) atomicOr(&ws->flags, f);
+}
+
+// Row-major planes: thread = 8 consecutive elements of a row (two 16-byte
+// loads, one 16-byte store per plane), no shared memory.  Rows advance by
+// the grid's y dimension.
+__global__ void __launch_bounds__(kThreads)
+split_f32_rows_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                      uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws)
+{
+    const bool vin = ((ldx & 3) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
+    const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
+    const int64_t j0 = ((int64_t)blockIdx.x * kThreads + threadIdx.x) * 8;
+    uint32_t amax = 0;
+    if (j0 < cols) {
+        const bool full = j0 + 8 <= cols;
+        for (int64_t i = blockIdx.y; i < rows; i += gridDim.y) {
+            const float *src = X + i * ldx + j0;
+            float x[8];
+            if (vin && full) {
+                const float4 a = reinterpret_cast<const float4 *>(src)[0], b = reinterpret_cast<const float4 *>(src)[1];
+                x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) x[e] = (j0 + e < cols) ? src[e] : 0.0f;
+            }
+            uint32_t w[3][4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                amax = max(amax, max(__float_as_uint(x[2 * e]) & 0x7FFFFFFFu, __float_as_uint(x[2 * e + 1]) & 0x7FFFFFFFu));
+                split_pair(x[2 * e], x[2 * e + 1], w[0][e], w[1][e], w[2][e]);
+            }
+            uint16_t *dst = comps + i * ldcomp + j0;
+#pragma unroll
+            for (int r = 0; r < 3; ++r) {
+                if (vout && full) {
+                    *reinterpret_cast<uint4 *>(dst + r * plane) = make_uint4(w[r][0], w[r][1], w[r][2], w[r][3]);
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        if (j0 + e < cols) dst[r * plane + e] = (uint16_t)(w[r][e >> 1] >> (16 * (e & 1)));
+                }
+            }
+        }
+    }
+    publish_f32_flags(amax, ws);
+}
+
+// Transposed (K-major) planes: a 64 x 64 tile of X.  Warp q takes columns
+// 8q .. 8q+7, lane p rows 2p and 2p+1, so each slice word packs the two
+// elements that are adjacent in the transposed row; the words go to shared
+// memory (one bank per lane: conflict-free) and leave as 16-byte chunks of
+// whole transposed rows.
+__global__ void __launch_bounds__(kThreads)
+split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                           uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws)
+{
+    __shared__ __align__(16) uint32_t sm[3][kTile][kTile / 2];   // [plane][transposed row][word]
+    const bool vin = ((ldx & 3) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
+    const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
+    const int q = threadIdx.x >> 5, p = lane_id();
+    const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
+    // the next tile's rows are loaded before this tile is split and stored,
+    // so that the loads of a block overlap its own stores
+    auto load_tile = [&](int64_t t, float (&x)[2][8]) {
+        const int64_t r0 = (t / tiles_c) * kTile, gj = (t % tiles_c) * kTile + 8 * q;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int64_t gi = r0 + 2 * p + h;
+            const float *src = X + gi * ldx + gj;
+            if (gi < rows && vin && gj + 8 <= cols) {
+                const float4 a = reinterpret_cast<const float4 *>(src)[0], b = reinterpret_cast<const float4 *>(src)[1];
+                x[h][0] = a.x; x[h][1] = a.y; x[h][2] = a.z; x[h][3] = a.w;
+                x[h][4] = b.x; x[h][5] = b.y; x[h][6] = b.z; x[h][7] = b.w;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) x[h][e] = (gi < rows && gj + e < cols) ? src[e] : 0.0f;
+            }
+        }
+    };
+    uint32_t amax = 0;
+    float x[2][8];
+    if ((int64_t)blockIdx.x < tiles_r * tiles_c) load_tile(blockIdx.x, x);
+    for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
+        const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
+        float xn[2][8];
+        if (t + gridDim.x < tiles_r * tiles_c) load_tile(t + gridDim.x, xn);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            amax = max(amax, max(__float_as_uint(x[0][e]) & 0x7FFFFFFFu, __float_as_uint(x[1][e]) & 0x7FFFFFFFu));
+            uint32_t w0, w1, w2;
+            split_pair(x[0][e], x[1][e], w0, w1, w2);
+            sm[0][8 * q + e][p] = w0;
+            sm[1][8 * q + e][p] = w1;
+            sm[2][8 * q + e][p] = w2;
+        }
+        __syncthreads();
+        // 3 planes x 64 transposed rows x 8 chunks of 16 bytes
+#pragma unroll
+        for (int it = 0; it < 3 * kTile * 8 / kThreads; ++it) {
+            const int c = threadIdx.x + it * kThreads;
+            const int r = c >> 9, orow = (c >> 3) & 63, ch = c & 7;
+            const int64_t go = c0 + orow, gk = r0 + 8 * ch;
+            if (go < cols && gk < rows) {
+                const uint4 v = *reinterpret_cast<const uint4 *>(&sm[r][orow][4 * ch]);
+                uint16_t *dst = comps + r * plane + go * ldcomp + gk;
+                if (vout && gk + 8 <= rows) {
+                    *reinterpret_cast<uint4 *>(dst) = v;
+                } else {
+                    const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        if (gk + e < rows) dst[e] = (uint16_t)(wv[e >> 1] >> (16 * (e & 1)));
+                }
+            }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int e = 0; e < 8; ++e) x[h][e] = xn[h][e];
+    }
+    publish_f32_flags(amax, ws);
+}
+
+}  // namespace
+
+// ----------------------------------------------------------- host launchers
+cudaError_t launch_split_f32(const float *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
+                             uint16_t *comps, int64_t ldcomp, WsHeader *ws, cudaStream_t st, int64_t plane_stride)
+{
+    if (rows == 0 || cols == 0) return cudaSuccess;
+    const int64_t plane = plane_stride ? plane_stride : (transpose ? cols : rows) * ldcomp;
+    if (transpose) {
+        const int64_t tiles = ((rows + kTile - 1) / kTile) * ((cols + kTile - 1) / kTile);
+        split_f32_transpose_kernel<<<grid_for(tiles, 152 * 8), kThreads, 0, st>>>(X, rows, cols, ldx, comps, ldcomp,
+                                                                                   plane, ws);
+    } else {
+        const int64_t bx = (cols + 8 * kThreads - 1) / (8 * kThreads);
+        const int64_t by = rows < 4096 ? rows : 4096;
+        split_f32_rows_kernel<<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, comps, ldcomp,
+                                                                                     plane, ws);
+    }
+    return cudaGetLastError();
+}
+
+}  // namespace emu

@@ -1,0 +1,189 @@
+// FP64 fixed six-slice simplified Ozaki split, Eq. (fp64split), with one set
+// of level exponents per matrix, writing BF16 component planes row-major or
+// transposed (K-major for the B operand).
+//
+// The FP64 split reads a 64 x 64 tile of X with coalesced vector loads,
+// splits it in registers, stages it in shared memory and writes 16-byte
+// chunks of whole plane rows, so transposed B planes are written as
+// coalesced as row-major A planes.
+//
+// FP64 level exponents need a whole-matrix max per level (v^(r) of
+// Eq. (fp64split)), i.e. six dependent grid-wide reductions.  The split does
+// them speculatively in one pass: after the exact max of level 0, the fused
+// pass assumes v^(r) = v^(0) - 8r (a residual always shrinks by at least 2^-8
+// per level, and on full-size dense data by exactly that), writes all six
+// planes and records the true per-level maxima.  One cooperative launch then
+// checks the assumption level by level and, only if it fails, recomputes the
+// remaining levels literally.  The result is identical to the literal
+// definition in every case.
+#include "split_common.cuh"
+
+namespace emu {
+
+namespace {
+
+
+// Row-major planes: thread = 4 consecutive entries of a row (two 16-byte
+// loads, one 8-byte store per plane), rows advancing by the grid's y size.
+__global__ void __launch_bounds__(kThreads)
+f64_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                     uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
+{
+    __shared__ unsigned long long red[5 * (kThreads / 32)];
+    const int v0 = spec_v0(ws, slot);
+    const bool fast = v0 >= -78;
+    float P[6] = {};
+    if (fast) spec_units(v0 - 50, P);
+    const bool vin = ((ldx & 1) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
+    const bool vout = ((ldcomp & 3) == 0) && ((plane & 3) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 7u) == 0);
+    const int64_t j0 = ((int64_t)blockIdx.x * kThreads + threadIdx.x) * 4;
+    SpecState st;
+    if (j0 < cols) {
+        const bool full = j0 + 4 <= cols;
+        for (int64_t i = blockIdx.y; i < rows; i += gridDim.y) {
+            const double *src = X + i * ldx + j0;
+            double x[4];
+            if (vin && full) {
+                const double2 a = reinterpret_cast<const double2 *>(src)[0], c = reinterpret_cast<const double2 *>(src)[1];
+                x[0] = a.x; x[1] = a.y; x[2] = c.x; x[3] = c.y;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) x[e] = (j0 + e < cols) ? src[e] : 0.0;
+            }
+            uint32_t w[6][2];
+#pragma unroll
+            for (int e = 0; e < 4; e += 2) {
+                uint32_t sa[6], sb[6];
+                spec_element(x[e], v0, fast, P, sa, st);
+                spec_element(x[e + 1], v0, fast, P, sb, st);
+#pragma unroll
+                for (int r = 0; r < 6; ++r) w[r][e >> 1] = pack2(sa[r], sb[r]);
+            }
+            uint16_t *dst = comps + i * ldcomp + j0;
+#pragma unroll
+            for (int r = 0; r < 6; ++r) {
+                if (vout && full) {
+                    *reinterpret_cast<uint2 *>(dst + r * plane) = make_uint2(w[r][0], w[r][1]);
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        if (j0 + e < cols) dst[r * plane + e] = (uint16_t)(w[r][e >> 1] >> (16 * (e & 1)));
+                }
+            }
+        }
+    }
+    spec_publish(st, v0, ws, slot, red);
+}
+
+// Transposed (K-major) planes: a 64 x 64 tile, warp q on columns 8q .. 8q+7,
+// lane p on rows 2p and 2p+1; each plane word packs the two entries adjacent
+// in the transposed row, staged one bank per lane and written as 16-byte
+// chunks of whole transposed rows.  Shared memory: [6][64][32] words.
+__global__ void __launch_bounds__(kThreads)
+f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                          uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
+{
+    extern __shared__ __align__(16) uint32_t smw[];                  // [6][kTile][kTile / 2]
+    __shared__ unsigned long long red[5 * (kThreads / 32)];
+    const int v0 = spec_v0(ws, slot);
+    const bool fast = v0 >= -78;
+    float P[6] = {};
+    if (fast) spec_units(v0 - 50, P);
+    const bool vin = ((ldx & 1) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
+    const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
+    const int q = threadIdx.x >> 5, p = lane_id();
+    const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
+    SpecState st;
+    for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
+        const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
+        const int64_t gj = c0 + 8 * q;
+        // two adjacent columns per step (one 16-byte load per row), so that
+        // the element body appears four times in the loop, not sixteen
+#pragma unroll 1
+        for (int k = 0; k < 8; k += 2) {
+            double x[2][2];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int64_t gi = r0 + 2 * p + h;
+                const double *src = X + gi * ldx + gj + k;
+                if (gi < rows && vin && gj + 8 <= cols) {
+                    const double2 a = *reinterpret_cast<const double2 *>(src);
+                    x[h][0] = a.x; x[h][1] = a.y;
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) x[h][e] = (gi < rows && gj + k + e < cols) ? src[e] : 0.0;
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                uint32_t s0[6], s1[6];
+                spec_element(x[0][e], v0, fast, P, s0, st);
+                spec_element(x[1][e], v0, fast, P, s1, st);
+#pragma unroll
+                for (int r = 0; r < 6; ++r) smw[(r * kTile + 8 * q + k + e) * (kTile / 2) + p] = pack2(s0[r], s1[r]);
+            }
+        }
+        __syncthreads();
+#pragma unroll 4
+        for (int it = 0; it < 6 * kTile * 8 / kThreads; ++it) {
+            const int c = threadIdx.x + it * kThreads;
+            const int r = c >> 9, orow = (c >> 3) & 63, ch = c & 7;
+            const int64_t go = c0 + orow, gk = r0 + 8 * ch;
+            if (go < cols && gk < rows) {
+                const uint4 v = *reinterpret_cast<const uint4 *>(&smw[(r * kTile + orow) * (kTile / 2) + 4 * ch]);
+                uint16_t *dst = comps + r * plane + go * ldcomp + gk;
+                if (vout && gk + 8 <= rows) {
+                    *reinterpret_cast<uint4 *>(dst) = v;
+                } else {
+                    const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        if (gk + e < rows) dst[e] = (uint16_t)(wv[e >> 1] >> (16 * (e & 1)));
+                }
+            }
+        }
+        __syncthreads();
+    }
+    spec_publish(st, v0, ws, slot, red);
+}
+
+}  // namespace
+
+cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
+                             uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
+                             cudaStream_t st)
+{
+    const int64_t plane = (transpose ? cols : rows) * ldcomp;
+    if (rows > 0 && cols > 0) {
+        const int64_t segs = rows * ((cols + 4 * kThreads - 1) / (4 * kThreads));
+        const int gmax = grid_for(segs, 152 * 8);
+        const int64_t tiles = ((rows + kTile - 1) / kTile) * ((cols + kTile - 1) / kTile);
+        const int gt = grid_for(tiles, 152 * 8);
+        cudaError_t e = cudaSuccess;
+        if (transpose) {
+            e = cudaFuncSetAttribute(f64_spec_transpose_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)kSpecTransposeSmem);
+        }
+        if (e != cudaSuccess) return e;
+        f64_max_kernel<0><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
+        if (transpose) {
+            f64_spec_transpose_kernel<<<gt, kThreads, kSpecTransposeSmem, st>>>(X, rows, cols, ldx, comps, ldcomp,
+                                                                            plane, ws, slot);
+        } else {
+            // about eight blocks per SM, each over several rows
+            const int64_t bx = (cols + 4 * kThreads - 1) / (4 * kThreads);
+            const int64_t want = (152 * 8 + bx - 1) / bx;
+            const int64_t by = rows < want ? rows : (want < 65535 ? want : 65535);
+            f64_spec_rows_kernel<<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, comps,
+                                                                                       ldcomp, plane, ws, slot);
+        }
+        if (e == cudaSuccess) e = cudaGetLastError();
+        if (e == cudaSuccess) e = launch_f64_fix(X, rows, cols, ldx, transpose, comps, ldcomp, plane, ws, slot, v_out, st);
+        return e;
+    }
+    // an empty matrix: all levels zero, nothing to fix
+    return launch_f64_fix_empty(ws, slot, v_out, st);
+}
+
+
+}  // namespace emu
