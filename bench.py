@@ -174,7 +174,7 @@ def kernel_traffic(kernel: str, workload_name: str):
 class Case:
     """Device-resident inputs, planes and output of one GEMM workload."""
 
-    def __init__(self, name: str, rank: int, nprod: int | None = None):
+    def __init__(self, name: str, rank: int, nprod: int | None = None, fused: bool = False):
         import numpy as np
         import torch
         import synth
@@ -185,6 +185,8 @@ class Case:
         self.kind, self.M, self.N, self.K = kind, M, N, K
         self.mode = 32 if kind.startswith("f32") else 64
         self.nprod = nprod or nprods[0]
+        # FP32 only: the whole path in one kernel (emu_gemm_f32_fused), no planes
+        self.fused = fused and self.mode == 32
         # each rank draws its own problem (replicas): offset the seed by the rank
         A, B = synth.gemm_inputs(kind, M, N, K, seed + 1000003 * rank, phi=phi)
         self.A_host, self.B_host = A, B
@@ -203,12 +205,14 @@ class Case:
         self.flop = 2.0 * M * N * K
         self.exec_flop = self.flop * (6 if self.mode == 32 else self.nprod)
         # kernels of ours per step: FP32 split = 1 launch, FP64 split = 10, product-sum = 1
-        self.launches = (2 * 1 + 1) if self.mode == 32 else (2 * 10 + 1)
+        self.launches = 1 if self.fused else (2 * 1 + 1) if self.mode == 32 else (2 * 10 + 1)
         del np
 
     def split(self, stream):
         emu, st = self.emu, stream.cuda_stream
         ws, n = self.ws.data_ptr(), self.ws.numel()
+        if self.fused:
+            return                                # the split runs inside prodsum()
         if self.mode == 32:
             r = emu.emu_split_f32(self.A.data_ptr(), self.M, self.K, self.A.stride(0), 0, self.Ap.data_ptr(),
                                   self.ldk, ws, n, st)
@@ -223,7 +227,10 @@ class Case:
 
     def prodsum(self, stream):
         emu, st = self.emu, stream.cuda_stream
-        if self.mode == 32:
+        if self.fused:
+            r = emu.emu_gemm_f32_fused(self.M, self.N, self.K, self.A.data_ptr(), self.K, self.B.data_ptr(), self.N,
+                                       self.C.data_ptr(), self.N, self.ws.data_ptr(), self.ws.numel(), st)
+        elif self.mode == 32:
             r = emu.emu_prodsum_f32(self.M, self.N, self.K, self.Ap.data_ptr(), self.Bp.data_ptr(), self.ldk,
                                     self.C.data_ptr(), self.N, self.ws.data_ptr(), self.ws.numel(), st)
         else:
@@ -467,18 +474,20 @@ def gpu_arm(args, rank, world, local):
 def variants(args, rank, world, pk):
     """The other workloads, a few steps each, L2 flushed between steps."""
     out = {}
-    todo = [("fp32_n8192", None), ("fp64_n4096", 6), ("fp64_n4096", 10), ("fp64_n4096", 15), ("fp64_n4096", 21)]
+    todo = [("fp32_n8192", None), ("fp32_n8192", "fused"), ("fp64_n4096", 6), ("fp64_n4096", 10),
+            ("fp64_n4096", 15), ("fp64_n4096", 21)]
     if args.all_variants:
         todo += [("fp32_n1024", None), ("fp32_n2048", None), ("fp32_n4096", None), ("fp32_largek", None),
-                 ("fp64_scaled_phi4_n8192", 21), ("fp64_scaled_phi4_n8192", 10), ("fp64_largek", 21),
-                 ("fp32_cancel_n4096", None), ("fp64_cancel_n4096", 21)]
+                 ("fp32_n16384", "fused"), ("fp64_scaled_phi4_n8192", 21), ("fp64_scaled_phi4_n8192", 10),
+                 ("fp64_largek", 21), ("fp32_cancel_n4096", None), ("fp64_cancel_n4096", 21)]
     torch = __import__("torch")
     for name, nprod in todo:
-        case = Case(name, rank, nprod)
+        fused = nprod == "fused"
+        case = Case(name, rank, None if fused else nprod, fused=fused)
         res = time_device(case, max(3, args.variant_steps), 2, world, flush=True)
         t = max_over_ranks(sum(res["step_ms"]) / 1e3, world)
         pm = statistics.mean(res["prodsum_ms"])
-        key = f"{name}" + (f"_np{case.nprod}" if case.mode == 64 else "")
+        key = f"{name}" + (f"_np{case.nprod}" if case.mode == 64 else "_fused" if fused else "")
         out[key] = {"tflops": job_throughput(case.flop, len(res["step_ms"]), world, t),
                     "ms_per_step": 1e3 * t / len(res["step_ms"]),
                     "prodsum_ms": pm, "split_ms": statistics.mean(res["split_ms"]),

@@ -147,6 +147,18 @@ emu_status emu_gemm_f32(int64_t M, int64_t N, int64_t K, const float *A, int64_t
                         const float *B, int64_t ldb, float *C, int64_t ldc, void *ws,
                         size_t ws_bytes, emu_stream_t stream);
 
+/* FP32-mode emulated GEMM, Algorithm 1, with the split of Eq. (fp32split)
+ * done inside the product-sum's producer (the streamed-slice variant that
+ * Section 6.2 sets aside for the AMX loop order): each CTA splits the FP32
+ * tiles of A and B it is about to multiply, so no slice planes are written
+ * to or read from memory.  Same arguments, slices, product order and
+ * accumulator as emu_gemm_f32, and C is bit-identical to it.  ws: device
+ * workspace of at least emu_split_workspace_bytes(32) bytes (the flag word),
+ * 16-byte aligned.  Errors and flags as emu_gemm_f32. */
+emu_status emu_gemm_f32_fused(int64_t M, int64_t N, int64_t K, const float *A, int64_t lda,
+                              const float *B, int64_t ldb, float *C, int64_t ldc, void *ws,
+                              size_t ws_bytes, emu_stream_t stream);
+
 /* FP64-mode emulated GEMM, Algorithm 2: C = A . B for FP64 inputs, nprod in
  * {6, 10, 15, 21}.  Products are taken in Algorithm 2's diagonal order; for
  * each, the FP32 component product fl32(A_i B_j) is formed on the tensor

@@ -34,6 +34,7 @@ _SIGS = {
     "emu_gemm_workspace_bytes": ("size", ["i", "l", "l", "l"]),
     "emu_gemm_f32": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "p", "size", "p"]),
     "emu_gemm_f64": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "size", "p"]),
+    "emu_gemm_f32_fused": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "p", "size", "p"]),
     "emu_prodsum_f32": ("i", ["l", "l", "l", "p", "p", "l", "p", "l", "p", "size", "p"]),
     "emu_prodsum_f64": ("i", ["l", "l", "l", "p", "p", "l", "p", "p", "i", "p", "l", "p", "size", "p"]),
     "emu_gemm_f64_noalloc": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "p"]),
@@ -96,6 +97,7 @@ emu_split_f64 = _mk("emu_split_f64")
 emu_gemm_workspace_bytes = _mk("emu_gemm_workspace_bytes")
 emu_gemm_f32 = _mk("emu_gemm_f32")
 emu_gemm_f64 = _mk("emu_gemm_f64")
+emu_gemm_f32_fused = _mk("emu_gemm_f32_fused")
 emu_prodsum_f32 = _mk("emu_prodsum_f32")
 emu_prodsum_f64 = _mk("emu_prodsum_f64")
 emu_gemm_f64_noalloc = _mk("emu_gemm_f64_noalloc")
@@ -213,6 +215,19 @@ def gemm_f32(A, B, C=None, ws=None, stream=None):
     ws = ws if ws is not None else workspace(emu_gemm_workspace_bytes(32, M, N, K), A.device)
     _check(emu_gemm_f32(M, N, K, A.data_ptr(), A.stride(0), B.data_ptr(), B.stride(0), C.data_ptr(), C.stride(0),
                         ws.data_ptr(), ws.numel(), _stream(stream)), "emu_gemm_f32")
+    return C, ws
+
+
+def gemm_f32_fused(A, B, C=None, ws=None, stream=None):
+    """emu_gemm_f32_fused: Algorithm 1 with the split inside the product-sum
+    (no planes in memory); C bit-identical to gemm_f32."""
+    torch = _torch()
+    M, K = A.shape
+    N = B.shape[1]
+    C = C if C is not None else torch.empty((M, N), dtype=torch.float32, device=A.device)
+    ws = ws if ws is not None else workspace(emu_split_workspace_bytes(32), A.device)
+    _check(emu_gemm_f32_fused(M, N, K, A.data_ptr(), A.stride(0), B.data_ptr(), B.stride(0), C.data_ptr(),
+                              C.stride(0), ws.data_ptr(), ws.numel(), _stream(stream)), "emu_gemm_f32_fused")
     return C, ws
 
 

@@ -148,6 +148,23 @@ emu_status emu_gemm_f32(int64_t M, int64_t N, int64_t K, const float *A, int64_t
     return cuda_status(e);
 }
 
+emu_status emu_gemm_f32_fused(int64_t M, int64_t N, int64_t K, const float *A, int64_t lda, const float *B,
+                              int64_t ldb, float *C, int64_t ldc, void *ws, size_t ws_bytes, emu_stream_t stream)
+{
+    emu_status s = check_gemm_dims(M, N, K, lda, ldb, ldc);
+    if (s != EMU_OK) return s;
+    if (!ws || (M > 0 && N > 0 && (!C || (K > 0 && (!A || !B))))) return EMU_ERR_INVALID_ARG;
+    if (ws_bytes < kWsHeaderBytes) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
+    if (e != cudaSuccess) return EMU_ERR_CUDA;
+    if (M == 0 || N == 0) return EMU_OK;
+    if (K == 0) return zero_c(C, M, N, ldc, st);
+    return cuda_status(launch_gemm_f32_fused(M, N, K, A, lda, B, ldb, C, ldc, &h->flags, st));
+}
+
 emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda, const double *B,
                         int64_t ldb, double *C, int64_t ldc, int nprod, void *ws, size_t ws_bytes,
                         emu_stream_t stream)

@@ -40,6 +40,11 @@ inline size_t rc_scratch_bytes(int64_t plane_rows) { return (size_t)plane_rows *
 cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
                                int64_t a_plane = 0, int64_t b_plane = 0);
+// Eq. (fp32split) and the FP32 product-sum in one kernel: A (M x K, lda) and
+// B (K x N, ldb) FP32 row-major are split inside the product-sum's producer;
+// no planes are written.  flags receives the split's domain flags.
+cudaError_t launch_gemm_f32_fused(int64_t M, int64_t N, int64_t K, const float *A, int64_t lda, const float *B,
+                                  int64_t ldb, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st);
 // acc: FP64 accumulator scratch of f64_acc_bytes(M, N) bytes (16-byte aligned).
 // rowcol: vA / vB are levels per row of A ([6][M]) and per column of B ([6][N]).
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,

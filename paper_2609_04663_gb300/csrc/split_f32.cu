@@ -2,46 +2,13 @@
 // the hardware BF16x2 conversion; row-major planes straight from registers,
 // transposed (K-major) planes through a conflict-free shared-memory tile.
 #include "split_common.cuh"
+#include "split_f32_pair.cuh"
 
 namespace emu {
 
 namespace {
 
 // ------------------------------------------------------ FP32 split kernels
-// Eq. (fp32split) on pairs of elements: the hardware conversion
-// cvt.rn.bf16x2.f32 rounds two FP32 values to BF16 (round to nearest, ties
-// to even, subnormals kept) and packs them into one 32-bit word, low element
-// in the low half.  The residual of each is an exact FP32 subtraction of its
-// slice, whose FP32 value is the BF16 bits shifted into the upper half.
-__device__ __forceinline__ uint32_t bf16x2_rn(float lo, float hi)
-{
-    uint32_t d;
-    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
-    return d;
-}
-
-// Three slice words (planes 0, 1, 2) of the element pair (x0, x1).
-__device__ __forceinline__ void split_pair(float x0, float x1, uint32_t &w0, uint32_t &w1, uint32_t &w2)
-{
-    w0 = bf16x2_rn(x0, x1);
-    const float r0 = __fsub_rn(x0, __uint_as_float(w0 << 16)), r1 = __fsub_rn(x1, __uint_as_float(w0 & 0xFFFF0000u));
-    w1 = bf16x2_rn(r0, r1);
-    const float q0 = __fsub_rn(r0, __uint_as_float(w1 << 16)), q1 = __fsub_rn(r1, __uint_as_float(w1 & 0xFFFF0000u));
-    w2 = bf16x2_rn(q0, q1);
-}
-
-// Flags of Eq. (fp32split)'s domain from the largest |x| bit pattern seen:
-// a non-finite input, and a slice that is not finite.  For a finite x the
-// only non-finite slice is slice 0 rounding up to infinity, which happens
-// exactly when |x| >= 0x7F7F8000 (half a BF16 ulp above the largest BF16).
-__device__ __forceinline__ void publish_f32_flags(uint32_t amax, WsHeader *ws)
-{
-    uint32_t f = (amax >= 0x7F800000u ? (uint32_t)EMU_FLAG_NONFINITE : 0u) |
-                 (amax >= 0x7F7F8000u ? (uint32_t)EMU_FLAG_SLICE : 0u);
-    f = __reduce_or_sync(0xFFFFFFFFu, f);
-    if (f && lane_id() == 0) atomicOr(&ws->flags, f);
-}
-
 // Row-major planes: thread = 8 consecutive elements of a row (two 16-byte
 // loads, one 16-byte store per plane), no shared memory.  Rows advance by
 // the grid's y dimension.
@@ -68,7 +35,7 @@ split_f32_rows_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, i
             uint32_t w[3][4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
-                amax = max(amax, max(__float_as_uint(x[2 * e]) & 0x7FFFFFFFu, __float_as_uint(x[2 * e + 1]) & 0x7FFFFFFFu));
+                amax = abs_bits_max(amax, x[2 * e], x[2 * e + 1]);
                 split_pair(x[2 * e], x[2 * e + 1], w[0][e], w[1][e], w[2][e]);
             }
             uint16_t *dst = comps + i * ldcomp + j0;
@@ -84,7 +51,7 @@ split_f32_rows_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, i
             }
         }
     }
-    publish_f32_flags(amax, ws);
+    publish_f32_flags(amax, &ws->flags);
 }
 
 // Transposed (K-major) planes: a 64 x 64 tile of X.  Warp q takes columns
@@ -128,7 +95,7 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
         if (t + gridDim.x < tiles_r * tiles_c) load_tile(t + gridDim.x, xn);
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-            amax = max(amax, max(__float_as_uint(x[0][e]) & 0x7FFFFFFFu, __float_as_uint(x[1][e]) & 0x7FFFFFFFu));
+            amax = abs_bits_max(amax, x[0][e], x[1][e]);
             uint32_t w0, w1, w2;
             split_pair(x[0][e], x[1][e], w0, w1, w2);
             sm[0][8 * q + e][p] = w0;
@@ -161,7 +128,7 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
 #pragma unroll
             for (int e = 0; e < 8; ++e) x[h][e] = xn[h][e];
     }
-    publish_f32_flags(amax, ws);
+    publish_f32_flags(amax, &ws->flags);
 }
 
 }  // namespace

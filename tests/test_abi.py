@@ -64,6 +64,11 @@ def test_host_argument_checks_need_no_gpu(lib):
     assert emu.emu_gemm_f32(1 << 31, 4, 4, P, 4, P, 4, P, 4, P, 1 << 62, None) == 5  # size limit
     assert emu.emu_split_f64(P, 4, 4, 2, 0, P, 4, P, P, 4096, None) == 1              # ldx < cols
     assert emu.emu_selftest_timeout(P, 4096, 0, None) == 1
+    # the fused FP32 GEMM needs only the flag word
+    assert emu.emu_gemm_f32_fused(4, 4, 4, P, 3, P, 4, P, 4, P, 512, None) == 1       # lda < K
+    assert emu.emu_gemm_f32_fused(4, 4, 4, P, 4, P, 4, P, 4, P, 511, None) == 3       # workspace
+    assert emu.emu_gemm_f32_fused(4, 4, 4, P, 4, P, 4, P, 4, P + 8, 512, None) == 2   # ws alignment
+    assert emu.emu_gemm_f32_fused(4, 4, 4, 0, 4, P, 4, P, 4, P, 512, None) == 1       # null A
     # host-buffer GEMMs: validation precedes every CUDA call
     W = 256  # 256-byte aligned dummy workspace address
     assert emu.emu_gemm_f32_host(4, 4, 4, P, 3, P, 4, P, 4, W, 1 << 40, None) == 1      # lda < K
