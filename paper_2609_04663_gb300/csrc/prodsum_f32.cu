@@ -191,8 +191,9 @@ prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
 // Cost: a CTA splits every tile it multiplies, so each element of A is split
 // once per 256-column tile of C and each element of B once per 128-row tile
 // (32 and 64 times at 8192^3).  With 16 converter warps this kernel is
-// slower than split + product-sum (4.2 against 3.4 ms at 8192^3); the global
-// loads and the repeated split arithmetic, not the tensor cores, bound it.
+// slower than split + product-sum (4.1 against 3.45 ms at 8192^3): the
+// repeated split arithmetic and the loads keep the schedulers two-thirds busy
+// and leave the tensor pipe idle 28 % of the time.
 constexpr int kFusedPrefetch = 4;        // K-blocks between the L2 prefetch and the loads
 
 __device__ __forceinline__ void st_shared_v2(uint32_t addr, uint32_t a, uint32_t b)
