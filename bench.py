@@ -144,14 +144,27 @@ def peaks():
 
 
 def code_digest(path: str) -> str:
-    """sha256 prefix of a CUDA source with comments and whitespace removed, so
-    that a comment edit does not invalidate counters taken on the same code."""
+    """sha256 prefix of a CUDA source and of the project headers it includes
+    (recursively), with comments and whitespace removed, so that a comment
+    edit does not invalidate counters taken on the same code but a change to
+    any code the kernel is built from does."""
     import re
-    text = open(path).read()
-    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    text = re.sub(r"//[^\n]*", "", text)
-    text = re.sub(r"\s+", "", text)
-    return hashlib.sha256(text.encode()).hexdigest()[:16]
+    seen, parts = set(), []
+
+    def walk(p):
+        p = os.path.normpath(p)
+        if p in seen or not os.path.exists(p):
+            return
+        seen.add(p)
+        text = open(p).read()
+        for inc in re.findall(r'^\s*#\s*include\s+"([^"]+)"', text, flags=re.M):
+            walk(os.path.join(os.path.dirname(p), inc))
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", "", text)
+        parts.append(os.path.basename(p) + ":" + re.sub(r"\s+", "", text))
+
+    walk(path)
+    return hashlib.sha256("\n".join(parts).encode()).hexdigest()[:16]
 
 
 def kernel_traffic(kernel: str, workload_name: str):
