@@ -195,6 +195,68 @@ def gemm_f64(A: np.ndarray, B: np.ndarray, nprod: int, rows=None, order: str = "
     return prodsum_f64(Ap, Bp, nprod, rows=rows, order=order), fa | fb
 
 
+def tail_products(nprod: int, merge_from: int):
+    """Products (i, j) with merge_from <= i + j < d, in Algorithm 2's diagonal
+    order (the tail that the merged variant accumulates in one FP32 sum)."""
+    d = NPROD_TO_D[nprod]
+    return [(i, l - i) for l in range(merge_from, d) for i in range(l + 1)]
+
+
+def _slice_ints(planes: np.ndarray, v: np.ndarray, r: int):
+    """Slice r as exact integers n with value n * 2^(v[r] - 8) (Eq. (fp64split):
+    every slice entry is a multiple of 2^(v - 8) of magnitude <= 2^v), and that
+    exponent; (None, None) for an all-zero level."""
+    if int(v[r]) == ZERO_LEVEL:
+        return None, None
+    e = int(v[r]) - 8
+    vals = np.ldexp(bf16_to_f32(planes[r]).astype(np.float64), -e)
+    n = vals.astype(np.int64)
+    assert np.array_equal(n.astype(np.float64), vals), "slice entry not a multiple of 2^(v-8)"
+    return n, e
+
+
+def gemm_f64_merged(A: np.ndarray, B: np.ndarray, nprod: int, merge_from: int, rows=None):
+    """FP64 mode with merged tail diagonals (an extension, not in the paper).
+
+    The products with i + j < merge_from are summed as in Algorithm 2 (product
+    outer, diagonal order, one FP64 addition each); the remaining products of
+    S_d (merge_from <= i + j < d) form one tail T = sum of A_i B_j that is added
+    once, last: C = fl64(C_head + T).  The GPU accumulates T in FP32 on the
+    tensor cores (order unspecified); here T is the EXACT sum, computed in
+    integers (slice entries are integer multiples of 2^(v - 8)), and rounded
+    once to FP64 only if it needs more than 53 bits.  Returns (C, T, S, flags)
+    with S = sum over the tail of |A_i| |B_j| (the scale of the FP32
+    accumulation error bound)."""
+    d = NPROD_TO_D[nprod]
+    if not 1 <= merge_from <= d:
+        raise ValueError("merge_from must lie in 1 .. d")
+    Ap, va, fa = split_f64(A)
+    Bp, vb, fb = split_f64(B)
+    r0, r1 = (0, A.shape[0]) if rows is None else rows
+    n_head = merge_from * (merge_from + 1) // 2
+    C = prodsum_f64(Ap, Bp, n_head, rows=(r0, r1))
+    N = B.shape[1]
+    terms = []
+    for i, j in tail_products(nprod, merge_from):
+        na, ea = _slice_ints(Ap[:, r0:r1], va, i)
+        nb, eb = _slice_ints(Bp, vb, j)
+        if na is None or nb is None:
+            continue
+        terms.append((na @ nb, ea + eb))          # exact: |entries| <= K * 2^16
+    T = np.zeros((r1 - r0, N), dtype=np.float64)
+    S = np.zeros((r1 - r0, N), dtype=np.float64)
+    if terms:
+        e_min = min(e for _, e in terms)
+        tot = np.zeros((r1 - r0, N), dtype=object)
+        for prod, e in terms:
+            tot = tot + prod.astype(object) * (1 << (e - e_min))
+        T = np.array([[float(x) for x in row] for row in tot], dtype=np.float64).reshape(r1 - r0, N)
+        T = np.ldexp(T, e_min)
+        for i, j in tail_products(nprod, merge_from):
+            S += np.abs(bf16_to_f32(Ap[i, r0:r1]).astype(np.float64)) @ np.abs(bf16_to_f32(Bp[j]).astype(np.float64))
+    return C + T, T, S, fa | fb
+
+
 def gemm_ex(opA: int, opB: int, alpha, A: np.ndarray, B: np.ndarray, beta, C: np.ndarray | None = None,
             nprod: int | None = None):
     """General GEMM C <- alpha op(A) op(B) + beta C (the BLAS semantics that
