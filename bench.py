@@ -187,7 +187,8 @@ def kernel_traffic(kernel: str, workload_name: str):
 class Case:
     """Device-resident inputs, planes and output of one GEMM workload."""
 
-    def __init__(self, name: str, rank: int, nprod: int | None = None, fused: bool = False):
+    def __init__(self, name: str, rank: int, nprod: int | None = None, fused: bool = False,
+                 merge_from: int | None = None):
         import numpy as np
         import torch
         import synth
@@ -200,6 +201,8 @@ class Case:
         self.nprod = nprod or nprods[0]
         # FP32 only: the whole path in one kernel (emu_gemm_f32_fused), no planes
         self.fused = fused and self.mode == 32
+        # FP64 only: the tail diagonals from merge_from on in one FP32 sum (emu_gemm_f64_merged)
+        self.merge_from = merge_from if self.mode == 64 else None
         # each rank draws its own problem (replicas): offset the seed by the rank
         A, B = synth.gemm_inputs(kind, M, N, K, seed + 1000003 * rank, phi=phi)
         self.A_host, self.B_host = A, B
@@ -215,17 +218,21 @@ class Case:
         self.ws = emu.workspace(max(emu.emu_split_workspace_bytes(self.mode),
                                     emu.emu_prodsum_workspace_bytes(self.mode, M, N)), dev)
         self.gemm_ws = None
+        if self.merge_from is not None:
+            self.gemm_ws = emu.workspace(emu.emu_gemm_f64_merged_workspace_bytes(M, N, K), dev)
         self.flop = 2.0 * M * N * K
         self.exec_flop = self.flop * (6 if self.mode == 32 else self.nprod)
         # kernels of ours per step: FP32 split = 1 launch, FP64 split = 10, product-sum = 1
         self.launches = 1 if self.fused else (2 * 1 + 1) if self.mode == 32 else (2 * 10 + 1)
+        if self.merge_from is not None:
+            self.launches += 1                    # the tail kernel
         del np
 
     def split(self, stream):
         emu, st = self.emu, stream.cuda_stream
         ws, n = self.ws.data_ptr(), self.ws.numel()
-        if self.fused:
-            return                                # the split runs inside prodsum()
+        if self.fused or self.merge_from is not None:
+            return                                # the whole GEMM runs in prodsum()
         if self.mode == 32:
             r = emu.emu_split_f32(self.A.data_ptr(), self.M, self.K, self.A.stride(0), 0, self.Ap.data_ptr(),
                                   self.ldk, ws, n, st)
@@ -240,7 +247,11 @@ class Case:
 
     def prodsum(self, stream):
         emu, st = self.emu, stream.cuda_stream
-        if self.fused:
+        if self.merge_from is not None:
+            r = emu.emu_gemm_f64_merged(self.M, self.N, self.K, self.A.data_ptr(), self.K, self.B.data_ptr(), self.N,
+                                        self.C.data_ptr(), self.N, self.nprod, self.merge_from,
+                                        self.gemm_ws.data_ptr(), self.gemm_ws.numel(), st)
+        elif self.fused:
             r = emu.emu_gemm_f32_fused(self.M, self.N, self.K, self.A.data_ptr(), self.K, self.B.data_ptr(), self.N,
                                        self.C.data_ptr(), self.N, self.ws.data_ptr(), self.ws.numel(), st)
         elif self.mode == 32:
@@ -489,26 +500,31 @@ def gpu_arm(args, rank, world, local):
 def variants(args, rank, world, pk):
     """The other workloads, a few steps each, L2 flushed between steps."""
     out = {}
+    # entries: (workload, FP64 product count | "fused" | (product count, merge_from))
     todo = [("fp32_n8192", None), ("fp32_n8192", "fused"), ("fp64_n4096", 6), ("fp64_n4096", 10),
-            ("fp64_n4096", 15), ("fp64_n4096", 21)]
+            ("fp64_n4096", 15), ("fp64_n4096", 21), ("fp64_n4096", (21, 4)), ("fp64_n4096", (15, 4))]
     if args.all_variants:
         todo += [("fp32_n1024", None), ("fp32_n2048", None), ("fp32_n4096", None), ("fp32_largek", None),
                  ("fp32_n16384", "fused"), ("fp64_scaled_phi4_n8192", 21), ("fp64_scaled_phi4_n8192", 10),
+                 ("fp64_scaled_phi4_n8192", (21, 4)), ("fp64_scaled_phi0.5_n8192", 21), ("fp64_scaled_phi0.5_n8192", (21, 4)),
                  ("fp64_largek", 21), ("fp32_cancel_n4096", None), ("fp64_cancel_n4096", 21)]
     torch = __import__("torch")
     for name, nprod in todo:
         fused = nprod == "fused"
-        case = Case(name, rank, None if fused else nprod, fused=fused)
+        merge_from = nprod[1] if isinstance(nprod, tuple) else None
+        nprod = nprod[0] if isinstance(nprod, tuple) else None if fused else nprod
+        case = Case(name, rank, nprod, fused=fused, merge_from=merge_from)
         res = time_device(case, max(3, args.variant_steps), 2, world, flush=True)
         t = max_over_ranks(sum(res["step_ms"]) / 1e3, world)
         pm = statistics.mean(res["prodsum_ms"])
-        key = f"{name}" + (f"_np{case.nprod}" if case.mode == 64 else "_fused" if fused else "")
+        key = f"{name}" + (f"_np{case.nprod}" if case.mode == 64 else "_fused" if fused else "") + \
+            (f"_merged{merge_from}" if merge_from else "")
         out[key] = {"tflops": job_throughput(case.flop, len(res["step_ms"]), world, t),
                     "ms_per_step": 1e3 * t / len(res["step_ms"]),
                     "prodsum_ms": pm, "split_ms": statistics.mean(res["split_ms"]),
                     "executed_tflops": case.exec_flop / (pm / 1e3) / 1e12,
                     "frac_of_bf16_peak": case.exec_flop / (pm / 1e3) / 1e12 / pk["bf16_burst"],
-                    "flags": case.emu.read_flags(case.ws)}
+                    "flags": case.emu.read_flags(case.gemm_ws if case.gemm_ws is not None else case.ws)}
         del case
         torch.cuda.empty_cache()
     return out

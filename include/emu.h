@@ -171,6 +171,26 @@ emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_
                         const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,
                         void *ws, size_t ws_bytes, emu_stream_t stream);
 
+/* FP64 mode with merged tail diagonals (an extension of Algorithm 2, not in
+ * the paper): the products with i + j < merge_from are taken as in
+ * emu_gemm_f64 (diagonal order, each summed exactly over K and added once in
+ * FP64); the remaining products of S_d (merge_from <= i + j < d, with d = 3, 4,
+ * 5, 6 for nprod = 6, 10, 15, 21) are accumulated together in ONE FP32 sum T
+ * over all of K on the tensor cores, and C = fl64(C_head + T) adds it last.
+ * The FP32 rounding of T is bounded by (number of tail MMA steps) x 2^-22 x
+ * sum over the tail of |A_i||B_j|; in practice, at 4096^3 with nprod = 21
+ * and merge_from = 4, e_F is about twice emu_gemm_f64's (still about 100x
+ * below nprod = 15).  In exchange one operand stage feeds every tail product.
+ * merge_from in {3, 4, 5, 6} and <= d;
+ * merge_from = d gives emu_gemm_f64's result bit for bit.  ws: at least
+ * emu_gemm_f64_merged_workspace_bytes(M, N, K) bytes (the FP64 GEMM workspace
+ * plus an M x N FP32 buffer for T), 16-byte aligned.  Errors and flags as
+ * emu_gemm_f64; EMU_ERR_INVALID_ARG also for merge_from out of range. */
+size_t emu_gemm_f64_merged_workspace_bytes(int64_t M, int64_t N, int64_t K);
+emu_status emu_gemm_f64_merged(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda,
+                               const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,
+                               int merge_from, void *ws, size_t ws_bytes, emu_stream_t stream);
+
 /* General GEMM (the "more complete BLAS semantics" of Section 9's future
  * work): C (M x N, ldc) <- alpha * op(A) op(B) + beta * C, all row-major.
  * op(X) is X as stored (EMU_OP_N) or its transpose (EMU_OP_T): with opA = N,

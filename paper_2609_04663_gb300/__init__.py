@@ -35,6 +35,8 @@ _SIGS = {
     "emu_gemm_f32": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "p", "size", "p"]),
     "emu_gemm_f64": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "size", "p"]),
     "emu_gemm_f32_fused": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "p", "size", "p"]),
+    "emu_gemm_f64_merged_workspace_bytes": ("size", ["l", "l", "l"]),
+    "emu_gemm_f64_merged": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "i", "p", "size", "p"]),
     "emu_prodsum_f32": ("i", ["l", "l", "l", "p", "p", "l", "p", "l", "p", "size", "p"]),
     "emu_prodsum_f64": ("i", ["l", "l", "l", "p", "p", "l", "p", "p", "i", "p", "l", "p", "size", "p"]),
     "emu_gemm_f64_noalloc": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "p"]),
@@ -98,6 +100,8 @@ emu_gemm_workspace_bytes = _mk("emu_gemm_workspace_bytes")
 emu_gemm_f32 = _mk("emu_gemm_f32")
 emu_gemm_f64 = _mk("emu_gemm_f64")
 emu_gemm_f32_fused = _mk("emu_gemm_f32_fused")
+emu_gemm_f64_merged_workspace_bytes = _mk("emu_gemm_f64_merged_workspace_bytes")
+emu_gemm_f64_merged = _mk("emu_gemm_f64_merged")
 emu_prodsum_f32 = _mk("emu_prodsum_f32")
 emu_prodsum_f64 = _mk("emu_prodsum_f64")
 emu_gemm_f64_noalloc = _mk("emu_gemm_f64_noalloc")
@@ -240,6 +244,20 @@ def gemm_f64(A, B, nprod: int, C=None, ws=None, stream=None):
     ws = ws if ws is not None else workspace(emu_gemm_workspace_bytes(64, M, N, K), A.device)
     _check(emu_gemm_f64(M, N, K, A.data_ptr(), A.stride(0), B.data_ptr(), B.stride(0), C.data_ptr(), C.stride(0),
                         int(nprod), ws.data_ptr(), ws.numel(), _stream(stream)), "emu_gemm_f64")
+    return C, ws
+
+
+def gemm_f64_merged(A, B, nprod: int, merge_from: int, C=None, ws=None, stream=None):
+    """emu_gemm_f64_merged: Algorithm 2's head (i + j < merge_from) plus the
+    remaining products of S_d accumulated in one FP32 tail, added last."""
+    torch = _torch()
+    M, K = A.shape
+    N = B.shape[1]
+    C = C if C is not None else torch.empty((M, N), dtype=torch.float64, device=A.device)
+    ws = ws if ws is not None else workspace(emu_gemm_f64_merged_workspace_bytes(M, N, K), A.device)
+    _check(emu_gemm_f64_merged(M, N, K, A.data_ptr(), A.stride(0), B.data_ptr(), B.stride(0), C.data_ptr(),
+                               C.stride(0), int(nprod), int(merge_from), ws.data_ptr(), ws.numel(), _stream(stream)),
+           "emu_gemm_f64_merged")
     return C, ws
 
 

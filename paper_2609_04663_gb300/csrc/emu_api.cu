@@ -165,6 +165,42 @@ emu_status emu_gemm_f32_fused(int64_t M, int64_t N, int64_t K, const float *A, i
     return cuda_status(launch_gemm_f32_fused(M, N, K, A, lda, B, ldb, C, ldc, &h->flags, st));
 }
 
+size_t emu_gemm_f64_merged_workspace_bytes(int64_t M, int64_t N, int64_t K)
+{
+    if (M < 0 || N < 0 || K < 0) return 0;
+    return gemm_ws_bytes(6, M, N, K) + (size_t)round_up(M * N * 4, 256);
+}
+
+emu_status emu_gemm_f64_merged(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda, const double *B,
+                               int64_t ldb, double *C, int64_t ldc, int nprod, int merge_from, void *ws,
+                               size_t ws_bytes, emu_stream_t stream)
+{
+    emu_status s = check_gemm_dims(M, N, K, lda, ldb, ldc);
+    if (s != EMU_OK) return s;
+    const int d = nprod == 6 ? 3 : nprod == 10 ? 4 : nprod == 15 ? 5 : nprod == 21 ? 6 : 0;
+    if (d == 0 || merge_from < 3 || merge_from > d) return EMU_ERR_INVALID_ARG;
+    if (!ws || (M > 0 && N > 0 && (!C || (K > 0 && (!A || !B))))) return EMU_ERR_INVALID_ARG;
+    if (ws_bytes < emu_gemm_f64_merged_workspace_bytes(M, N, K)) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
+    if (e != cudaSuccess) return EMU_ERR_CUDA;
+    if (M == 0 || N == 0) return EMU_OK;
+    if (K == 0) return zero_c(C, M, N, ldc, st);
+    const int64_t ldk = gemm_ldk(K);
+    uint16_t *Ap = reinterpret_cast<uint16_t *>(static_cast<char *>(ws) + kWsHeaderBytes);
+    uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(6 * M * ldk * 2, 256));
+    float *T = merge_from < d ? reinterpret_cast<float *>(static_cast<char *>(ws) + gemm_ws_bytes(6, M, N, K)) : nullptr;
+    e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st);
+    if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st);
+    if (e == cudaSuccess && T) e = launch_prodsum_tail(M, N, K, Ap, Bp, ldk, merge_from, d, T, N, &h->flags, st);
+    if (e == cudaSuccess)
+        e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], merge_from * (merge_from + 1) / 2, C,
+                               ldc, gemm_acc(ws, M, N, K), &h->flags, st, 0, false, T, N);
+    return cuda_status(e);
+}
+
 emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda, const double *B,
                         int64_t ldb, double *C, int64_t ldc, int nprod, void *ws, size_t ws_bytes,
                         emu_stream_t stream)

@@ -1,6 +1,7 @@
 // Shared pieces of the tensor-core product-sum kernels: output-tile
-// rasterisation, the bounded drain of in-flight TMA copies, and the host-side
-// tensor-map encoding of a BF16 plane set.
+// rasterisation, the FP64 diagonal product order, the FP32 TMEM epilogue, the
+// bounded drain of in-flight TMA copies, and the host-side tensor-map
+// encoding of a BF16 plane set.
 #pragma once
 
 #include "common.cuh"
@@ -18,6 +19,45 @@ __device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, 
     const int local = tile % group_size;
     tm = first_m + local % gm;
     tn = local / gm;
+}
+
+// FP64 diagonal order (Algorithm 2): diagonal l = 0..5, i ascending, j = l - i.
+// The first 6 / 10 / 15 / 21 entries are the sets S_3 .. S_6.
+namespace {
+__constant__ int8_t kDiag[21][2] = {{0, 0}, {0, 1}, {1, 0}, {0, 2}, {1, 1}, {2, 0}, {0, 3},
+                                    {1, 2}, {2, 1}, {3, 0}, {0, 4}, {1, 3}, {2, 2}, {3, 1},
+                                    {4, 0}, {0, 5}, {1, 4}, {2, 3}, {3, 2}, {4, 1}, {5, 0}};
+}  // namespace
+
+// Epilogue of one warp: accumulator columns [c0, c1) of the warp's TMEM lane
+// quarter (tile rows quarter * 32 ..) -> C.
+__device__ __forceinline__ void store_tile(uint32_t tmem, int quarter, int c0, int c1, int m0, int n0, int M, int N,
+                                           float *__restrict__ C, int64_t ldc)
+{
+    tc_fence_after();
+    const int row = m0 + quarter * 32 + lane_id();
+    float *crow = C + (int64_t)row * ldc;
+    const bool vec = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15u) == 0);
+#pragma unroll 1
+    for (int c = c0; c < c1; c += 32) {
+        uint32_t v[32];
+        tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)c, v);
+        tmem_ld_wait();
+        const int col = n0 + c;
+        if (row < M) {
+            if (vec && col + 32 <= N) {
+#pragma unroll
+                for (int j = 0; j < 32; j += 4)
+                    *reinterpret_cast<float4 *>(crow + col + j) =
+                        make_float4(__uint_as_float(v[j]), __uint_as_float(v[j + 1]),
+                                    __uint_as_float(v[j + 2]), __uint_as_float(v[j + 3]));
+            } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    if (col + j < N) crow[col + j] = __uint_as_float(v[j]);
+            }
+        }
+    }
 }
 
 // Wait (bounded) for the TMA loads the producer issued that the MMA warp may

@@ -47,10 +47,18 @@ cudaError_t launch_gemm_f32_fused(int64_t M, int64_t N, int64_t K, const float *
                                   int64_t ldb, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st);
 // acc: FP64 accumulator scratch of f64_acc_bytes(M, N) bytes (16-byte aligned).
 // rowcol: vA / vB are levels per row of A ([6][M]) and per column of B ([6][N]).
+// T (optional, M x N FP32 with leading dimension ldt): a merged tail, added to
+// every element once after the last product.
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
                                int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane = 0,
-                               bool rowcol = false);
+                               bool rowcol = false, const float *T = nullptr, int64_t ldt = 0);
+// Merged tail of the FP64 mode: T (M x N FP32, leading dimension ldt) = the
+// sum over the products (i, j) with L <= i + j < d of A_i B_j, accumulated in
+// one FP32 tensor-memory accumulator over all of K; 3 <= L < d <= 6.
+cudaError_t launch_prodsum_tail(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
+                                int64_t ldcomp, int L, int d, float *T, int64_t ldt, uint32_t *flags,
+                                cudaStream_t st);
 
 // Bytes of the FP64 product-sum's accumulator: one 128 x 128 FP64 tile per CTA tile.
 inline size_t f64_acc_bytes(int64_t M, int64_t N)

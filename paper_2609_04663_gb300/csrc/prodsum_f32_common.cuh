@@ -1,6 +1,7 @@
 // Pieces shared by the FP32-mode product-sum kernels (the TMA-fed one and the
 // one that splits inside its producer): tile configuration, the MMA issue
-// loop of Eq. (fp32reuseorder) over a ring of stages, and the epilogue.
+// loop of Eq. (fp32reuseorder) over a ring of stages (the epilogue is
+// store_tile of gemm_common.cuh).
 #pragma once
 
 #include "gemm_common.cuh"
@@ -54,37 +55,6 @@ __device__ __forceinline__ void mma_loop(uint32_t tmem, uint32_t base, uint32_t 
     }
     mma_commit(accum_bar);                   // all MMAs issued so far are done
     (void)mbar_wait(accum_bar, 0, flags);
-}
-
-// Epilogue of one warp: accumulator columns [c0, c1) of the warp's TMEM lane
-// quarter (tile rows quarter * 32 ..) -> C.
-__device__ __forceinline__ void store_tile(uint32_t tmem, int quarter, int c0, int c1, int m0, int n0, int M, int N,
-                                           float *__restrict__ C, int64_t ldc)
-{
-    tc_fence_after();
-    const int row = m0 + quarter * 32 + lane_id();
-    float *crow = C + (int64_t)row * ldc;
-    const bool vec = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15u) == 0);
-#pragma unroll 1
-    for (int c = c0; c < c1; c += 32) {
-        uint32_t v[32];
-        tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)c, v);
-        tmem_ld_wait();
-        const int col = n0 + c;
-        if (row < M) {
-            if (vec && col + 32 <= N) {
-#pragma unroll
-                for (int j = 0; j < 32; j += 4)
-                    *reinterpret_cast<float4 *>(crow + col + j) =
-                        make_float4(__uint_as_float(v[j]), __uint_as_float(v[j + 1]),
-                                    __uint_as_float(v[j + 2]), __uint_as_float(v[j + 3]));
-            } else {
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    if (col + j < N) crow[col + j] = __uint_as_float(v[j]);
-            }
-        }
-    }
 }
 
 }  // namespace

@@ -40,12 +40,6 @@ namespace emu {
 
 namespace {
 
-// FP64 diagonal order (Algorithm 2): diagonal l = 0..5, i ascending, j = l - i.
-// The first 6 / 10 / 15 / 21 entries are the sets S_3 .. S_6.
-__constant__ int8_t kDiag[21][2] = {{0, 0}, {0, 1}, {1, 0}, {0, 2}, {1, 1}, {2, 0}, {0, 3},
-                                    {1, 2}, {2, 1}, {3, 0}, {0, 4}, {1, 3}, {2, 2}, {3, 1},
-                                    {4, 0}, {0, 5}, {1, 4}, {2, 3}, {3, 2}, {4, 1}, {5, 0}};
-
 struct F64Cfg {
     // A stage holds SUB K-blocks of 64 (one 128-byte swizzle row each) of the
     // A slice and of the B slice.
@@ -203,7 +197,8 @@ template <int NPROD, bool ROWCOL>
 __global__ void __launch_bounds__(F64Cfg::THREADS, 1)
 prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    int M, int N, int K, const int32_t *__restrict__ vA, const int32_t *__restrict__ vB,
-                   double *__restrict__ C, int64_t ldc, double *__restrict__ acc, uint32_t *flags)
+                   double *__restrict__ C, int64_t ldc, double *__restrict__ acc, uint32_t *flags,
+                   const float *__restrict__ T, int64_t ldt)
 {
     using Cfg = F64Cfg;
     extern __shared__ uint8_t smem_raw[];
@@ -401,6 +396,8 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
         double *tacc = acc + ((size_t)tm * tiles_n + tn) * (size_t)(kBM * Cfg::BN) + r;
         const int lim = row < M ? N - n0 : 0;
         const bool vec = ((ldc & 1) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15u) == 0);
+        // merged tail (when T is given): one more addition after the last product
+        const float *trow = T ? T + (int64_t)(row < M ? row : 0) * ldt + n0 : nullptr;
         for (int q = 0; q < NPROD; ++q) {
             const bool ok = mbar_wait(hfull, (uint32_t)(q & 1), flags);
             __syncwarp();
@@ -435,6 +432,11 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                     if (dg && col + j < lim) sq = __dadd_rn(sq, widen_exact(lrow[2 * (col + j)]));   // exact
                     out[j] = first ? sq : __dadd_rn(cur[j], sq);
                 }
+                if (last && trow) {
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        if (col + j < lim) out[j] = __dadd_rn(out[j], widen_exact(trow[col + j]));
+                }
                 if (!last) {
 #pragma unroll
                     for (int j = 0; j < 8; ++j) tacc[(col + j) * kBM] = out[j];
@@ -465,7 +467,7 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
 template <int NPROD, bool ROWCOL>
 cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
                     const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, double *acc, uint32_t *flags,
-                    cudaStream_t st, int64_t a_plane)
+                    cudaStream_t st, int64_t a_plane, const float *T, int64_t ldt)
 {
     using Cfg = F64Cfg;
     CUtensorMap ta, tb;
@@ -475,7 +477,8 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
     const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + Cfg::BN - 1) / Cfg::BN);
-    kern<<<(unsigned)tiles, Cfg::THREADS, Cfg::SMEM, st>>>(ta, tb, (int)M, (int)N, (int)K, vA, vB, C, ldc, acc, flags);
+    kern<<<(unsigned)tiles, Cfg::THREADS, Cfg::SMEM, st>>>(ta, tb, (int)M, (int)N, (int)K, vA, vB, C, ldc, acc, flags,
+                                                           T, ldt);
     return cudaGetLastError();
 }
 
@@ -484,17 +487,17 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
                                int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
-                               bool rowcol)
+                               bool rowcol, const float *T, int64_t ldt)
 {
     switch (nprod) {
-    case 6: return rowcol ? run_f64<6, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane)
-                   : run_f64<6, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
-    case 10: return rowcol ? run_f64<10, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane)
-                   : run_f64<10, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
-    case 15: return rowcol ? run_f64<15, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane)
-                   : run_f64<15, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
-    case 21: return rowcol ? run_f64<21, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane)
-                   : run_f64<21, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane);
+    case 6: return rowcol ? run_f64<6, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt)
+                   : run_f64<6, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
+    case 10: return rowcol ? run_f64<10, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt)
+                   : run_f64<10, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
+    case 15: return rowcol ? run_f64<15, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt)
+                   : run_f64<15, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
+    case 21: return rowcol ? run_f64<21, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt)
+                   : run_f64<21, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
     default: return cudaErrorInvalidValue;
     }
 }

@@ -64,6 +64,12 @@ def test_host_argument_checks_need_no_gpu(lib):
     assert emu.emu_gemm_f32(1 << 31, 4, 4, P, 4, P, 4, P, 4, P, 1 << 62, None) == 5  # size limit
     assert emu.emu_split_f64(P, 4, 4, 2, 0, P, 4, P, P, 4096, None) == 1              # ldx < cols
     assert emu.emu_selftest_timeout(P, 4096, 0, None) == 1
+    # merged FP64 tail: merge_from range and workspace size are checked on the host
+    assert emu.emu_gemm_f64_merged(4, 4, 4, P, 4, P, 4, P, 4, 21, 2, P, 1 << 30, None) == 1
+    assert emu.emu_gemm_f64_merged(4, 4, 4, P, 4, P, 4, P, 4, 10, 5, P, 1 << 30, None) == 1
+    assert emu.emu_gemm_f64_merged(4, 4, 4, P, 4, P, 4, P, 4, 21, 4, P, 16, None) == 3
+    assert emu.emu_gemm_f64_merged_workspace_bytes(300, 200, 700) == \
+        emu.emu_gemm_workspace_bytes(64, 300, 200, 700) + 300 * 200 * 4 + 128
     # the fused FP32 GEMM needs only the flag word
     assert emu.emu_gemm_f32_fused(4, 4, 4, P, 3, P, 4, P, 4, P, 512, None) == 1       # lda < K
     assert emu.emu_gemm_f32_fused(4, 4, 4, P, 4, P, 4, P, 4, P, 511, None) == 3       # workspace
