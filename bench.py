@@ -450,7 +450,7 @@ def gpu_arm(args, rank, world, local):
     __graft_entry__.build()
     pk = peaks()
     name = args.workload
-    case = Case(name, rank, args.nprod, fused=args.fused)
+    case = Case(name, rank, args.nprod, fused=args.fused, merge_from=args.merge_from)
     clocks = ClockSampler(local)
     clocks.start()
     res = time_device(case, args.steps, args.warmup, world, flush=False)
@@ -467,17 +467,18 @@ def gpu_arm(args, rank, world, local):
                 "peak_source": f"{pk['source']} bf16 burst (cuBLAS 8192^3); sustained {pk['bf16_sustained']}",
                 "kernel": "gemm_f32_fused_kernel" if case.fused else
                           "prodsum_f32_kernel" if case.mode == 32 else "prodsum_f64_kernel",
-                "traffic": None if case.fused else
+                "traffic": None if case.fused or case.merge_from else
                            kernel_traffic("prodsum_f32" if case.mode == 32 else "prodsum_f64",
                                           name if case.mode == 32 else f"{name}_np{case.nprod}")}
-    flags = case.emu.read_flags(case.ws)
+    flags = case.emu.read_flags(case.gemm_ws if case.gemm_ws is not None else case.ws)
     e2e = None if args.no_e2e else time_e2e(case, max(2, min(args.steps, 5)), 1, world)
     split_gbs = case.split_bytes() / (split_ms / 1e3) / 1e9
     line = {
         "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * t_job / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": name, "mode": f"fp{case.mode}" + ("_fused" if case.fused else ""), "nprod": case.nprod if case.mode == 64 else 6,
+        "config": {"workload": name, "mode": f"fp{case.mode}" + ("_fused" if case.fused else "") +
+                   (f"_merged{case.merge_from}" if case.merge_from else ""), "nprod": case.nprod if case.mode == 64 else 6,
                    "M": case.M, "N": case.N, "K": case.K, "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (no flush needed)"},
         "breakdown": {"split_ms": split_ms, "prodsum_ms": prod_ms, "split_gbs": split_gbs,
@@ -540,6 +541,8 @@ def main(argv=None):
     ap.add_argument("--nprod", type=int, default=None, help="FP64 product count (6, 10, 15, 21)")
     ap.add_argument("--fused", action="store_true",
                     help="FP32 workloads: time emu_gemm_f32_fused (split inside the product-sum) as the step")
+    ap.add_argument("--merge-from", type=int, default=None,
+                    help="FP64 workloads: time emu_gemm_f64_merged with the tail from this diagonal as the step")
     ap.add_argument("--variant-steps", type=int, default=5)
     ap.add_argument("--all-variants", action="store_true")
     ap.add_argument("--no-variants", action="store_true")
