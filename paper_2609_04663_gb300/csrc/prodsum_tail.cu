@@ -18,8 +18,7 @@
 //
 // What bounds it: with two stages, about one stage of copies is in flight
 // while the other is multiplied, and at the loaded L2 latency (about 1.4 us)
-// that delivers some 66 GB/s per SM, enough for 0.6 of the tensor peak at
-// 11 products per 12 tiles.  Wider tiles need 16-wide K-blocks to fit three
+// that keeps the tensor pipe about 63 % busy at 11 products per 12 tiles.  Wider tiles need 16-wide K-blocks to fit three
 // stages, and TMA copies of 32-byte rows were slower still (measured).
 #include "gemm_common.cuh"
 #include "launchers.cuh"
