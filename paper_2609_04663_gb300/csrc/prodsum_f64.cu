@@ -193,7 +193,8 @@ __device__ __forceinline__ float two_sum(float a, float b, float &e)
     return s;
 }
 
-template <int NPROD, bool ROWCOL>
+// TAIL: add the merged tail T (an M x N FP32 matrix) once after the last product.
+template <int NPROD, bool ROWCOL, bool TAIL>
 __global__ void __launch_bounds__(F64Cfg::THREADS, 1)
 prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    int M, int N, int K, const int32_t *__restrict__ vA, const int32_t *__restrict__ vB,
@@ -314,6 +315,11 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
             const float bound = ROWCOL ? exact_bound_rowcol(vA, vB, M, N, kDiag[q][0], kDiag[q][1], row,
                                                             n0 + cq * Cfg::COLS, Cfg::COLS)
                                        : exact_bound(vA, vB, kDiag[q][0], kDiag[q][1]);
+            // Carry instead of TwoSums when all elements share the unit u = 2^-24 bound
+            // (levels per matrix) and the split constant 1.5 * 2^35 u is finite:
+            // the coarse part (multiples of 2^12 u) moves to the low word in C and
+            // stays exact below 2^36 u, i.e. for up to 2^11 chunks of at most 2^25 u.
+            const bool carry = !ROWCOL && bound > 0.0f && bound <= 0x1p116f && nch <= 2048;
             for (int c = 0; c < nch; ++c) {
                 const int t = q * nch + c, b = t % Cfg::NBUF;
                 ok = mbar_wait(tfull0 + 8u * b, (uint32_t)((t / Cfg::NBUF) & 1), flags);
@@ -336,6 +342,28 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                     if (!__any_sync(0xFFFFFFFFu, big)) {
 #pragma unroll
                         for (int j = 0; j < 16; ++j) hi[h + j] = __uint_as_float(v[j]);
+                    } else if (carry) {
+                        // rare: some sum would reach 2^24 u.  Split the running sum and
+                        // the partial (read again from TMEM: the buffer is not yet
+                        // released) at multiples of 2^12 u by the add-subtract
+                        // projection; the coarse parts go to the low word in C, the
+                        // remainders (below 2^12 u) restart the running sum.  All exact.
+                        const bool was = (dirty >> (h / 16)) & 1u;
+                        dirty |= 1u << (h / 16);
+                        const float cm = 3072.0f * bound;         // 1.5 * 2^35 u
+                        float *lrow = reinterpret_cast<float *>(crow) + (q & 1);
+#pragma unroll
+                        for (int jj = 0; jj < 16; ++jj) {
+                            const int j = h + jj;
+                            const float p = __uint_as_float(tmem_ld1(taddr + (uint32_t)jj));
+                            tmem_ld_wait();
+                            const float h1 = __fsub_rn(__fadd_rn(hi[j], cm), cm), l1 = __fsub_rn(hi[j], h1);
+                            const float h2 = __fsub_rn(__fadd_rn(p, cm), cm), l2 = __fsub_rn(p, h2);
+                            const bool mine = j < lim;
+                            const float s2 = __fadd_rn((was && mine) ? lrow[2 * j] : 0.0f, __fadd_rn(h1, h2));
+                            hi[j] = __fadd_rn(l1, l2);
+                            if (mine) lrow[2 * j] = s2;
+                        }
                     } else {
                         // rare: redo the 16 additions as TwoSums, the errors summed
                         // exactly into the low part; the partials are read again from
@@ -396,8 +424,8 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
         double *tacc = acc + ((size_t)tm * tiles_n + tn) * (size_t)(kBM * Cfg::BN) + r;
         const int lim = row < M ? N - n0 : 0;
         const bool vec = ((ldc & 1) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15u) == 0);
-        // merged tail (when T is given): one more addition after the last product
-        const float *trow = T ? T + (int64_t)(row < M ? row : 0) * ldt + n0 : nullptr;
+        // merged tail: one more addition after the last product
+        const float *trow = TAIL ? T + (int64_t)(row < M ? row : 0) * ldt + n0 : nullptr;
         for (int q = 0; q < NPROD; ++q) {
             const bool ok = mbar_wait(hfull, (uint32_t)(q & 1), flags);
             __syncwarp();
@@ -431,11 +459,7 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                     double sq = widen_exact(__uint_as_float(hv[j]));
                     if (dg && col + j < lim) sq = __dadd_rn(sq, widen_exact(lrow[2 * (col + j)]));   // exact
                     out[j] = first ? sq : __dadd_rn(cur[j], sq);
-                }
-                if (last && trow) {
-#pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        if (col + j < lim) out[j] = __dadd_rn(out[j], widen_exact(trow[col + j]));
+                    if (TAIL && last && col + j < lim) out[j] = __dadd_rn(out[j], widen_exact(trow[col + j]));
                 }
                 if (!last) {
 #pragma unroll
@@ -464,7 +488,7 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     }
 }
 
-template <int NPROD, bool ROWCOL>
+template <int NPROD, bool ROWCOL, bool TAIL = false>
 cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
                     const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, double *acc, uint32_t *flags,
                     cudaStream_t st, int64_t a_plane, const float *T, int64_t ldt)
@@ -473,7 +497,7 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
     CUtensorMap ta, tb;
     if (!make_plane_map(&ta, Ap, K, M, 6, ldcomp, Cfg::KB, kBM, a_plane) || !make_plane_map(&tb, Bp, K, N, 6, ldcomp, Cfg::KB, Cfg::BN))
         return cudaErrorInvalidValue;
-    auto kern = prodsum_f64_kernel<NPROD, ROWCOL>;
+    auto kern = prodsum_f64_kernel<NPROD, ROWCOL, TAIL>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
     const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + Cfg::BN - 1) / Cfg::BN);
@@ -489,15 +513,24 @@ cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *
                                int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
                                bool rowcol, const float *T, int64_t ldt)
 {
+    if (T) {                                          // merged tail: whole-matrix levels only
+        if (rowcol) return cudaErrorInvalidValue;
+        switch (nprod) {
+        case 6: return run_f64<6, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
+        case 10: return run_f64<10, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
+        case 15: return run_f64<15, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
+        default: return cudaErrorInvalidValue;
+        }
+    }
     switch (nprod) {
-    case 6: return rowcol ? run_f64<6, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt)
-                   : run_f64<6, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
-    case 10: return rowcol ? run_f64<10, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt)
-                   : run_f64<10, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
-    case 15: return rowcol ? run_f64<15, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt)
-                   : run_f64<15, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
-    case 21: return rowcol ? run_f64<21, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt)
-                   : run_f64<21, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
+    case 6: return rowcol ? run_f64<6, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0)
+                   : run_f64<6, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
+    case 10: return rowcol ? run_f64<10, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0)
+                   : run_f64<10, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
+    case 15: return rowcol ? run_f64<15, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0)
+                   : run_f64<15, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
+    case 21: return rowcol ? run_f64<21, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0)
+                   : run_f64<21, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
     default: return cudaErrorInvalidValue;
     }
 }

@@ -177,6 +177,20 @@ def test_prodsum_f64_error_free_path_at_the_2pow24_edge(dev):
         assert np.all(C.cpu().numpy() == want)
 
 
+@pytest.mark.parametrize("nprod", [6, 21])
+def test_gemm_f64_long_k_positive_sums(dev, nprod):
+    """Positive inputs: every product's running sum grows linearly, passes
+    2^24 units within a few chunks and keeps moving its coarse part into the
+    low word (40 chunks of K, ragged tiles); still bit for bit."""
+    M, N, K = 130, 200, 256 * 40 + 17
+    rng = np.random.default_rng(31)
+    A = rng.uniform(0.5, 1.0, size=(M, K))
+    B = rng.uniform(0.5, 1.0, size=(K, N))
+    C, ws = emu.gemm_f64(to_dev(A, dev), to_dev(B, dev), nprod)
+    assert emu.read_flags(ws) == 0
+    assert np.array_equal(C.cpu().numpy(), oracle.gemm_f64(A, B, nprod)[0])
+
+
 # ------------------------------------------------------------ edges, errors
 def test_zero_sizes_and_empty_k(dev):
     torch = emu._torch()
