@@ -86,6 +86,10 @@ prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     }
 }
 
+// Per-SM rates of the narrower tiles relative to 128 x 256 (measured at 8192^3:
+// 274 and 164 against 316 TFLOP/s for the whole GEMM).
+constexpr double kRate128 = 0.87, kRate64 = 0.52;
+
 template <int BN, int KB, int STAGES>
 cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
                     float *C, int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane, int64_t b_plane)
@@ -105,18 +109,42 @@ cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
 
 }  // namespace
 
-// FP32 tile shape: 128 x 256 with 32-wide K-blocks (64-byte swizzle, 3 stages)
-// by default; EMU_F32_TILE=128x128 selects 128 x 128 with 64-wide K-blocks
-// (128-byte swizzle, 2 stages).
+// FP32 tile shape.  128 x 256 with 32-wide K-blocks (64-byte swizzle, three
+// stages) is the fastest per SM; 128 x 128 (64-wide K-blocks, 128-byte
+// swizzle, two stages) and 128 x 64 (64-wide K-blocks, three stages) reach
+// smaller fractions of it but give more CTAs, which pays when there are too
+// few 128 x 256 tiles to fill the GPU.  The choice maximises (SMs kept busy
+// over the waves) x (relative per-SM rate).  Every shape issues the same MMAs
+// in the same order for each output element, so C does not depend on it.
+// EMU_F32_TILE=128x256 / 128x128 / 128x64 forces one.
 cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
                                int64_t a_plane, int64_t b_plane)
 {
-    static const bool narrow = [] {
+    static const int forced = [] {
         const char *e = std::getenv("EMU_F32_TILE");
-        return e && e[0] == '1' && e[1] == '2' && e[2] == '8' && e[3] == 'x' && e[4] == '1';
+        if (!e || e[0] != '1' || e[1] != '2' || e[2] != '8' || e[3] != 'x') return 0;
+        return (e[4] == '2' && e[5] == '5' && e[6] == '6') ? 256 : (e[4] == '1' && e[5] == '2' && e[6] == '8') ? 128
+               : (e[4] == '6' && e[5] == '4') ? 64 : 0;
     }();
-    if (narrow) return run_f32<128, 64, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
+    int bn = forced;
+    if (bn == 0) {
+        int dev = 0, sms = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+            sms = 152;
+        const int widths[3] = {256, 128, 64};
+        const double rate[3] = {1.0, kRate128, kRate64};
+        double best = -1.0;
+        for (int i = 0; i < 3; ++i) {
+            const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + widths[i] - 1) / widths[i]);
+            const int64_t waves = (tiles + sms - 1) / sms;
+            const double score = rate[i] * (double)tiles / (double)(waves * sms);
+            if (score > best * 1.02) { best = score; bn = widths[i]; }   // prefer the wider tile on near ties
+        }
+    }
+    if (bn == 128) return run_f32<128, 64, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
+    if (bn == 64) return run_f32<64, 64, 3>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
     return run_f32<256, 32, 3>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
 }
 
