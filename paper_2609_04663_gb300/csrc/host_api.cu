@@ -4,10 +4,10 @@
 // and the copy of C back to the host are pipelined over panels on internal
 // streams, so that the host link and the GPU work at the same time:
 //
-//   FP32: the first two row panels of A arrive, then B in column panels; as
-//   each column panel lands it is split and both leading row panels multiply
-//   it (one block of C each, on the two compute streams), so the GPU works
-//   while B streams in.  The remaining row panels of A then arrive, are split
+//   FP32: the first row panel of A arrives, then B's first column panel, A's
+//   second row panel and the rest of B in column panels; as each column panel
+//   lands it is split and both leading row panels multiply it (one block of C
+//   each, on the two compute streams), so the GPU works while B streams in.  The remaining row panels of A then arrive, are split
 //   and multiplied with all of B.  Every finished row panel of C goes back
 //   while the next one is computed; row panels alternate between the two
 //   compute streams so that one panel's last wave of CTAs overlaps the next.
@@ -240,9 +240,11 @@ emu_status emu_gemm_f32_host(int64_t M, int64_t N, int64_t K, const float *A, in
     };
 
     // the leading row panels, then B column by column, each column panel
-    // multiplied by the leading row panels as soon as it is split
+    // multiplied by the leading row panels as soon as it is split.  Copy
+    // order: A row panel 0, B column panel 0, A row panel 1, then the rest of
+    // B, so that the first product-sum waits for two copies, not three.
     const int64_t lead = g.PM < 2 ? g.PM : 2;
-    for (int64_t i = 0; i < lead && e == cudaSuccess; ++i) e = load_a(i, cx->comp[i]);
+    if (e == cudaSuccess) e = load_a(0, cx->comp[0]);
     cudaEvent_t bsplit[kPanelsN] = {};
     for (int64_t j = 0; j < g.PN && e == cudaSuccess; ++j) {
         const int64_t n0 = j * g.Nb, nb = (N - n0 < g.Nb) ? N - n0 : g.Nb;
@@ -253,6 +255,7 @@ emu_status emu_gemm_f32_host(int64_t M, int64_t N, int64_t K, const float *A, in
                                   cudaMemcpyHostToDevice, cx->cin);
         cudaEvent_t landed = cx->ev[ne++];
         if (e == cudaSuccess) e = cudaEventRecord(landed, cx->cin);
+        if (e == cudaSuccess && j == 0 && lead > 1) e = load_a(1, cx->comp[1]);
         if (e == cudaSuccess) e = cudaStreamWaitEvent(cx->comp[0], landed, 0);
         if (e == cudaSuccess) e = launch_split_f32(bs, K, nb, nb, true, Bp + n0 * g.ldk, g.ldk, h, cx->comp[0], b_plane);
         bsplit[j] = cx->ev[ne++];
