@@ -239,10 +239,12 @@ class Case:
             r |= emu.emu_split_f32(self.B.data_ptr(), self.K, self.N, self.B.stride(0), 1, self.Bp.data_ptr(),
                                    self.ldk, ws, n, st)
         else:
-            r = emu.emu_split_f64(self.A.data_ptr(), self.M, self.K, self.A.stride(0), 0, self.Ap.data_ptr(),
-                                  self.ldk, self.v.data_ptr(), ws, n, st)
-            r |= emu.emu_split_f64(self.B.data_ptr(), self.K, self.N, self.B.stride(0), 1, self.Bp.data_ptr(),
-                                   self.ldk, self.v.data_ptr() + 24, ws, n, st)
+            # only the d slices the product-sum reads (d = 3, 4, 5, 6 for nprod = 6, 10, 15, 21)
+            d = {6: 3, 10: 4, 15: 5, 21: 6}[self.nprod]
+            r = emu.emu_split_f64_slices(self.A.data_ptr(), self.M, self.K, self.A.stride(0), 0, self.Ap.data_ptr(),
+                                         self.ldk, d, self.v.data_ptr(), ws, n, st)
+            r |= emu.emu_split_f64_slices(self.B.data_ptr(), self.K, self.N, self.B.stride(0), 1, self.Bp.data_ptr(),
+                                          self.ldk, d, self.v.data_ptr() + 24, ws, n, st)
         assert r == 0, r
 
     def prodsum(self, stream):

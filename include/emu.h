@@ -136,6 +136,18 @@ emu_status emu_gemm_f64_rowcol(int64_t M, int64_t N, int64_t K, const double *A,
  * the flag word plus the slice planes of A (M x K) and B (K x N), and in
  * mode 64 the product-sum's FP64 accumulator (8 bytes per element of C,
  * rounded up to 128 x 128 tiles). */
+/* emu_split_f64 for a product-sum that reads slices 0 .. nslices-1 only
+ * (nslices = d = 3, 4, 5, 6 for nprod = 6, 10, 15, 21): the fused pass forms
+ * and writes only those planes, and only their levels are verified.  Planes
+ * 0 .. nslices-1 and v_out[0 .. nslices-1] equal emu_split_f64's; planes and
+ * levels from nslices on are unspecified (left as they were, or formed
+ * literally when a speculative level below nslices failed).  The GEMM entry
+ * points split this way.  Errors as emu_split_f64; EMU_ERR_INVALID_ARG also
+ * for nslices outside 3 .. 6. */
+emu_status emu_split_f64_slices(const double *X, int64_t rows, int64_t cols, int64_t ldx, int transpose,
+                                uint16_t *comps, int64_t ldcomp, int nslices, int32_t *v_out, void *ws,
+                                size_t ws_bytes, emu_stream_t stream);
+
 size_t emu_gemm_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K);
 
 /* FP32-mode emulated GEMM, Algorithm 1: C (M x N, ldc) = A (M x K, lda) . B

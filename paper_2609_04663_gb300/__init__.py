@@ -31,6 +31,7 @@ _SIGS = {
     "emu_split_workspace_bytes": ("size", ["i"]),
     "emu_split_f32": ("i", ["p", "l", "l", "l", "i", "p", "l", "p", "size", "p"]),
     "emu_split_f64": ("i", ["p", "l", "l", "l", "i", "p", "l", "p", "p", "size", "p"]),
+    "emu_split_f64_slices": ("i", ["p", "l", "l", "l", "i", "p", "l", "i", "p", "p", "size", "p"]),
     "emu_gemm_workspace_bytes": ("size", ["i", "l", "l", "l"]),
     "emu_gemm_f32": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "p", "size", "p"]),
     "emu_gemm_f64": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "size", "p"]),
@@ -96,6 +97,7 @@ def _mk(name):
 emu_split_workspace_bytes = _mk("emu_split_workspace_bytes")
 emu_split_f32 = _mk("emu_split_f32")
 emu_split_f64 = _mk("emu_split_f64")
+emu_split_f64_slices = _mk("emu_split_f64_slices")
 emu_gemm_workspace_bytes = _mk("emu_gemm_workspace_bytes")
 emu_gemm_f32 = _mk("emu_gemm_f32")
 emu_gemm_f64 = _mk("emu_gemm_f64")
@@ -168,8 +170,9 @@ def split_f32(X, transpose: bool = False, ldcomp: int | None = None, ws=None, st
     return planes, ws
 
 
-def split_f64(X, transpose: bool = False, ldcomp: int | None = None, ws=None, stream=None):
-    """Eq. (fp64split) on the GPU: returns (planes int16 [6, rows_out, ldcomp], v int32[6] (device), ws)."""
+def split_f64(X, transpose: bool = False, ldcomp: int | None = None, ws=None, stream=None, nslices: int = 6):
+    """Eq. (fp64split) on the GPU: returns (planes int16 [6, rows_out, ldcomp], v int32[6] (device), ws).
+    nslices < 6 calls emu_split_f64_slices (planes and levels from nslices on unspecified)."""
     torch = _torch()
     rows, cols = X.shape
     rows_out, cols_out = (cols, rows) if transpose else (rows, cols)
@@ -177,8 +180,13 @@ def split_f64(X, transpose: bool = False, ldcomp: int | None = None, ws=None, st
     planes = torch.zeros((6, rows_out, ldcomp), dtype=torch.int16, device=X.device)
     v = torch.empty(6, dtype=torch.int32, device=X.device)
     ws = ws if ws is not None else workspace(emu_split_workspace_bytes(64), X.device)
-    _check(emu_split_f64(X.data_ptr(), rows, cols, X.stride(0), int(transpose), planes.data_ptr(), ldcomp,
-                         v.data_ptr(), ws.data_ptr(), ws.numel(), _stream(stream)), "emu_split_f64")
+    if nslices == 6:
+        _check(emu_split_f64(X.data_ptr(), rows, cols, X.stride(0), int(transpose), planes.data_ptr(), ldcomp,
+                             v.data_ptr(), ws.data_ptr(), ws.numel(), _stream(stream)), "emu_split_f64")
+    else:
+        _check(emu_split_f64_slices(X.data_ptr(), rows, cols, X.stride(0), int(transpose), planes.data_ptr(), ldcomp,
+                                    int(nslices), v.data_ptr(), ws.data_ptr(), ws.numel(), _stream(stream)),
+               "emu_split_f64_slices")
     return planes, v, ws
 
 

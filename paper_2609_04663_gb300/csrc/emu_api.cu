@@ -119,6 +119,24 @@ emu_status emu_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ld
     return cuda_status(e);
 }
 
+emu_status emu_split_f64_slices(const double *X, int64_t rows, int64_t cols, int64_t ldx, int transpose,
+                                uint16_t *comps, int64_t ldcomp, int nslices, int32_t *v_out, void *ws,
+                                size_t ws_bytes, emu_stream_t stream)
+{
+    if (nslices < 3 || nslices > 6) return EMU_ERR_INVALID_ARG;
+    if (rows < 0 || cols < 0 || ldx < (cols > 0 ? cols : 1) || !ws || !v_out) return EMU_ERR_INVALID_ARG;
+    if (ldcomp < (transpose ? rows : cols) || ldcomp < 1) return EMU_ERR_INVALID_ARG;
+    if (rows > 0 && cols > 0 && (!X || !comps)) return EMU_ERR_INVALID_ARG;
+    if (ws_bytes < kWsHeaderBytes) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
+    if (e == cudaSuccess)
+        e = launch_split_f64(X, rows, cols, ldx, transpose != 0, comps, ldcomp, v_out, h, 0, st, nslices);
+    return cuda_status(e);
+}
+
 size_t emu_gemm_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K)
 {
     if (M < 0 || N < 0 || K < 0) return 0;
@@ -192,8 +210,10 @@ emu_status emu_gemm_f64_merged(int64_t M, int64_t N, int64_t K, const double *A,
     uint16_t *Ap = reinterpret_cast<uint16_t *>(static_cast<char *>(ws) + kWsHeaderBytes);
     uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(6 * M * ldk * 2, 256));
     float *T = merge_from < d ? reinterpret_cast<float *>(static_cast<char *>(ws) + gemm_ws_bytes(6, M, N, K)) : nullptr;
-    e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st);
-    if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st);
+    // the product-sum uses slices 0 .. d-1 only
+    const int nlev = nprod == 6 ? 3 : nprod == 10 ? 4 : nprod == 15 ? 5 : 6;
+    e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st, nlev);
+    if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st, nlev);
     if (e == cudaSuccess && T) e = launch_prodsum_tail(M, N, K, Ap, Bp, ldk, merge_from, d, T, N, &h->flags, st);
     if (e == cudaSuccess)
         e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], merge_from * (merge_from + 1) / 2, C,
@@ -220,8 +240,10 @@ emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_
     const int64_t ldk = gemm_ldk(K);
     uint16_t *Ap = reinterpret_cast<uint16_t *>(static_cast<char *>(ws) + kWsHeaderBytes);
     uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(6 * M * ldk * 2, 256));
-    e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st);
-    if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st);
+    // the product-sum uses slices 0 .. d-1 only
+    const int nlev = nprod == 6 ? 3 : nprod == 10 ? 4 : nprod == 15 ? 5 : 6;
+    e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st, nlev);
+    if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st, nlev);
     if (e == cudaSuccess)
         e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, C, ldc, gemm_acc(ws, M, N, K),
                                &h->flags, st);
@@ -284,8 +306,9 @@ emu_status gemm_ex(int opA, int opB, int64_t M, int64_t N, int64_t K, T alpha, c
         const bool ta = opA == EMU_OP_T, tb = opB == EMU_OP_N;
         const int64_t ar = ta ? K : M, ac = ta ? M : K, br = tb ? K : N, bc = tb ? N : K;
         if constexpr (f64) {
-            e = launch_split_f64(A, ar, ac, lda, ta, Ap, ldk, h->vout[0], h, 0, st);
-            if (e == cudaSuccess) e = launch_split_f64(B, br, bc, ldb, tb, Bp, ldk, h->vout[1], h, 1, st);
+            const int nlev = nprod == 6 ? 3 : nprod == 10 ? 4 : nprod == 15 ? 5 : 6;   // slices the product-sum uses
+            e = launch_split_f64(A, ar, ac, lda, ta, Ap, ldk, h->vout[0], h, 0, st, nlev);
+            if (e == cudaSuccess) e = launch_split_f64(B, br, bc, ldb, tb, Bp, ldk, h->vout[1], h, 1, st, nlev);
             if (e == cudaSuccess)
                 e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, out, ldo,
                                        gemm_acc(ws, M, N, K), &h->flags, st);

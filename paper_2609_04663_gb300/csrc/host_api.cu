@@ -289,6 +289,7 @@ emu_status emu_gemm_f64_host(int64_t M, int64_t N, int64_t K, const double *A, i
                              emu_stream_t stream)
 {
     if (nprod != 6 && nprod != 10 && nprod != 15 && nprod != 21) return EMU_ERR_INVALID_ARG;
+    const int nlev = nprod == 6 ? 3 : nprod == 10 ? 4 : nprod == 15 ? 5 : 6;   // slices the product-sum uses
     emu_status s = check_args(M, N, K, A, lda, B, ldb, C, ldc, ws, ws_bytes, 64);
     if (s != EMU_OK) return s;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -320,9 +321,11 @@ emu_status emu_gemm_f64_host(int64_t M, int64_t N, int64_t K, const double *A, i
                                   cudaMemcpyHostToDevice, cx->cin);
         if (e == cudaSuccess) e = cudaEventRecord(b_in, cx->cin);
         if (e == cudaSuccess) e = cudaStreamWaitEvent(cx->comp[0], a_in, 0);
-        if (e == cudaSuccess) e = launch_split_f64(Ast, M, K, K, false, Ap, g.ldk, h->vout[0], h, 0, cx->comp[0]);
+        if (e == cudaSuccess)
+            e = launch_split_f64(Ast, M, K, K, false, Ap, g.ldk, h->vout[0], h, 0, cx->comp[0], nlev);
         if (e == cudaSuccess) e = cudaStreamWaitEvent(cx->comp[0], b_in, 0);
-        if (e == cudaSuccess) e = launch_split_f64(Bst, K, N, N, true, Bp, g.ldk, h->vout[1], h, 1, cx->comp[0]);
+        if (e == cudaSuccess)
+            e = launch_split_f64(Bst, K, N, N, true, Bp, g.ldk, h->vout[1], h, 1, cx->comp[0], nlev);
         if (e == cudaSuccess) e = cudaEventRecord(split, cx->comp[0]);
         if (e == cudaSuccess) e = cudaStreamWaitEvent(cx->comp[1], split, 0);
     }

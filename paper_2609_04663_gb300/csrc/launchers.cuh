@@ -13,10 +13,14 @@ cudaError_t launch_split_f32(const float *X, int64_t rows, int64_t cols, int64_t
                              uint16_t *comps, int64_t ldcomp, WsHeader *ws, cudaStream_t st, int64_t plane = 0);
 
 // Eq. (fp64split): X -> 6 BF16 planes and the level exponents v_out[6]; `slot`
-// selects the header's per-operand state (0 = A, 1 = B).
+// selects the header's per-operand state (0 = A, 1 = B).  nlev (3..6): only
+// slices 0 .. nlev-1 are wanted (a product-sum with d = nlev uses no more);
+// planes from nlev on are then left as they were and their levels read as
+// zero levels, unless the speculative levels failed and the literal passes
+// redid all six.
 cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
                              uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
-                             cudaStream_t st);
+                             cudaStream_t st, int nlev = 6);
 
 // Eq. (fp64split) with one set of levels per plane row (an input row, or an
 // input column when transposed): v_out[6][plane rows] (level-major);
@@ -26,7 +30,8 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
 // cooperative launch after the speculative pass), and its form for an empty
 // matrix.
 cudaError_t launch_f64_fix(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose, uint16_t *comps,
-                           int64_t ldcomp, int64_t plane, WsHeader *ws, int slot, int32_t *v_out, cudaStream_t st);
+                           int64_t ldcomp, int64_t plane, WsHeader *ws, int slot, int32_t *v_out, cudaStream_t st,
+                           int nlev);
 cudaError_t launch_f64_fix_empty(WsHeader *ws, int slot, int32_t *v_out, cudaStream_t st);
 cudaError_t launch_split_f64_rc(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
                                 uint16_t *comps, int64_t ldcomp, int32_t *v_out, void *scratch, WsHeader *ws,

@@ -457,13 +457,18 @@ f64_max_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t
 }
 
 // One thread: checks the speculative levels in order.  Level r's max from
-// the fused pass is literal as long as levels < r were right, so the first
-// mismatch r gives the true v^(r) directly; levels after r are redone.  A
+// the fused pass is literal as long as levels < r were right and it spans
+// at least two units 2^(v0 - 50) of the fixed point (below that the sticky
+// bit of the truncated residual decides its power of two), so the first
+// mismatch r gives the true v^(r) directly when v^(r) >= v0 - 48 and levels
+// after r are redone; a smaller one is redone from level r itself.  A
 // slice outside the BF16 normal range at level r (a domain violation, which
 // the finalizer flags) also ends the trusted levels at r: the fused pass
 // subtracts the exact projection Z there, while Eq. (fp64split) subtracts
 // fl_BF16(Z), so the literal passes redo the levels after r.
-__device__ __forceinline__ int f64_verify_levels(const WsHeader *ws, int slot, int (&v)[6])
+// Only levels below nlev are checked (the speculative pass formed no more);
+// later ones are reported as zero levels.
+__device__ __forceinline__ int f64_verify_levels(const WsHeader *ws, int slot, int (&v)[6], int nlev = 6)
 {
     int ff = 6;
     const uint32_t sb = ws->slice_bad[slot] & 0x3Fu;
@@ -478,12 +483,13 @@ __device__ __forceinline__ int f64_verify_levels(const WsHeader *ws, int slot, i
         if (badlvl == 0) ff = 0;
         bool zero = false;
         for (int r = 1; r < 6 && ff == 6; ++r) {
-            if (zero) { v[r] = kZeroLevel; continue; }
+            if (zero || r >= nlev) { v[r] = kZeroLevel; continue; }
             const unsigned long long m = ws->maxbits[slot][r];
             if (m == 0) { v[r] = kZeroLevel; zero = true; continue; }
             const int vr = ceil_log2_bits(m);
             v[r] = vr;
-            if (vr != v0 - 8 * r || r == badlvl) ff = r;
+            if (r == badlvl) ff = r;
+            else if (vr != v0 - 8 * r) ff = vr >= v0 - 48 ? r : r - 1;
         }
     }
     return ff;
@@ -575,6 +581,7 @@ __device__ __forceinline__ void spec_units(int F, float (&P)[6])
     for (int r = 1; r < 6; ++r) P[r] = __fmul_rn(P[r - 1], 0.00390625f);          // 2^-8
 }
 
+template <int NLEV>
 __device__ __forceinline__ void spec_levels_fast(double x, int F, const float (&P)[6], uint32_t (&s)[6],
                                                  uint32_t &badmask, unsigned long long &m1, unsigned long long &m2,
                                                  uint32_t (&m)[3])
@@ -634,6 +641,7 @@ __device__ __forceinline__ void spec_levels_fast(double x, int F, const float (&
         Y = rem + up * ((uint32_t)d + lsb);
         sg ^= up;
     }
+    if constexpr (NLEV <= 3) return;                   // levels from NLEV on are not wanted
     // level 3: |X| <= 2^26, grid 2^19 / 2^18
     {
         m[0] = Y > m[0] ? Y : m[0];
@@ -647,12 +655,14 @@ __device__ __forceinline__ void spec_levels_fast(double x, int F, const float (&
         Y = rem + up * ((uint32_t)d + lsb);
         sg ^= up;
     }
+    if constexpr (NLEV <= 4) return;
     // levels 4, 5: |X| <= 2^18, exact in FP32; the add-subtract projection
     // with C = 1.5 * 2^(23 + g) rounds to the grid 2^g to nearest, ties to even
     float y = __fsub_rn(__uint_as_float(0x4B000000u | Y), 8388608.0f);
     y = sg ? -y : y;
 #pragma unroll
     for (int r = 4; r < 6; ++r) {
+        if (r >= NLEV) break;
         const float ay = fabsf(y);
         m[r - 3] = max(m[r - 3], (uint32_t)ay);                   // exact: an integer below 2^24
         const float C = (y < 0.0f) ? (r == 4 ? 12884901888.0f : 50331648.0f)      // 1.5 * 2^33, 1.5 * 2^25
@@ -670,6 +680,8 @@ struct SpecState {
     uint32_t badmask = 0;
 };
 
+// Slices 0 .. NLEV-1 of one entry (NLEV = 3..6; later ones are not formed).
+template <int NLEV = 6>
 __device__ __forceinline__ void spec_element(double x, int v0, bool fast, const float (&P)[6], uint32_t (&s)[6],
                                              SpecState &st)
 {
@@ -677,7 +689,7 @@ __device__ __forceinline__ void spec_element(double x, int v0, bool fast, const 
 #pragma unroll
         for (int r = 0; r < 6; ++r) s[r] = 0;
     } else if (fast) {
-        spec_levels_fast(x, v0 - 50, P, s, st.badmask, st.m1, st.m2, st.m);
+        spec_levels_fast<NLEV>(x, v0 - 50, P, s, st.badmask, st.m1, st.m2, st.m);
     } else {                                          // tiny matrices: the checked general form
         uint16_t t[6];
         unsigned long long mx[5] = {st.m1, st.m2, st.m[0], st.m[1], st.m[2]};

@@ -25,6 +25,7 @@ namespace {
 
 // Row-major planes: thread = 4 consecutive entries of a row (two 16-byte
 // loads, one 8-byte store per plane), rows advancing by the grid's y size.
+template <int NLEV>
 __global__ void __launch_bounds__(kThreads)
 f64_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
                      uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
@@ -50,18 +51,18 @@ f64_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, i
 #pragma unroll
                 for (int e = 0; e < 4; ++e) x[e] = (j0 + e < cols) ? src[e] : 0.0;
             }
-            uint32_t w[6][2];
+            uint32_t w[NLEV][2];
 #pragma unroll
             for (int e = 0; e < 4; e += 2) {
                 uint32_t sa[6], sb[6];
-                spec_element(x[e], v0, fast, P, sa, st);
-                spec_element(x[e + 1], v0, fast, P, sb, st);
+                spec_element<NLEV>(x[e], v0, fast, P, sa, st);
+                spec_element<NLEV>(x[e + 1], v0, fast, P, sb, st);
 #pragma unroll
-                for (int r = 0; r < 6; ++r) w[r][e >> 1] = pack2(sa[r], sb[r]);
+                for (int r = 0; r < NLEV; ++r) w[r][e >> 1] = pack2(sa[r], sb[r]);
             }
             uint16_t *dst = comps + i * ldcomp + j0;
 #pragma unroll
-            for (int r = 0; r < 6; ++r) {
+            for (int r = 0; r < NLEV; ++r) {
                 if (vout && full) {
                     *reinterpret_cast<uint2 *>(dst + r * plane) = make_uint2(w[r][0], w[r][1]);
                 } else {
@@ -79,6 +80,7 @@ f64_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, i
 // lane p on rows 2p and 2p+1; each plane word packs the two entries adjacent
 // in the transposed row, staged one bank per lane and written as 16-byte
 // chunks of whole transposed rows.  Shared memory: [6][64][32] words.
+template <int NLEV>
 __global__ void __launch_bounds__(kThreads)
 f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
                           uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
@@ -117,15 +119,16 @@ f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t co
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
                 uint32_t s0[6], s1[6];
-                spec_element(x[0][e], v0, fast, P, s0, st);
-                spec_element(x[1][e], v0, fast, P, s1, st);
+                spec_element<NLEV>(x[0][e], v0, fast, P, s0, st);
+                spec_element<NLEV>(x[1][e], v0, fast, P, s1, st);
 #pragma unroll
-                for (int r = 0; r < 6; ++r) smw[(r * kTile + 8 * q + k + e) * (kTile / 2) + p] = pack2(s0[r], s1[r]);
+                for (int r = 0; r < NLEV; ++r) smw[(r * kTile + 8 * q + k + e) * (kTile / 2) + p] = pack2(s0[r], s1[r]);
             }
         }
         __syncthreads();
+        // NLEV planes x 64 transposed rows x 8 chunks (two iterations per plane)
 #pragma unroll 4
-        for (int it = 0; it < 6 * kTile * 8 / kThreads; ++it) {
+        for (int it = 0; it < NLEV * kTile * 8 / kThreads; ++it) {
             const int c = threadIdx.x + it * kThreads;
             const int r = c >> 9, orow = (c >> 3) & 63, ch = c & 7;
             const int64_t go = c0 + orow, gk = r0 + 8 * ch;
@@ -147,12 +150,35 @@ f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t co
     spec_publish(st, v0, ws, slot, red);
 }
 
+// The fused speculative pass for slices 0 .. NLEV-1.
+template <int NLEV>
+cudaError_t launch_spec(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose, uint16_t *comps,
+                        int64_t ldcomp, int64_t plane, WsHeader *ws, int slot, int gt, cudaStream_t st)
+{
+    if (transpose) {
+        cudaError_t e = cudaFuncSetAttribute(f64_spec_transpose_kernel<NLEV>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSpecTransposeSmem);
+        if (e != cudaSuccess) return e;
+        f64_spec_transpose_kernel<NLEV><<<gt, kThreads, kSpecTransposeSmem, st>>>(X, rows, cols, ldx, comps, ldcomp,
+                                                                                  plane, ws, slot);
+    } else {
+        // about eight blocks per SM, each over several rows
+        const int64_t bx = (cols + 4 * kThreads - 1) / (4 * kThreads);
+        const int64_t want = (152 * 8 + bx - 1) / bx;
+        const int64_t by = rows < want ? rows : (want < 65535 ? want : 65535);
+        f64_spec_rows_kernel<NLEV><<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, comps,
+                                                                                          ldcomp, plane, ws, slot);
+    }
+    return cudaSuccess;
+}
+
 }  // namespace
 
 cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose,
                              uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
-                             cudaStream_t st)
+                             cudaStream_t st, int nlev)
 {
+    if (nlev < 3 || nlev > 6) return cudaErrorInvalidValue;
     const int64_t plane = (transpose ? cols : rows) * ldcomp;
     if (rows > 0 && cols > 0) {
         const int64_t segs = rows * ((cols + 4 * kThreads - 1) / (4 * kThreads));
@@ -160,25 +186,16 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
         const int64_t tiles = ((rows + kTile - 1) / kTile) * ((cols + kTile - 1) / kTile);
         const int gt = grid_for(tiles, 152 * 8);
         cudaError_t e = cudaSuccess;
-        if (transpose) {
-            e = cudaFuncSetAttribute(f64_spec_transpose_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)kSpecTransposeSmem);
-        }
-        if (e != cudaSuccess) return e;
         f64_max_kernel<0><<<gmax, kThreads, 0, st>>>(X, rows, cols, ldx, ws, slot);
-        if (transpose) {
-            f64_spec_transpose_kernel<<<gt, kThreads, kSpecTransposeSmem, st>>>(X, rows, cols, ldx, comps, ldcomp,
-                                                                            plane, ws, slot);
-        } else {
-            // about eight blocks per SM, each over several rows
-            const int64_t bx = (cols + 4 * kThreads - 1) / (4 * kThreads);
-            const int64_t want = (152 * 8 + bx - 1) / bx;
-            const int64_t by = rows < want ? rows : (want < 65535 ? want : 65535);
-            f64_spec_rows_kernel<<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, comps,
-                                                                                       ldcomp, plane, ws, slot);
+        switch (nlev) {
+        case 3: e = launch_spec<3>(X, rows, cols, ldx, transpose, comps, ldcomp, plane, ws, slot, gt, st); break;
+        case 4: e = launch_spec<4>(X, rows, cols, ldx, transpose, comps, ldcomp, plane, ws, slot, gt, st); break;
+        case 5: e = launch_spec<5>(X, rows, cols, ldx, transpose, comps, ldcomp, plane, ws, slot, gt, st); break;
+        default: e = launch_spec<6>(X, rows, cols, ldx, transpose, comps, ldcomp, plane, ws, slot, gt, st); break;
         }
         if (e == cudaSuccess) e = cudaGetLastError();
-        if (e == cudaSuccess) e = launch_f64_fix(X, rows, cols, ldx, transpose, comps, ldcomp, plane, ws, slot, v_out, st);
+        if (e == cudaSuccess)
+            e = launch_f64_fix(X, rows, cols, ldx, transpose, comps, ldcomp, plane, ws, slot, v_out, st, nlev);
         return e;
     }
     // an empty matrix: all levels zero, nothing to fix

@@ -16,12 +16,12 @@ namespace {
 template <bool TRANSPOSE>
 __global__ void __launch_bounds__(kThreads)
 f64_fix_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx, uint16_t *__restrict__ comps,
-               int64_t ldcomp, int64_t plane, WsHeader *ws, int slot, int32_t *v_out)
+               int64_t ldcomp, int64_t plane, WsHeader *ws, int slot, int32_t *v_out, int nlev)
 {
     extern __shared__ __align__(16) uint16_t smdyn[];
     __shared__ unsigned long long red[kThreads / 32];
     int v[6];
-    const int ff = f64_verify_levels(ws, slot, v);
+    const int ff = f64_verify_levels(ws, slot, v, nlev);
     if (ff == 6) {
         if (blockIdx.x == 0 && threadIdx.x == 0) {
             for (int r = 0; r < 6; ++r) ws->v[slot][r] = v[r];
@@ -57,7 +57,8 @@ f64_fix_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t
 // at once (at most 152 x 8), found once per device.
 template <bool TRANSPOSE>
 static cudaError_t launch_f64_fix_t(const double *X, int64_t rows, int64_t cols, int64_t ldx, uint16_t *comps,
-                           int64_t ldcomp, int64_t plane, WsHeader *ws, int slot, int32_t *v_out, cudaStream_t st)
+                           int64_t ldcomp, int64_t plane, WsHeader *ws, int slot, int32_t *v_out, cudaStream_t st,
+                           int nlev)
 {
     constexpr int kMaxDev = 64;
     static int grid_of[kMaxDev] = {};
@@ -81,22 +82,23 @@ static cudaError_t launch_f64_fix_t(const double *X, int64_t rows, int64_t cols,
         grid_of[dev] = grid;
     }
     void *args[] = {(void *)&X, (void *)&rows, (void *)&cols, (void *)&ldx, (void *)&comps, (void *)&ldcomp,
-                    (void *)&plane, (void *)&ws, (void *)&slot, (void *)&v_out};
+                    (void *)&plane, (void *)&ws, (void *)&slot, (void *)&v_out, (void *)&nlev};
     return cudaLaunchCooperativeKernel((const void *)kern, dim3((unsigned)grid), dim3(kThreads), args, sm, st);
 }
 
 
 cudaError_t launch_f64_fix(const double *X, int64_t rows, int64_t cols, int64_t ldx, bool transpose, uint16_t *comps,
-                           int64_t ldcomp, int64_t plane, WsHeader *ws, int slot, int32_t *v_out, cudaStream_t st)
+                           int64_t ldcomp, int64_t plane, WsHeader *ws, int slot, int32_t *v_out, cudaStream_t st,
+                           int nlev)
 {
-    return transpose ? launch_f64_fix_t<true>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, v_out, st)
-                     : launch_f64_fix_t<false>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, v_out, st);
+    return transpose ? launch_f64_fix_t<true>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, v_out, st, nlev)
+                     : launch_f64_fix_t<false>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, v_out, st, nlev);
 }
 
 // an empty matrix: all levels zero, nothing to fix (one block, no grid barrier)
 cudaError_t launch_f64_fix_empty(WsHeader *ws, int slot, int32_t *v_out, cudaStream_t st)
 {
-    f64_fix_kernel<false><<<1, kThreads, 0, st>>>(nullptr, 0, 0, 1, nullptr, 1, 0, ws, slot, v_out);
+    f64_fix_kernel<false><<<1, kThreads, 0, st>>>(nullptr, 0, 0, 1, nullptr, 1, 0, ws, slot, v_out, 6);
     return cudaGetLastError();
 }
 

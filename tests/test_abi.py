@@ -64,6 +64,9 @@ def test_host_argument_checks_need_no_gpu(lib):
     assert emu.emu_gemm_f32(1 << 31, 4, 4, P, 4, P, 4, P, 4, P, 1 << 62, None) == 5  # size limit
     assert emu.emu_split_f64(P, 4, 4, 2, 0, P, 4, P, P, 4096, None) == 1              # ldx < cols
     assert emu.emu_selftest_timeout(P, 4096, 0, None) == 1
+    assert emu.emu_split_f64_slices(P, 4, 4, 4, 0, P, 4, 2, P, P, 4096, None) == 1      # nslices < 3
+    assert emu.emu_split_f64_slices(P, 4, 4, 4, 0, P, 4, 7, P, P, 4096, None) == 1      # nslices > 6
+    assert emu.emu_split_f64_slices(P, 4, 4, 4, 0, P, 4, 4, P, P, 16, None) == 3        # workspace
     # merged FP64 tail: merge_from range and workspace size are checked on the host
     assert emu.emu_gemm_f64_merged(4, 4, 4, P, 4, P, 4, P, 4, 21, 2, P, 1 << 30, None) == 1
     assert emu.emu_gemm_f64_merged(4, 4, 4, P, 4, P, 4, P, 4, 10, 5, P, 1 << 30, None) == 1

@@ -191,6 +191,34 @@ def test_gemm_f64_long_k_positive_sums(dev, nprod):
     assert np.array_equal(C.cpu().numpy(), oracle.gemm_f64(A, B, nprod)[0])
 
 
+def _level_gap_inputs(shape, seed, gap_level):
+    """Entries whose residual after level gap_level - 1 is far below the
+    speculative 2^-8 step, so the speculative levels hold below gap_level and
+    fail at it."""
+    rng = np.random.default_rng(seed)
+    X = rng.integers(-127, 128, size=shape) * 2.0**10
+    for r in range(1, gap_level):
+        X = X + rng.integers(-127, 128, size=shape) * 2.0**(10 - 8 * r)
+    X = X + rng.integers(-127, 128, size=shape) * 2.0**(10 - 8 * gap_level - 30)
+    X.flat[0] = 127 * 2.0**10
+    return X
+
+
+@pytest.mark.parametrize("gap_level", [1, 4])
+@pytest.mark.parametrize("nprod", [6, 10, 15, 21])
+def test_gemm_f64_speculation_fails(dev, nprod, gap_level):
+    """The GEMM's split forms only the d slices its product-sum uses; when the
+    speculative levels fail below d the literal passes redo them, when they
+    fail only from d on they are never needed.  Either way C is the oracle's."""
+    A = _level_gap_inputs((300, 400), 40 + gap_level, gap_level)
+    B = _level_gap_inputs((400, 260), 50 + gap_level, gap_level)
+    _, vA, _ = oracle.split_f64(A)
+    assert vA[gap_level] != vA[0] - 8 * gap_level
+    C, ws = emu.gemm_f64(to_dev(A, dev), to_dev(B, dev), nprod)
+    assert emu.read_flags(ws) == 0
+    assert np.array_equal(C.cpu().numpy(), oracle.gemm_f64(A, B, nprod)[0])
+
+
 # ------------------------------------------------------------ edges, errors
 def test_zero_sizes_and_empty_k(dev):
     torch = emu._torch()

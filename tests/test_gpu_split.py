@@ -123,6 +123,52 @@ def test_split_f64_fix_path_large(dev, transpose):
     assert wv[1] != wv[0] - 8
 
 
+@pytest.mark.parametrize("gap_level", [1, 2, 3, 4, 5])
+@pytest.mark.parametrize("scale", [30, 3])
+def test_split_f64_level_gap(dev, gap_level, scale):
+    """The speculative levels hold below gap_level and fail at it, the residual
+    there 2^-scale below the speculative step: far below (scale 30, under the
+    fused pass's fixed-point unit, where only a sticky bit is left of it) or
+    just below (scale 3).  Planes and levels as the oracle's, both layouts."""
+    rng = np.random.default_rng(60 + gap_level)
+    shape = (300, 270)
+    X = rng.integers(-127, 128, size=shape) * 2.0**10
+    for r in range(1, gap_level):
+        X = X + rng.integers(-127, 128, size=shape) * 2.0**(10 - 8 * r)
+    X = X + rng.integers(-127, 128, size=shape) * 2.0**(10 - 8 * gap_level - scale)
+    X[0, 0] = 127 * 2.0**10
+    for transpose in (False, True):
+        wv = _check_f64(X, dev, transpose)
+        assert wv[gap_level] != wv[0] - 8 * gap_level
+
+
+@pytest.mark.parametrize("nslices", [3, 4, 5, 6])
+@pytest.mark.parametrize("gap_level", [0, 2, 4])
+def test_split_f64_slices(dev, nslices, gap_level):
+    """emu_split_f64_slices: planes and levels below nslices as the oracle's,
+    with the speculative levels holding (gap_level 0) or failing below or
+    above nslices."""
+    rng = np.random.default_rng(80 + gap_level)
+    shape = (260, 190)
+    if gap_level == 0:
+        X = synth.uniform_f64(7, 0, shape)
+    else:
+        X = rng.integers(-127, 128, size=shape) * 2.0**10
+        for r in range(1, gap_level):
+            X = X + rng.integers(-127, 128, size=shape) * 2.0**(10 - 8 * r)
+        X = X + rng.integers(-127, 128, size=shape) * 2.0**(10 - 8 * gap_level - 30)
+        X[0, 0] = 127 * 2.0**10
+    want, wv, wflags = oracle.split_f64(X)
+    assert wflags == 0
+    for transpose in (False, True):
+        planes, v, ws = emu.split_f64(to_dev(X, dev), transpose=transpose, nslices=nslices)
+        assert emu.read_flags(ws) == 0
+        got = planes_np(planes)
+        ref = want.transpose(0, 2, 1) if transpose else want
+        assert np.array_equal(v.cpu().numpy()[:nslices], wv[:nslices])
+        assert np.array_equal(got[:nslices], ref[:nslices])
+
+
 def test_split_f64_flags(dev):
     X = synth.uniform_f64(3, 0, (33, 47))
     for val in (np.nan, np.inf, 2.0**-127, 2.0**129):
