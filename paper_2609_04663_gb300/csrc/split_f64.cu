@@ -11,11 +11,12 @@
 // Eq. (fp64split)), i.e. six dependent grid-wide reductions.  The split does
 // them speculatively in one pass: after the exact max of level 0, the fused
 // pass assumes v^(r) = v^(0) - 8r (a residual always shrinks by at least 2^-8
-// per level, and on full-size dense data by exactly that), writes all six
-// planes and records the true per-level maxima.  One cooperative launch then
-// checks the assumption level by level and, only if it fails, recomputes the
-// remaining levels literally.  The result is identical to the literal
-// definition in every case.
+// per level, and on full-size dense data by exactly that), writes the planes
+// (all six, or only the d a product-sum of d diagonals reads) and records the
+// true per-level maxima.  One cooperative launch then checks the assumption
+// level by level and, only if it fails, recomputes the remaining levels
+// literally.  The result is identical to the literal definition in every
+// case.
 #include "split_common.cuh"
 
 namespace emu {
