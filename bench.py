@@ -267,8 +267,9 @@ class Case:
 
     def split_bytes(self):
         """Algorithmic HBM bytes of the two splits: FP32 4 B read + 6 B written
-        per entry; FP64 8 B (level-0 max) + 8 B (fused pass) read + 12 B written."""
-        per = 10 if self.mode == 32 else 28
+        per entry; FP64 8 B (level-0 max) + 8 B (fused pass) read + 2 B written
+        per slice formed (the d slices the product-sum reads)."""
+        per = 10 if self.mode == 32 else 16 + 2 * {6: 3, 10: 4, 15: 5, 21: 6}[self.nprod]
         return per * (self.M * self.K + self.K * self.N)
 
 
