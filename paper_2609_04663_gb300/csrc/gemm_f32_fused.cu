@@ -220,8 +220,7 @@ cudaError_t launch_gemm_f32_fused(int64_t M, int64_t N, int64_t K, const float *
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
     const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + 255) / 256);
-    kern<<<(unsigned)tiles, 32 + kConv, Cfg::SMEM, st>>>(A, lda, B, ldb, (int)M, (int)N, (int)K, C, ldc,
-                                                               flags);
+    kern<<<(unsigned)tiles, 32 + kConv, Cfg::SMEM, st>>>(A, lda, B, ldb, (int)M, (int)N, (int)K, C, ldc, flags);
     return cudaGetLastError();
 }
 
