@@ -320,6 +320,8 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
             // the coarse part (multiples of 2^12 u) moves to the low word in C and
             // stays exact below 2^36 u, i.e. for up to 2^11 chunks of at most 2^25 u.
             const bool carry = !ROWCOL && bound > 0.0f && bound <= 0x1p116f && nch <= 2048;
+            // this thread's row level of slice i (levels per row / column only)
+            const int a_row = (ROWCOL && row < M) ? vA[(int64_t)kDiag[q][0] * M + row] : kZeroLevel;
             for (int c = 0; c < nch; ++c) {
                 const int t = q * nch + c, b = t % Cfg::NBUF;
                 ok = mbar_wait(tfull0 + 8u * b, (uint32_t)((t / Cfg::NBUF) & 1), flags);
@@ -367,7 +369,9 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                     } else {
                         // rare: redo the 16 additions as TwoSums, the errors summed
                         // exactly into the low part; the partials are read again from
-                        // TMEM (the buffer is not yet released)
+                        // TMEM (the buffer is not yet released).  With levels per row /
+                        // column an element whose own unit allows it takes the carry
+                        // above instead (its own split constant).
                         const bool was = (dirty >> (h / 16)) & 1u;
                         dirty |= 1u << (h / 16);
                         const float renorm = 0.5f * bound;        // lo is kept below 2^23 u
@@ -377,12 +381,23 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                             const int j = h + jj;
                             const float p = __uint_as_float(tmem_ld1(taddr + (uint32_t)jj));
                             tmem_ld_wait();
-                            float e, lo;
-                            const float sm = two_sum(hi[j], p, e);
                             const bool mine = j < lim;
-                            lo = __fadd_rn((was && mine) ? lrow[2 * j] : 0.0f, e);
-                            hi[j] = (fabsf(lo) < renorm) ? sm : two_sum(sm, lo, lo);   // renormalise (hi, lo)
-                            if (mine) lrow[2 * j] = lo;
+                            float be = 0.0f;
+                            if (ROWCOL && mine && nch <= 2048)
+                                be = bound_of_levels(a_row, vB[(int64_t)kDiag[q][1] * N + n0 + cq * Cfg::COLS + j]);
+                            if (be > 0.0f && be <= 0x1p116f) {
+                                const float cm = 3072.0f * be;
+                                const float h1 = __fsub_rn(__fadd_rn(hi[j], cm), cm), l1 = __fsub_rn(hi[j], h1);
+                                const float h2 = __fsub_rn(__fadd_rn(p, cm), cm), l2 = __fsub_rn(p, h2);
+                                lrow[2 * j] = __fadd_rn(was ? lrow[2 * j] : 0.0f, __fadd_rn(h1, h2));
+                                hi[j] = __fadd_rn(l1, l2);
+                            } else {
+                                float e, lo;
+                                const float sm = two_sum(hi[j], p, e);
+                                lo = __fadd_rn((was && mine) ? lrow[2 * j] : 0.0f, e);
+                                hi[j] = (fabsf(lo) < renorm) ? sm : two_sum(sm, lo, lo);   // renormalise (hi, lo)
+                                if (mine) lrow[2 * j] = lo;
+                            }
                         }
                     }
                     if (h + 16 == Cfg::COLS) {                   // buffer free: all values are in registers

@@ -84,6 +84,25 @@ def test_gemm_rowcol_bitexact(dev, M, N, K, nprod):
     np.testing.assert_array_equal(C.cpu().numpy().view(np.uint64), want.view(np.uint64))
 
 
+@pytest.mark.parametrize("nprod", [6, 21])
+def test_gemm_rowcol_long_k_positive_sums(dev, nprod):
+    """Positive entries over 40 K-chunks with row and column scalings of up
+    to 2^6 either way: the running sums pass 2^24 units of the smallest unit
+    of a thread's columns within a few chunks, and each element then carries
+    at its own unit (or redoes its additions as TwoSums); bit for bit."""
+    M, N, K = 130, 200, 256 * 40 + 17
+    rng = np.random.default_rng(48)
+    U = rng.uniform(0.5, 1.0, size=(M, K))
+    V = rng.uniform(0.5, 1.0, size=(K, N))
+    A = U * np.ldexp(1.0, rng.integers(-6, 7, size=M))[:, None]
+    B = V * np.ldexp(1.0, rng.integers(-6, 7, size=N))[None, :]
+    C, ws = emu.gemm_f64_rowcol(to_dev(A, dev), to_dev(B, dev), nprod)
+    assert emu.read_flags(ws) == 0
+    want, flags = oracle.gemm_f64_rowcol(A, B, nprod)
+    assert flags == 0
+    np.testing.assert_array_equal(C.cpu().numpy().view(np.uint64), want.view(np.uint64))
+
+
 def test_gemm_rowcol_commutes_with_scaling_on_gpu(dev):
     """D_A U times V D_B equals D_A (U V) D_B exactly on the GPU path too.
     Scalings stay where every product's unit 2^(vA_5 + vB_5 - 16), about
