@@ -5,8 +5,8 @@ Metric: emulated GEMM TFLOP/s = 2 M N K / t per step, where a step is one
 pass of the whole hot path on resident inputs: split A, split B (transposed)
 and the tensor-core product-sum.  The headline workload is FP32 mode (6
 products) at M = N = K = 16384, the top of the paper's square sweep; FP64
-mode at M = N = K = 4096 with 6, 10, 15 and 21 products and the other
-workloads are reported under "variants".
+mode (4096^3 at 6, 10, 15 and 21 products, 8192^3 scaled inputs, the
+large-K shape) and the rest of the FP32 sweep are reported under "variants".
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   (the CPU oracle on the host cores)
@@ -504,14 +504,21 @@ def gpu_arm(args, rank, world, local):
 def variants(args, rank, world, pk):
     """The other workloads, a few steps each, L2 flushed between steps."""
     out = {}
-    # entries: (workload, FP64 product count | "fused" | (product count, merge_from))
-    todo = [("fp32_n8192", None), ("fp32_n8192", "fused"), ("fp64_n4096", 6), ("fp64_n4096", 10),
-            ("fp64_n4096", 15), ("fp64_n4096", 21), ("fp64_n4096", (21, 4)), ("fp64_n4096", (15, 4))]
+    # entries: (workload, FP64 product count | "fused" | (product count, merge_from)).
+    # The default list covers every configuration of the paper's evaluation
+    # that these workloads stand in for: FP32 256^3; the FP32 square sweep
+    # 1024-8192 (16384 is the headline); FP64 4096^3 at 6/10/15/21 products;
+    # FP64 8192^3 scaled inputs at 21 and 10 products; the large-K shape
+    # 2048 x 2048 x 65536 in FP32 and at every FP64 product count.
+    todo = [("fp32_n256", None), ("fp32_n1024", None), ("fp32_n2048", None), ("fp32_n4096", None),
+            ("fp32_n8192", None), ("fp64_n4096", 6), ("fp64_n4096", 10), ("fp64_n4096", 15), ("fp64_n4096", 21),
+            ("fp64_scaled_phi4_n8192", 21), ("fp64_scaled_phi4_n8192", 10), ("fp64_scaled_phi0.5_n8192", 21),
+            ("fp64_scaled_phi2_n8192", 21), ("fp32_largek", None), ("fp64_largek", 6), ("fp64_largek", 10),
+            ("fp64_largek", 15), ("fp64_largek", 21)]
     if args.all_variants:
-        todo += [("fp32_n1024", None), ("fp32_n2048", None), ("fp32_n4096", None), ("fp32_largek", None),
-                 ("fp32_n16384", "fused"), ("fp64_scaled_phi4_n8192", 21), ("fp64_scaled_phi4_n8192", 10),
-                 ("fp64_scaled_phi4_n8192", (21, 4)), ("fp64_scaled_phi0.5_n8192", 21), ("fp64_scaled_phi0.5_n8192", (21, 4)),
-                 ("fp64_largek", 21), ("fp32_cancel_n4096", None), ("fp64_cancel_n4096", 21)]
+        todo += [("fp32_n8192", "fused"), ("fp32_n16384", "fused"), ("fp64_n4096", (21, 4)), ("fp64_n4096", (15, 4)),
+                 ("fp64_scaled_phi4_n8192", (21, 4)), ("fp64_scaled_phi0.5_n8192", (21, 4)),
+                 ("fp32_cancel_n4096", None), ("fp64_cancel_n4096", 21)]
     torch = __import__("torch")
     for name, nprod in todo:
         fused = nprod == "fused"
@@ -528,6 +535,9 @@ def variants(args, rank, world, pk):
                     "prodsum_ms": pm, "split_ms": statistics.mean(res["split_ms"]),
                     "executed_tflops": case.exec_flop / (pm / 1e3) / 1e12,
                     "frac_of_bf16_peak": case.exec_flop / (pm / 1e3) / 1e12 / pk["bf16_burst"],
+                    "traffic": None if fused or merge_from else
+                               kernel_traffic("prodsum_f32" if case.mode == 32 else "prodsum_f64",
+                                              name if case.mode == 32 else f"{name}_np{case.nprod}"),
                     "flags": case.emu.read_flags(case.gemm_ws if case.gemm_ws is not None else case.ws)}
         del case
         torch.cuda.empty_cache()

@@ -304,11 +304,13 @@ emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
  * accumulator must fit the array, e.g. M = N = K = 1024; larger problems
  * return EMU_ERR_UNSUPPORTED before any work is enqueued.
  * flags_out: device pointer receiving the EMU_FLAG_* word of this call
- * (may be NULL).  The first call on each device looks up the array's device
- * address (with that device current); make that first call before any
- * stream capture.  All calls on a device share the array: calls whose work
- * may overlap on the GPU (different streams or host threads without
- * ordering) race and must be serialised by the caller. */
+ * (may be NULL).  Every call looks up the array's device address in the
+ * current context (a lookup that allocates nothing, so it stays right after
+ * cudaDeviceReset re-creates the context); the first call on a device may
+ * load the library's device code, so make that first call before any stream
+ * capture.  All calls on a device share the array: calls whose work may
+ * overlap on the GPU (different streams or host threads without ordering)
+ * race and must be serialised by the caller. */
 #define EMU_NOALLOC_SCRATCH_BYTES (40u << 20)
 emu_status emu_gemm_f64_noalloc(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda,
                                 const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,

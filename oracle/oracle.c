@@ -18,7 +18,7 @@
  *   B planes  [s][K][N]  BF16 bit patterns
  *   C         [nrows][N] rows r0 .. r0+nrows-1 of the product
  *
- * Readings of points the paper leaves open (each listed in the design doc):
+ * Readings of points the paper leaves open (each also listed in the design notes):
  *   - fl_BF16 rounds to nearest, ties to even, with BF16 subnormals and
  *     overflow to infinity (Section 4.2 says "round-to-nearest").
  *   - v^(r) of Eq. (fp64split) is one scalar per operand and level: the max is

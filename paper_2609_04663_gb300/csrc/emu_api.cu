@@ -195,7 +195,7 @@ emu_status emu_gemm_f64_merged(int64_t M, int64_t N, int64_t K, const double *A,
 {
     emu_status s = check_gemm_dims(M, N, K, lda, ldb, ldc);
     if (s != EMU_OK) return s;
-    const int d = nprod == 6 ? 3 : nprod == 10 ? 4 : nprod == 15 ? 5 : nprod == 21 ? 6 : 0;
+    const int d = f64_diagonals(nprod);
     if (d == 0 || merge_from < 3 || merge_from > d) return EMU_ERR_INVALID_ARG;
     if (!ws || (M > 0 && N > 0 && (!C || (K > 0 && (!A || !B))))) return EMU_ERR_INVALID_ARG;
     if (ws_bytes < emu_gemm_f64_merged_workspace_bytes(M, N, K)) return EMU_ERR_WORKSPACE_TOO_SMALL;
@@ -211,7 +211,7 @@ emu_status emu_gemm_f64_merged(int64_t M, int64_t N, int64_t K, const double *A,
     uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(6 * M * ldk * 2, 256));
     float *T = merge_from < d ? reinterpret_cast<float *>(static_cast<char *>(ws) + gemm_ws_bytes(6, M, N, K)) : nullptr;
     // the product-sum uses slices 0 .. d-1 only
-    const int nlev = nprod == 6 ? 3 : nprod == 10 ? 4 : nprod == 15 ? 5 : 6;
+    const int nlev = f64_diagonals(nprod);
     e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st, nlev);
     if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st, nlev);
     if (e == cudaSuccess && T) e = launch_prodsum_tail(M, N, K, Ap, Bp, ldk, merge_from, d, T, N, &h->flags, st);
@@ -241,7 +241,7 @@ emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_
     uint16_t *Ap = reinterpret_cast<uint16_t *>(static_cast<char *>(ws) + kWsHeaderBytes);
     uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(6 * M * ldk * 2, 256));
     // the product-sum uses slices 0 .. d-1 only
-    const int nlev = nprod == 6 ? 3 : nprod == 10 ? 4 : nprod == 15 ? 5 : 6;
+    const int nlev = f64_diagonals(nprod);
     e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st, nlev);
     if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st, nlev);
     if (e == cudaSuccess)
@@ -306,7 +306,7 @@ emu_status gemm_ex(int opA, int opB, int64_t M, int64_t N, int64_t K, T alpha, c
         const bool ta = opA == EMU_OP_T, tb = opB == EMU_OP_N;
         const int64_t ar = ta ? K : M, ac = ta ? M : K, br = tb ? K : N, bc = tb ? N : K;
         if constexpr (f64) {
-            const int nlev = nprod == 6 ? 3 : nprod == 10 ? 4 : nprod == 15 ? 5 : 6;   // slices the product-sum uses
+            const int nlev = f64_diagonals(nprod);   // slices the product-sum uses
             e = launch_split_f64(A, ar, ac, lda, ta, Ap, ldk, h->vout[0], h, 0, st, nlev);
             if (e == cudaSuccess) e = launch_split_f64(B, br, bc, ldb, tb, Bp, ldk, h->vout[1], h, 1, st, nlev);
             if (e == cudaSuccess)

@@ -289,7 +289,7 @@ emu_status emu_gemm_f64_host(int64_t M, int64_t N, int64_t K, const double *A, i
                              emu_stream_t stream)
 {
     if (nprod != 6 && nprod != 10 && nprod != 15 && nprod != 21) return EMU_ERR_INVALID_ARG;
-    const int nlev = nprod == 6 ? 3 : nprod == 10 ? 4 : nprod == 15 ? 5 : 6;   // slices the product-sum uses
+    const int nlev = f64_diagonals(nprod);   // slices the product-sum uses
     emu_status s = check_args(M, N, K, A, lda, B, ldb, C, ldc, ws, ws_bytes, 64);
     if (s != EMU_OK) return s;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);

@@ -22,6 +22,14 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
                              uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
                              cudaStream_t st, int nlev = 6);
 
+// Number of diagonals d of an FP64-mode product count (Eq. (fp64productcounts):
+// nprod = d (d + 1) / 2), i.e. the slices 0 .. d-1 a product-sum reads; 0 for
+// any other count.
+inline int f64_diagonals(int nprod)
+{
+    return nprod == 6 ? 3 : nprod == 10 ? 4 : nprod == 15 ? 5 : nprod == 21 ? 6 : 0;
+}
+
 // Eq. (fp64split) with one set of levels per plane row (an input row, or an
 // input column when transposed): v_out[6][plane rows] (level-major);
 // scratch: rc_scratch_bytes(plane rows) bytes, 8-byte aligned; slot: the

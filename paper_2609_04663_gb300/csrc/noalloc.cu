@@ -6,16 +6,15 @@
 // and some latency-critical paths cannot accept the implicit device
 // synchronisation a cudaMalloc may cause.  Such callers can still pass their
 // inputs and outputs, but not a workspace.  emu_gemm_f64_noalloc runs the
-// same split and product-sum kernels as emu_gemm_f64 with their scratch (flag
-// word, level maxima, BF16 planes) in the file-scope device array below.
+// same split and product-sum kernels as emu_gemm_f64, with the same number of
+// slices, and keeps their scratch (flag word, level maxima, BF16 planes, FP64
+// accumulator) in the file-scope device array below.
 //
 // The array is EMU_NOALLOC_SCRATCH_BYTES (40 MiB) on every GPU that loads the
 // library, for as long as the library stays loaded.  All calls on a device
 // share it: each call clears the parts that must start at zero and overwrites
 // the rest, and calls whose work overlaps on the GPU (other streams, other
 // host threads) race on it.
-#include <mutex>
-
 #include "launchers.cuh"
 
 using namespace emu;
@@ -24,27 +23,18 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[EMU_NOALLOC_SCR
 
 namespace {
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mutex;
-unsigned char *g_scratch_addr[kMaxDevices] = {};
-
-// Device address of the scratch array on the current device.  The name of a
-// __device__ variable is only a host-side handle; the first call on each
-// device asks the runtime for the real address once, with that device current.
+// Device address of the scratch array in the current context.  The name of a
+// __device__ variable is only a host-side handle, so every call asks the
+// runtime for the real address with the caller's device current.  The lookup
+// allocates nothing, and asking each time (rather than caching per device)
+// stays right when the context is torn down and re-created (cudaDeviceReset),
+// after which the module, and with it the array, may sit elsewhere.
 cudaError_t scratch_address(unsigned char **out)
 {
-    int dev = -1;
-    cudaError_t e = cudaGetDevice(&dev);
+    void *p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-    std::lock_guard<std::mutex> lock(g_mutex);
-    if (!g_scratch_addr[dev]) {
-        void *p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-        if (e != cudaSuccess) return e;
-        g_scratch_addr[dev] = static_cast<unsigned char *>(p);
-    }
-    *out = g_scratch_addr[dev];
+    *out = static_cast<unsigned char *>(p);
     return cudaSuccess;
 }
 
@@ -60,14 +50,19 @@ extern "C" emu_status emu_gemm_f64_noalloc(int64_t M, int64_t N, int64_t K, cons
     if (lda < (K > 0 ? K : 1) || ldb < (N > 0 ? N : 1) || ldc < (N > 0 ? N : 1)) return EMU_ERR_INVALID_ARG;
     if (nprod != 6 && nprod != 10 && nprod != 15 && nprod != 21) return EMU_ERR_INVALID_ARG;
     if (M > 0 && N > 0 && (!C || (K > 0 && (!A || !B)))) return EMU_ERR_INVALID_ARG;
-    // scratch: header, 6 A planes [M][ldk] and 6 B planes [N][ldk] of BF16, FP64 accumulator
+    // scratch: header, 6 A planes [M][ldk] and 6 B planes [N][ldk] of BF16, FP64 accumulator.
+    // Every factor is below 2^31 once the first check has passed, so each term
+    // is computed without overflow and compared with the array on its own.
+    const int64_t cap = (int64_t)EMU_NOALLOC_SCRATCH_BYTES;
+    if (M >= ((int64_t)1 << 31) || N >= ((int64_t)1 << 31) || K >= ((int64_t)1 << 31)) return EMU_ERR_UNSUPPORTED;
     const int64_t ldk = round_up(K < 1 ? 1 : K, 8);
+    if (M > cap / (12 * ldk) || N > cap / (12 * ldk)) return EMU_ERR_UNSUPPORTED;
     const int64_t a_bytes = round_up(6 * M * ldk * 2, 256);
     const int64_t b_bytes = round_up(6 * N * ldk * 2, 256);
-    const int64_t need = (int64_t)kWsHeaderBytes + a_bytes + b_bytes + (int64_t)f64_acc_bytes(M, N);
-    if (M >= ((int64_t)1 << 31) || N >= ((int64_t)1 << 31) || K >= ((int64_t)1 << 31) ||
-        need > (int64_t)EMU_NOALLOC_SCRATCH_BYTES)
-        return EMU_ERR_UNSUPPORTED;
+    if ((M + 127) / 128 > cap / 131072 || (N + 127) / 128 > cap / 131072) return EMU_ERR_UNSUPPORTED;
+    const int64_t acc_bytes = (int64_t)f64_acc_bytes(M, N);
+    if ((int64_t)kWsHeaderBytes + a_bytes + b_bytes + acc_bytes > cap) return EMU_ERR_UNSUPPORTED;
+    const int nlev = f64_diagonals(nprod);      // the slices the product-sum reads, as emu_gemm_f64 splits
 
     unsigned char *scratch = nullptr;
     if (scratch_address(&scratch) != cudaSuccess) return EMU_ERR_CUDA;
@@ -80,8 +75,8 @@ extern "C" emu_status emu_gemm_f64_noalloc(int64_t M, int64_t N, int64_t K, cons
         } else {
             uint16_t *Ap = reinterpret_cast<uint16_t *>(scratch + kWsHeaderBytes);
             uint16_t *Bp = reinterpret_cast<uint16_t *>(scratch + kWsHeaderBytes + a_bytes);
-            e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st);
-            if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st);
+            e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st, nlev);
+            if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st, nlev);
             if (e == cudaSuccess)
                 e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, C, ldc,
                                        reinterpret_cast<double *>(scratch + kWsHeaderBytes + a_bytes + b_bytes),

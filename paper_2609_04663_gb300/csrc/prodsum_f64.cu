@@ -316,9 +316,11 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                                                             n0 + cq * Cfg::COLS, Cfg::COLS)
                                        : exact_bound(vA, vB, kDiag[q][0], kDiag[q][1]);
             // Carry instead of TwoSums when all elements share the unit u = 2^-24 bound
-            // (levels per matrix) and the split constant 1.5 * 2^35 u is finite:
-            // the coarse part (multiples of 2^12 u) moves to the low word in C and
-            // stays exact below 2^36 u, i.e. for up to 2^11 chunks of at most 2^25 u.
+            // (levels per matrix) and the split constant 1.5 * 2^35 u is finite.  A
+            // carry splits the running sum and the partial (each at most 2^24 u) at
+            // multiples of 2^12 u and moves both coarse parts (together at most
+            // 2^25 u) to the low word in C, which stays exact below 2^36 u, i.e. for
+            // up to 2^11 carries.
             const bool carry = !ROWCOL && bound > 0.0f && bound <= 0x1p116f && nch <= 2048;
             // this thread's row level of slice i (levels per row / column only)
             const int a_row = (ROWCOL && row < M) ? vA[(int64_t)kDiag[q][0] * M + row] : kZeroLevel;

@@ -1,8 +1,9 @@
 """emu_gemm_f64_noalloc: the FP64-mode GEMM for callers that cannot allocate
 device memory (it keeps its scratch in a static device array instead of a
 caller-provided workspace).  It must give what emu_gemm_f64 gives -- FP64
-mode is bit-exact, so the bar here is equality -- on consecutive calls that
-reuse the shared array, and refuse problems too large for the array.
+mode is bit-exact, so the bar here is equality, both with that entry point
+and with the oracle -- on consecutive calls that reuse the shared array,
+report the same flags, and refuse problems too large for the array.
 
 This file is collected last on purpose: it also runs after every other test
 in the same process, and on its own in a fresh one."""
@@ -11,6 +12,7 @@ import ctypes
 import numpy as np
 import pytest
 
+import oracle
 import synth
 import paper_2609_04663_gb300 as emu
 from helpers import device, to_dev
@@ -43,7 +45,33 @@ def test_noalloc_matches_workspace_entry_point_twice():
         Cref, ws = emu.gemm_f64(Ad, Bd, nprod)
         assert emu.read_flags(ws) == 0
         assert int(flags.item()) == 0
-        assert np.array_equal(C.cpu().numpy(), Cref.cpu().numpy())
+        Cn = C.cpu().numpy()
+        assert np.array_equal(Cn, Cref.cpu().numpy())
+        C_or, f_or = oracle.gemm_f64(A, B, nprod)
+        assert f_or == 0
+        assert np.array_equal(Cn, C_or)
+
+
+def test_noalloc_flags_equal_workspace_entry_point_on_small_slices():
+    """A scaled by 2^-80: its slices 0-2 are normal BF16 values, but slices 4
+    and 5 hold values below 2^-126.  With 6 products only slices 0-2 are
+    formed and read, so neither entry point may flag anything, and C equals
+    the oracle's bit for bit (every product unit stays a normal FP32 number)."""
+    dev = device()
+    torch = emu._torch()
+    flags = torch.full((1,), 0xFFFF, dtype=torch.int32, device=dev)
+    A, B = synth.gemm_inputs("f64", 160, 144, 520, 4)
+    A = A * 2.0**-80
+    assert np.all(np.abs(A[A != 0]) >= 2.0**-126)
+    Ad, Bd = to_dev(A, dev), to_dev(B, dev)
+    for _ in range(2):
+        st, C = _noalloc(Ad, Bd, 6, flags)
+        assert st == 0
+        Cref, ws = emu.gemm_f64(Ad, Bd, 6)
+        assert int(flags.item()) == emu.read_flags(ws) == 0
+        Cn = C.cpu().numpy()
+        assert np.array_equal(Cn, Cref.cpu().numpy())
+        assert np.array_equal(Cn, oracle.gemm_f64(A, B, 6)[0])
 
 
 def test_noalloc_limit_and_flags():
@@ -63,6 +91,9 @@ def test_noalloc_limit_and_flags():
     assert st == 0
     Cref, _ = emu.gemm_f64(Ad, Bd, 6)
     assert np.array_equal(C.cpu().numpy(), Cref.cpu().numpy())
+    Cn = C.cpu().numpy()
+    for r in (0, 511, n - 1):                              # sampled rows against the oracle
+        assert np.array_equal(Cn[r], oracle.gemm_f64(A, B, 6, rows=(r, r + 1))[0][0])
     big = torch.zeros((1184, 1184), dtype=torch.float64, device=dev)
     st, _ = _noalloc(big, big, 6, flags)
     assert st == 5                                       # EMU_ERR_UNSUPPORTED: beyond the static scratch
