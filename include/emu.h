@@ -300,7 +300,7 @@ emu_status emu_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
  * FP64 accumulator) in a static device array of EMU_NOALLOC_SCRATCH_BYTES
  * that every GPU loading the library holds until the library is unloaded.
  * Limit: 512 + 12 * (M + N) * roundup(K, 8) bytes of planes (256-byte
- * rounding per operand) plus 8 * roundup(M, 128) * roundup(N, 128) bytes of
+ * rounding per operand) plus 8 * roundup(M, 128) * roundup(N, 256) bytes of
  * accumulator must fit the array, e.g. M = N = K = 1024; larger problems
  * return EMU_ERR_UNSUPPORTED before any work is enqueued.
  * flags_out: device pointer receiving the EMU_FLAG_* word of this call

@@ -16,7 +16,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 SO = os.path.join(HERE, "_emu.so")
-SOURCES = ["emu_api.cu", "split_f32.cu", "split_f64.cu", "split_fix.cu", "split_rc.cu", "prodsum_f32.cu", "gemm_f32_fused.cu", "prodsum_f64.cu", "prodsum_tail.cu", "noalloc.cu", "host_api.cu", "epilogue.cu"]
+SOURCES = ["emu_api.cu", "split_f32.cu", "split_f64.cu", "split_fix.cu", "split_rc.cu", "prodsum_f32.cu", "gemm_f32_fused.cu", "prodsum_f64.cu", "prodsum_f64w.cu", "prodsum_tail.cu", "noalloc.cu", "host_api.cu", "epilogue.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-ftz=false", "-prec-div=true",
          "-prec-sqrt=true", "-fmad=true"]

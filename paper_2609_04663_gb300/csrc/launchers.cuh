@@ -73,10 +73,22 @@ cudaError_t launch_prodsum_tail(int64_t M, int64_t N, int64_t K, const uint16_t 
                                 int64_t ldcomp, int L, int d, float *T, int64_t ldt, uint32_t *flags,
                                 cudaStream_t st);
 
-// Bytes of the FP64 product-sum's accumulator: one 128 x 128 FP64 tile per CTA tile.
+// The FP64 product-sum on 128 x 256 tiles (prodsum_f64w.cu); launch_prodsum_f64
+// calls it when that tile shape is chosen.  acc: f64_acc_bytes(M, N) bytes.
+cudaError_t launch_prodsum_f64_wide(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
+                                    int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
+                                    int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
+                                    bool rowcol, const float *T, int64_t ldt);
+
+// Bytes of the FP64 product-sum's accumulator, enough for either tile shape:
+// one FP64 tile of 128 x 128 (narrow kernel) or 128 x 256 (wide kernel) per
+// CTA tile.
 inline size_t f64_acc_bytes(int64_t M, int64_t N)
 {
-    return (size_t)((M + 127) / 128) * (size_t)((N + 127) / 128) * 128u * 128u * sizeof(double);
+    const size_t tm = (size_t)((M + 127) / 128);
+    const size_t narrow = tm * (size_t)((N + 127) / 128) * 128u * 128u * sizeof(double);
+    const size_t wide = tm * (size_t)((N + 255) / 256) * 128u * 256u * sizeof(double);
+    return narrow > wide ? narrow : wide;
 }
 
 // General-GEMM epilogue: C <- fl(fl(alpha P) + fl(beta C)) (beta = 0: C <- fl(alpha P), C not read).

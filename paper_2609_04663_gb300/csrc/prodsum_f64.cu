@@ -33,8 +33,11 @@
 // each), warps 20-23 fold (one per lane quarter, 128 columns each).
 // setmaxnreg moves registers between the warpgroups.  Every wait is bounded
 // and reports EMU_FLAG_TIMEOUT instead of hanging.
-#include "gemm_common.cuh"
+#include <cstdlib>
+#include <cstring>
+
 #include "launchers.cuh"
+#include "prodsum_f64_common.cuh"
 
 namespace emu {
 
@@ -74,124 +77,6 @@ static_assert(F64Cfg::SMEM <= 232448, "shared memory per CTA");
 static_assert(128 * F64Cfg::REG_CTRL + 512 * F64Cfg::REG_DRAIN + 128 * F64Cfg::REG_FOLD <=
                   F64Cfg::THREADS * F64Cfg::REG_LAUNCH,
               "setmaxnreg split exceeds the registers reserved at launch");
-
-template <uint32_t R> __device__ __forceinline__ void regs_dec() { asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R)); }
-template <uint32_t R> __device__ __forceinline__ void regs_inc() { asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(R)); }
-
-// Exact FP32 -> FP64 widening by integer operations only (on GB300 a
-// conversion instruction would occupy the FP64 pipe, which the fold's adds
-// need): rebias the exponent and shift the significand of a normal value;
-// normalise a subnormal by its leading bit; keep zeros, infinities and NaN
-// payloads.
-__device__ __forceinline__ double widen_exact(float x)
-{
-    const uint32_t u = __float_as_uint(x);
-    const uint32_t sign = u & 0x80000000u, ex = (u >> 23) & 0xFFu, m = u & 0x7FFFFFu;
-    uint32_t e = ex + 896u, f = m;                     // normal: exponent rebased from bias 127 to 1023
-    if (ex == 0xFFu) e = 0x7FFu;                       // infinity / NaN
-    if (ex == 0u) {
-        if (m == 0u) { e = 0u; }                       // zero
-        else {                                         // subnormal: m * 2^-149, leading bit at p
-            const int p = 31 - __clz(m);
-            e = (uint32_t)(p + 874);                   // p - 149 + 1023
-            f = (m << (23 - p)) & 0x7FFFFFu;
-        }
-    }
-    return __hiloint2double((int)(sign | (e << 20) | (f >> 3)), (int)(f << 29));
-}
-
-
-// Largest running-sum magnitude below which adding a chunk partial of product
-// (i, j) in FP32 is provably exact: every partial is an integer multiple of the
-// unit u = 2^(vA_i + vB_j - 16), so any sum of magnitude below 2^24 u is
-// representable, and rounding is monotone, so a rounded sum below 2^24 u was
-// exact.  0 (always take the error-free path, renormalising every time) when
-// the levels are unknown or the bound is not a normal float; +inf for a
-// product of an all-zero slice.
-__device__ __forceinline__ float bound_of_levels(int a, int b)
-{
-    if (a == kZeroLevel || b == kZeroLevel) return __int_as_float(0x7F800000);
-    const int e = a + b + 8;                          // 2^24 * 2^(a + b - 16)
-    if (e < -126 || e > 127) return 0.0f;
-    return __int_as_float((e + 127) << 23);
-}
-
-__device__ __forceinline__ float exact_bound(const int32_t *vA, const int32_t *vB, int i, int j)
-{
-    if (!vA) return 0.0f;
-    return bound_of_levels(vA[i], vB[j]);
-}
-
-// The same bound with levels per row of A (vA[6][M]) and per column of B
-// (vB[6][N]), the vector scaling of Eq. (ozakiscaled): element (row, col) has
-// unit 2^(vA_i[row] + vB_j[col] - 16), so a thread summing columns col0 ..
-// col0 + ncols - 1 of one row may add plainly below 2^24 of the smallest of
-// its units (a column or row whose slice is all zero contributes nothing).
-__device__ __forceinline__ float exact_bound_rowcol(const int32_t *vA, const int32_t *vB, int M, int N, int i, int j,
-                                                    int row, int col0, int ncols)
-{
-    const int a = row < M ? vA[(int64_t)i * M + row] : kZeroLevel;
-    if (a == kZeroLevel) return __int_as_float(0x7F800000);
-    int bmin = 0x7FFFFFFF;
-    for (int c = 0; c < ncols; ++c) {
-        const int col = col0 + c;
-        if (col < N) {
-            const int b = vB[(int64_t)j * N + col];
-            if (b != kZeroLevel) bmin = b < bmin ? b : bmin;
-        }
-    }
-    if (bmin == 0x7FFFFFFF) return __int_as_float(0x7F800000);
-    return bound_of_levels(a, bmin);
-}
-
-// 16 consecutive 32-bit TMEM columns of this thread's lane: load / store.
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16])
-{
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr)
-        : "memory");
-}
-
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16])
-{
-    asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
-        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
-        ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
-          "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
-        : "memory");
-}
-
-__device__ __forceinline__ uint32_t tmem_ld1(uint32_t taddr)
-{
-    uint32_t r;
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(r) : "r"(taddr) : "memory");
-    return r;
-}
-
-__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&r)[8])
-{
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-                 : "r"(taddr)
-                 : "memory");
-}
-
-__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
-
-
-// Error-free sum of two FP32 values (Knuth's TwoSum): s = fl(a + b), a + b = s + e.
-__device__ __forceinline__ float two_sum(float a, float b, float &e)
-{
-    const float s = __fadd_rn(a, b);
-    const float bb = __fsub_rn(s, a);
-    e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
-    return s;
-}
 
 // TAIL: add the merged tail T (an M x N FP32 matrix) once after the last product.
 template <int NPROD, bool ROWCOL, bool TAIL>
@@ -505,6 +390,11 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     }
 }
 
+// Per-SM rate of the 128 x 128 kernel relative to the 128 x 256 one (measured
+// at 8192^3 with 21 products: 1128 against 1437 TFLOP/s executed, with 27 and
+// 14 waves of CTAs).
+constexpr double kF64RateNarrow = 0.76;
+
 template <int NPROD, bool ROWCOL, bool TAIL = false>
 cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
                     const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, double *acc, uint32_t *flags,
@@ -525,7 +415,7 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
 
 }  // namespace
 
-cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
+static cudaError_t launch_prodsum_f64_narrow(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
                                int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
                                bool rowcol, const float *T, int64_t ldt)
@@ -550,6 +440,45 @@ cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *
                    : run_f64<21, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
     default: return cudaErrorInvalidValue;
     }
+}
+
+// Tile shape of the FP64 product-sum.  128 x 256 (prodsum_f64w.cu) takes in
+// 0.75x the operand bytes per FLOP of 128 x 128 and is faster per SM, but
+// gives half as many CTAs; the choice maximises (SMs kept busy over the waves)
+// x (relative per-SM rate), as for the FP32 product-sum.  Both shapes form
+// the same exact per-product sums and fold them in the same order, so C does
+// not depend on the choice.  EMU_F64_TILE=128x128 / 128x256 forces one.
+cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
+                               int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
+                               int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
+                               bool rowcol, const float *T, int64_t ldt)
+{
+    static const int forced = [] {
+        const char *e = std::getenv("EMU_F64_TILE");
+        if (!e || std::strncmp(e, "128x", 4) != 0) return 0;
+        return std::strcmp(e + 4, "256") == 0 ? 256 : std::strcmp(e + 4, "128") == 0 ? 128 : 0;
+    }();
+    int bn = forced;
+    if (bn == 0) {
+        int dev = 0, sms = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+            sms = 152;
+        const int widths[2] = {256, 128};
+        const double rate[2] = {1.0, kF64RateNarrow};
+        double best = -1.0;
+        for (int i = 0; i < 2; ++i) {
+            const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + widths[i] - 1) / widths[i]);
+            const int64_t waves = (tiles + sms - 1) / sms;
+            const double score = rate[i] * (double)tiles / (double)(waves * sms);
+            if (score > best * 1.02) { best = score; bn = widths[i]; }   // prefer the wider tile on near ties
+        }
+    }
+    if (bn == 256)
+        return launch_prodsum_f64_wide(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane,
+                                       rowcol, T, ldt);
+    return launch_prodsum_f64_narrow(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane,
+                                     rowcol, T, ldt);
 }
 
 }  // namespace emu

@@ -495,8 +495,11 @@ __device__ __forceinline__ int f64_verify_levels(const WsHeader *ws, int slot, i
     return ff;
 }
 
-// One thread: publishes v_out and the slice flag of the levels actually used.
-__device__ __forceinline__ void f64_finalize(WsHeader *ws, int slot, int32_t *v_out)
+// One thread: publishes v_out and the slice flag of the levels actually used:
+// those of slices 0 .. nlev-1, the only ones a product-sum of nlev diagonals
+// reads (the checked general form of the speculative pass, and the literal
+// passes, examine all six levels).
+__device__ __forceinline__ void f64_finalize(WsHeader *ws, int slot, int32_t *v_out, int nlev = 6)
 {
     int v[6];
     final_levels(ws, slot, 6, v);
@@ -504,8 +507,9 @@ __device__ __forceinline__ void f64_finalize(WsHeader *ws, int slot, int32_t *v_
         for (int r = 0; r < 6; ++r) v_out[r] = v[r];
     const int ff = ws->fix_from[slot];
     const uint32_t keep = (1u << ff) - 1u;                       // levels taken from the fused pass
+    const uint32_t used = (1u << nlev) - 1u;
     const uint32_t sb = ws->slice_bad[slot];
-    const uint32_t bad = (sb & keep & 0x3Fu) | ((sb >> 8) & ~keep & 0x3Fu);
+    const uint32_t bad = ((sb & keep) | ((sb >> 8) & ~keep)) & used;
     if (bad) atomicOr(&ws->flags, (uint32_t)EMU_FLAG_SLICE);
 }
 

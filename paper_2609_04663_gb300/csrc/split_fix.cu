@@ -26,7 +26,7 @@ f64_fix_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t
         if (blockIdx.x == 0 && threadIdx.x == 0) {
             for (int r = 0; r < 6; ++r) ws->v[slot][r] = v[r];
             ws->fix_from[slot] = 6;
-            f64_finalize(ws, slot, v_out);
+            f64_finalize(ws, slot, v_out, nlev);
         }
         return;
     }
@@ -48,7 +48,7 @@ f64_fix_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t
     split_tile_pass<double, 2, TRANSPOSE>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, nullptr, nullptr,
                                           blockIdx.x, gridDim.x, smdyn);
     grid_sync(ws, slot);
-    if (blockIdx.x == 0 && threadIdx.x == 0) f64_finalize(ws, slot, v_out);
+    if (blockIdx.x == 0 && threadIdx.x == 0) f64_finalize(ws, slot, v_out, nlev);
 }
 
 }  // namespace

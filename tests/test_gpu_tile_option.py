@@ -1,4 +1,4 @@
-"""The FP32 product-sum's tile shapes (EMU_F32_TILE=128x256 / 128x128 /
+"""The product-sums' tile shapes. FP32 (EMU_F32_TILE=128x256 / 128x128 /
 128x64 forces one; unset, the library picks by tile count): every shape
 issues the same MMAs in the same order for each output element, so C must
 be bit-identical across shapes and within the FP32-mode bar of the oracle.
@@ -49,3 +49,72 @@ def test_f32_tile_shapes_parity_and_bit_identity():
     assert len(ref) == 4
     for tile in ("128x256", "128x128", "128x64"):
         assert _run(tile) == ref, tile
+
+
+CHILD64 = r"""
+import hashlib, sys
+sys.path.insert(0, {root!r})
+sys.path.insert(0, {tests!r})
+import numpy as np
+import oracle, synth
+import paper_2609_04663_gb300 as emu
+from helpers import device, to_dev
+dev = device()
+
+def digest(tag, C):
+    print("digest", tag, hashlib.sha256(C.tobytes()).hexdigest())
+
+# whole-matrix levels, Algorithm 2: ragged tiles, tiny and multi-chunk K, every product count
+for M, N, K, seed, nprod in [(300, 333, 700, 1, 21), (129, 257, 33, 3, 6), (256, 512, 1024, 8, 10),
+                             (520, 130, 300, 5, 15)]:
+    A, B = synth.gemm_inputs("f64", M, N, K, seed)
+    C, ws = emu.gemm_f64(to_dev(A, dev), to_dev(B, dev), nprod)
+    assert emu.read_flags(ws) == 0
+    Cn = C.cpu().numpy()
+    assert np.array_equal(Cn, oracle.gemm_f64(A, B, nprod)[0]), (M, N, K, nprod)
+    digest((M, N, K, nprod), Cn)
+# positive entries: every running sum passes 2^24 units, so the carries into the low words run
+A, B = synth.gemm_inputs("f64", 200, 300, 8192, 11)
+A, B = np.abs(A), np.abs(B)
+C, ws = emu.gemm_f64(to_dev(A, dev), to_dev(B, dev), 21)
+assert emu.read_flags(ws) == 0
+Cn = C.cpu().numpy()
+for r in (0, 77, 199):
+    assert np.array_equal(Cn[r], oracle.gemm_f64(A, B, 21, rows=(r, r + 1))[0][0]), r
+digest("carry", Cn)
+# levels per row / column (the TwoSum and per-element carry paths)
+A, B = synth.gemm_inputs("f64", 260, 300, 1000, 12)
+A = A * np.exp2(np.arange(260) % 7 - 3)[:, None]
+C, ws = emu.gemm_f64_rowcol(to_dev(A, dev), to_dev(B, dev), 15)
+assert emu.read_flags(ws) == 0
+Cn = C.cpu().numpy()
+assert np.array_equal(Cn, oracle.gemm_f64_rowcol(A, B, 15)[0])
+digest("rowcol", Cn)
+# merged tail: the head is the product-sum, the tail added last
+A, B = synth.gemm_inputs("f64", 300, 400, 600, 13)
+C, ws = emu.gemm_f64_merged(to_dev(A, dev), to_dev(B, dev), 21, 4)
+assert emu.read_flags(ws) == 0
+digest("merged", C.cpu().numpy())
+"""
+
+
+def _run64(tile):
+    env = dict(os.environ)
+    env.pop("EMU_F64_TILE", None)
+    if tile:
+        env["EMU_F64_TILE"] = tile
+    code = CHILD64.format(root=ROOT, tests=os.path.join(ROOT, "tests"))
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=900)
+    assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-2000:]
+    return [line for line in r.stdout.splitlines() if line.startswith("digest")]
+
+
+def test_f64_tile_shapes_parity_and_bit_identity():
+    """The FP64 product-sum's tile shapes (EMU_F64_TILE=128x128 / 128x256):
+    both form the same exact per-product sums and add them in Algorithm 2's
+    order, so C must equal the oracle bit for bit with either shape, through
+    the plain, carry, per-row/column and merged-tail paths."""
+    ref = _run64(None)
+    assert len(ref) == 7
+    for tile in ("128x256", "128x128"):
+        assert _run64(tile) == ref, tile

@@ -78,11 +78,10 @@ def test_noalloc_limit_and_flags():
     dev = device()
     torch = emu._torch()
     flags = torch.zeros((1,), dtype=torch.int32, device=dev)
-    # planes 512 + 2 * 12 * n * n plus the FP64 accumulator 8 * roundup(n, 128)^2 must fit 40 MiB:
-    # n = 1024 fits, 1184 does not
+    # planes 512 + 2 * 12 * n * n plus the FP64 accumulator 8 * roundup(n, 128) * roundup(n, 256)
+    # must fit 40 MiB: n = 1024 fits, 1184 does not
     def need(n):
-        r = (n + 127) // 128 * 128
-        return 512 + 2 * 6 * n * n * 2 + 8 * r * r
+        return 512 + 2 * 6 * n * n * 2 + 8 * ((n + 127) // 128 * 128) * ((n + 255) // 256 * 256)
     n = 1024
     assert need(n) <= SCRATCH_BYTES < need(1184)
     A, B = synth.gemm_inputs("f64", n, n, n, 3)
