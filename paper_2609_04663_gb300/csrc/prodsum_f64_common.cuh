@@ -34,6 +34,17 @@ __device__ __forceinline__ double widen_exact(float x)
 }
 
 
+// The same widening for a zero or normal FP32 value only (five integer
+// operations): rebias the exponent field by 1023 - 127 and move the
+// significand's low three bits into the low word.  Not for subnormals,
+// infinities or NaNs.
+__device__ __forceinline__ double widen_normal(float x)
+{
+    const uint32_t u = __float_as_uint(x), a = u & 0x7FFFFFFFu;
+    const uint32_t hi = (u & 0x80000000u) | (a ? (a >> 3) + 0x38000000u : 0u);
+    return __hiloint2double((int)hi, (int)(u << 29));
+}
+
 // Largest running-sum magnitude below which adding a chunk partial of product
 // (i, j) in FP32 is provably exact: every partial is an integer multiple of the
 // unit u = 2^(vA_i + vB_j - 16), so any sum of magnitude below 2^24 u is

@@ -294,10 +294,14 @@ prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                 }
             }
             if (!ok) break;
-            // C <- fl64(C + (hi + lo)) in L2, column by column (product 0: a plain store)
+            // C <- fl64(C + (hi + lo)) in L2, column by column (product 0: a plain store).
+            // The sums are integer multiples of the smallest unit of this thread's
+            // elements, 2^-24 bound; when that unit is a normal FP32 number so is
+            // every nonzero sum, and the short widening is exact.
+            const bool normal_sums = bound >= 0x1p-102f;
 #pragma unroll
             for (int j = 0; j < Cfg::COLS; ++j) {
-                double sq = widen_exact(hi[j]);
+                double sq = normal_sums ? widen_normal(hi[j]) : widen_exact(hi[j]);
                 if (((dirty >> (j >> 4)) & 1u) && j < lim) sq = __dadd_rn(sq, widen_exact(lrow[2 * j]));   // exact
                 if (q == 0) tacc[j * kBM] = sq;
                 else red_add_f64(tacc + j * kBM, sq);

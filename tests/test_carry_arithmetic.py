@@ -5,7 +5,9 @@ exact bound, or one chunk partial) split by the add-subtract projection with
 the constant 1.5 * 2^35 u into a multiple of 2^12 u and a remainder of at
 most 2^11 u, both exact; a coarse sum that takes the two coarse parts of a
 running sum and a partial per carry stays exact for 2^11 carries (below
-2^36 u)."""
+2^36 u).  Also the product-sums' short FP32 -> FP64 widening for zero and
+normal values, restated on the bit patterns and checked against numpy's
+conversion."""
 import numpy as np
 
 F = np.float32
@@ -48,3 +50,25 @@ def test_coarse_sum_stays_exact_for_2048_carries():
         exact += int(round(float(c) / float(u)))
     assert int(round(float(s2) / float(u))) == exact
     assert abs(exact) < 2**36
+
+
+def _widen_normal(x):
+    """The FP64 product-sum's short FP32 -> FP64 widening restated on the bit
+    patterns: rebias the exponent field by 1023 - 127 and keep the
+    significand; zeros keep their sign."""
+    u = np.asarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    a = u & 0x7FFFFFFF
+    hi = (u & 0x80000000) | np.where(a != 0, (a >> 3) + 0x38000000, 0)
+    lo = (u << 29) & 0xFFFFFFFF
+    return ((hi << 32) | lo).view(np.float64)
+
+
+def test_short_widening_is_exact_for_zero_and_normal_values():
+    rng = np.random.default_rng(3)
+    bits = rng.integers(0, 2**32, size=400000, dtype=np.uint64).astype(np.uint32)
+    x = bits.view(np.float32)
+    e = (bits >> 23) & 0xFF
+    x = x[(e > 0) & (e < 255)]                                  # normal values only
+    x = np.concatenate([x, np.float32([0.0, -0.0, 2.0**-126, -2.0**-126, 3.4028235e38, -1.0, 1.0])])
+    w = _widen_normal(x)
+    assert np.array_equal(w.view(np.uint64), x.astype(np.float64).view(np.uint64))
