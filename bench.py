@@ -220,6 +220,9 @@ class Case:
         self.gemm_ws = None
         if self.merge_from is not None:
             self.gemm_ws = emu.workspace(emu.emu_gemm_f64_merged_workspace_bytes(M, N, K), dev)
+        # the product-sum kernel that runs: FP64 mode has a 128 x 128 and a 128 x 256 tile
+        self.kernel = "prodsum_f32" if self.mode == 32 else \
+            "prodsum_f64w" if emu.emu_prodsum_f64_tile_columns(M, N) == 256 else "prodsum_f64"
         self.flop = 2.0 * M * N * K
         self.exec_flop = self.flop * (6 if self.mode == 32 else self.nprod)
         # kernels of ours per step: FP32 split = 1 launch, FP64 split = 10, product-sum = 1
@@ -468,11 +471,9 @@ def gpu_arm(args, rank, world, local):
     roofline = {"bound": "tensor", "achieved": achieved, "peak": pk["bf16_burst"], "unit": "TFLOP/s",
                 "frac": achieved / pk["bf16_burst"],
                 "peak_source": f"{pk['source']} bf16 burst (cuBLAS 8192^3); sustained {pk['bf16_sustained']}",
-                "kernel": "gemm_f32_fused_kernel" if case.fused else
-                          "prodsum_f32_kernel" if case.mode == 32 else "prodsum_f64_kernel",
+                "kernel": "gemm_f32_fused_kernel" if case.fused else case.kernel + "_kernel",
                 "traffic": None if case.fused or case.merge_from else
-                           kernel_traffic("prodsum_f32" if case.mode == 32 else "prodsum_f64",
-                                          name if case.mode == 32 else f"{name}_np{case.nprod}")}
+                           kernel_traffic(case.kernel, name if case.mode == 32 else f"{name}_np{case.nprod}")}
     flags = case.emu.read_flags(case.gemm_ws if case.gemm_ws is not None else case.ws)
     e2e = None if args.no_e2e else time_e2e(case, max(2, min(args.steps, 5)), 1, world)
     split_gbs = case.split_bytes() / (split_ms / 1e3) / 1e9
@@ -535,9 +536,9 @@ def variants(args, rank, world, pk):
                     "prodsum_ms": pm, "split_ms": statistics.mean(res["split_ms"]),
                     "executed_tflops": case.exec_flop / (pm / 1e3) / 1e12,
                     "frac_of_bf16_peak": case.exec_flop / (pm / 1e3) / 1e12 / pk["bf16_burst"],
+                    "kernel": case.kernel,
                     "traffic": None if fused or merge_from else
-                               kernel_traffic("prodsum_f32" if case.mode == 32 else "prodsum_f64",
-                                              name if case.mode == 32 else f"{name}_np{case.nprod}"),
+                               kernel_traffic(case.kernel, name if case.mode == 32 else f"{name}_np{case.nprod}"),
                     "flags": case.emu.read_flags(case.gemm_ws if case.gemm_ws is not None else case.ws)}
         del case
         torch.cuda.empty_cache()

@@ -273,8 +273,15 @@ emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
 /* Workspace bytes for emu_prodsum_f32 (mode 32: the flag word) and
  * emu_prodsum_f64 (mode 64: the flag word and the FP64 accumulator of the
  * product-outer sum, 8 bytes per element of C rounded up to 128 x 128
- * tiles).  0 for negative sizes or another mode. */
+ * tiles, or to 128 x 256 tiles where that is larger).  0 for negative sizes
+ * or another mode. */
 size_t emu_prodsum_workspace_bytes(int mode, int64_t M, int64_t N);
+
+/* Output-tile width (128 or 256 columns; 128 rows either way) that the
+ * FP64-mode product-sum picks for an M x N result, unless EMU_F64_TILE
+ * forces one.  The paper has no counterpart: both widths give identical
+ * results, and the call only reports which kernel runs.  0 for sizes < 1. */
+int emu_prodsum_f64_tile_columns(int64_t M, int64_t N);
 
 /* Product-sum alone for FP64 mode, Eq. (fp64reconstruction), summed as in
  * emu_gemm_f64: A planes [6][M][ldcomp], B planes [6][N][ldcomp]; nprod in

@@ -44,6 +44,7 @@ _SIGS = {
     "emu_gemm_host_workspace_bytes": ("size", ["i", "l", "l", "l"]),
     "emu_gemm_ex_workspace_bytes": ("size", ["i", "l", "l", "l"]),
     "emu_prodsum_workspace_bytes": ("size", ["i", "l", "l"]),
+    "emu_prodsum_f64_tile_columns": ("i", ["l", "l"]),
     "emu_split_f64_rowcol_workspace_bytes": ("size", ["l"]),
     "emu_split_f64_rowcol": ("i", ["p", "l", "l", "l", "i", "p", "l", "p", "p", "size", "p"]),
     "emu_gemm_f64_rowcol_workspace_bytes": ("size", ["l", "l", "l"]),
@@ -110,6 +111,7 @@ emu_gemm_f64_noalloc = _mk("emu_gemm_f64_noalloc")
 emu_gemm_host_workspace_bytes = _mk("emu_gemm_host_workspace_bytes")
 emu_gemm_ex_workspace_bytes = _mk("emu_gemm_ex_workspace_bytes")
 emu_prodsum_workspace_bytes = _mk("emu_prodsum_workspace_bytes")
+emu_prodsum_f64_tile_columns = _mk("emu_prodsum_f64_tile_columns")
 emu_split_f64_rowcol_workspace_bytes = _mk("emu_split_f64_rowcol_workspace_bytes")
 emu_split_f64_rowcol = _mk("emu_split_f64_rowcol")
 emu_gemm_f64_rowcol_workspace_bytes = _mk("emu_gemm_f64_rowcol_workspace_bytes")

@@ -250,6 +250,12 @@ emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_
     return cuda_status(e);
 }
 
+int emu_prodsum_f64_tile_columns(int64_t M, int64_t N)
+{
+    if (M < 1 || N < 1) return 0;
+    return f64_tile_columns(M, N);
+}
+
 size_t emu_prodsum_workspace_bytes(int mode, int64_t M, int64_t N)
 {
     if (M < 0 || N < 0 || (mode != 32 && mode != 64)) return 0;

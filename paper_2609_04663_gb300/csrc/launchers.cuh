@@ -73,6 +73,8 @@ cudaError_t launch_prodsum_tail(int64_t M, int64_t N, int64_t K, const uint16_t 
                                 int64_t ldcomp, int L, int d, float *T, int64_t ldt, uint32_t *flags,
                                 cudaStream_t st);
 
+// Tile width (128 or 256) the FP64 product-sum picks for an M x N result.
+int f64_tile_columns(int64_t M, int64_t N);
 // The FP64 product-sum on 128 x 256 tiles (prodsum_f64w.cu); launch_prodsum_f64
 // calls it when that tile shape is chosen.  acc: f64_acc_bytes(M, N) bytes.
 cudaError_t launch_prodsum_f64_wide(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,

@@ -448,10 +448,7 @@ static cudaError_t launch_prodsum_f64_narrow(int64_t M, int64_t N, int64_t K, co
 // x (relative per-SM rate), as for the FP32 product-sum.  Both shapes form
 // the same exact per-product sums and fold them in the same order, so C does
 // not depend on the choice.  EMU_F64_TILE=128x128 / 128x256 forces one.
-cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
-                               int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
-                               int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
-                               bool rowcol, const float *T, int64_t ldt)
+int f64_tile_columns(int64_t M, int64_t N)
 {
     static const int forced = [] {
         const char *e = std::getenv("EMU_F64_TILE");
@@ -474,7 +471,15 @@ cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *
             if (score > best * 1.02) { best = score; bn = widths[i]; }   // prefer the wider tile on near ties
         }
     }
-    if (bn == 256)
+    return bn;
+}
+
+cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
+                               int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
+                               int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
+                               bool rowcol, const float *T, int64_t ldt)
+{
+    if (f64_tile_columns(M, N) == 256)
         return launch_prodsum_f64_wide(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane,
                                        rowcol, T, ldt);
     return launch_prodsum_f64_narrow(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane,

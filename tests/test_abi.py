@@ -132,3 +132,14 @@ def test_rowcol_argument_checks_need_no_gpu(lib):
     assert need > emu.emu_gemm_workspace_bytes(64, 300, 200, 700)
     assert emu.emu_gemm_f64_rowcol(300, 200, 700, P, 700, P, 200, P, 200, 6, P, need - 1, None) == 3
     assert emu.emu_gemm_f64_rowcol(4, 4, 4, P, 4, P, 4, P, 4, 11, P, 1 << 30, None) == 1      # nprod
+
+
+def test_f64_tile_width_report(lib):
+    # no GPU here: the launcher assumes 152 SMs; with EMU_F64_TILE unset a
+    # large square result takes the 128 x 256 tile, a small one 128 x 128
+    if os.environ.get("EMU_F64_TILE"):
+        pytest.skip("EMU_F64_TILE forces a tile width")
+    assert emu.emu_prodsum_f64_tile_columns(8192, 8192) == 256
+    assert emu.emu_prodsum_f64_tile_columns(1024, 1024) == 128
+    assert emu.emu_prodsum_f64_tile_columns(0, 8) == 0
+
