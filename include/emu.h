@@ -78,6 +78,11 @@ typedef enum {
  * per-level maxima of the FP64 split).  mode is 32 or 64. */
 size_t emu_split_workspace_bytes(int mode);
 
+/* The splits take `transpose` (the B operand's K-major planes) and a plane
+ * row pitch `ldcomp` in place of a layout selector: planes in memory are
+ * always planar rows, and the shared-memory swizzle the tensor cores need is
+ * applied by the tensor memory accelerator when a tile is loaded. */
+
 /* FP32 three-slice split, Eq. (fp32split) / Algorithm 1 (Split_FP32):
  *   A_r = fl_BF16(A^(r)), A^(r+1) = fl32(A^(r) - A_r), r = 0, 1, 2,
  * fl_BF16 = round to nearest, ties to even (Section 4.2).
@@ -132,10 +137,6 @@ emu_status emu_gemm_f64_rowcol(int64_t M, int64_t N, int64_t K, const double *A,
                                const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,
                                void *ws, size_t ws_bytes, emu_stream_t stream);
 
-/* Workspace bytes for emu_gemm_f32 (mode 32) / emu_gemm_f64 (mode 64):
- * the flag word plus the slice planes of A (M x K) and B (K x N), and in
- * mode 64 the product-sum's FP64 accumulator (8 bytes per element of C,
- * rounded up to 128 x 128 tiles). */
 /* emu_split_f64 for a product-sum that reads slices 0 .. nslices-1 only
  * (nslices = d = 3, 4, 5, 6 for nprod = 6, 10, 15, 21): the fused pass forms
  * and writes only those planes, and only their levels are verified.  Planes
@@ -148,6 +149,11 @@ emu_status emu_split_f64_slices(const double *X, int64_t rows, int64_t cols, int
                                 uint16_t *comps, int64_t ldcomp, int nslices, int32_t *v_out, void *ws,
                                 size_t ws_bytes, emu_stream_t stream);
 
+/* Workspace bytes for emu_gemm_f32 (mode 32) / emu_gemm_f64 (mode 64):
+ * the flag word plus the slice planes of A (M x K) and B (K x N), and in
+ * mode 64 the product-sum's FP64 accumulator (8 bytes per element of C,
+ * rounded up to 128 x 128 tiles, or to 128 x 256 tiles where that is
+ * larger). */
 size_t emu_gemm_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K);
 
 /* FP32-mode emulated GEMM, Algorithm 1: C (M x N, ldc) = A (M x K, lda) . B
@@ -177,8 +183,8 @@ emu_status emu_gemm_f32_fused(int64_t M, int64_t N, int64_t K, const float *A, i
  * cores per K-chunk of 256 (every chunk partial is exact, Section 5.2), the
  * partials are summed exactly, and the total is added once into the FP64
  * result: C <- fl64(C + fl32(A_i B_j)).  C equals the oracle's product-outer
- * order bit for bit.  C also serves as the FP64 accumulator while the kernel
- * runs. */
+ * order bit for bit.  The FP64 accumulator lives in the workspace; C serves
+ * as scratch for low-order words of the exact sums while the kernel runs. */
 emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda,
                         const double *B, int64_t ldb, double *C, int64_t ldc, int nprod,
                         void *ws, size_t ws_bytes, emu_stream_t stream);
