@@ -188,7 +188,7 @@ class Case:
     """Device-resident inputs, planes and output of one GEMM workload."""
 
     def __init__(self, name: str, rank: int, nprod: int | None = None, fused: bool = False,
-                 merge_from: int | None = None):
+                 merge_from: int | None = None, api: bool = False):
         import numpy as np
         import torch
         import synth
@@ -203,6 +203,8 @@ class Case:
         self.fused = fused and self.mode == 32
         # FP64 only: the tail diagonals from merge_from on in one FP32 sum (emu_gemm_f64_merged)
         self.merge_from = merge_from if self.mode == 64 else None
+        # the whole GEMM through the public call (emu_gemm_f32 / emu_gemm_f64), timed as one region
+        self.api = api and not self.fused and self.merge_from is None
         # each rank draws its own problem (replicas): offset the seed by the rank
         A, B = synth.gemm_inputs(kind, M, N, K, seed + 1000003 * rank, phi=phi)
         self.A_host, self.B_host = A, B
@@ -220,6 +222,8 @@ class Case:
         self.gemm_ws = None
         if self.merge_from is not None:
             self.gemm_ws = emu.workspace(emu.emu_gemm_f64_merged_workspace_bytes(M, N, K), dev)
+        if self.api:
+            self.gemm_ws = emu.workspace(emu.emu_gemm_workspace_bytes(self.mode, M, N, K), dev)
         # the product-sum kernel that runs: FP64 mode has a 128 x 128 and a 128 x 256 tile
         self.kernel = "prodsum_f32" if self.mode == 32 else \
             "prodsum_f64w" if emu.emu_prodsum_f64_tile_columns(M, N) == 256 else "prodsum_f64"
@@ -229,12 +233,14 @@ class Case:
         self.launches = 1 if self.fused else (2 * 1 + 1) if self.mode == 32 else (2 * 10 + 1)
         if self.merge_from is not None:
             self.launches += 1                    # the tail kernel
+        if self.api and self.mode == 32:
+            self.launches = 2                     # both splits in one launch, then the product-sum
         del np
 
     def split(self, stream):
         emu, st = self.emu, stream.cuda_stream
         ws, n = self.ws.data_ptr(), self.ws.numel()
-        if self.fused or self.merge_from is not None:
+        if self.fused or self.merge_from is not None or self.api:
             return                                # the whole GEMM runs in prodsum()
         if self.mode == 32:
             r = emu.emu_split_f32(self.A.data_ptr(), self.M, self.K, self.A.stride(0), 0, self.Ap.data_ptr(),
@@ -252,7 +258,14 @@ class Case:
 
     def prodsum(self, stream):
         emu, st = self.emu, stream.cuda_stream
-        if self.merge_from is not None:
+        if self.api and self.mode == 32:
+            r = emu.emu_gemm_f32(self.M, self.N, self.K, self.A.data_ptr(), self.K, self.B.data_ptr(), self.N,
+                                 self.C.data_ptr(), self.N, self.gemm_ws.data_ptr(), self.gemm_ws.numel(), st)
+        elif self.api:
+            r = emu.emu_gemm_f64(self.M, self.N, self.K, self.A.data_ptr(), self.K, self.B.data_ptr(), self.N,
+                                 self.C.data_ptr(), self.N, self.nprod, self.gemm_ws.data_ptr(), self.gemm_ws.numel(),
+                                 st)
+        elif self.merge_from is not None:
             r = emu.emu_gemm_f64_merged(self.M, self.N, self.K, self.A.data_ptr(), self.K, self.B.data_ptr(), self.N,
                                         self.C.data_ptr(), self.N, self.nprod, self.merge_from,
                                         self.gemm_ws.data_ptr(), self.gemm_ws.numel(), st)
@@ -290,12 +303,14 @@ def time_device(case: Case, steps: int, warmup: int, world: int, flush: bool):
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     epoch0 = time.time()
+    one_region = case.api or case.fused or case.merge_from is not None
     for i in range(steps):
         if flush:
             scratch.fill_(i & 0xFF)              # evict the previous step from L2 (not timed)
         ev[i][0].record(stream)
-        case.split(stream)
-        ev[i][1].record(stream)
+        if not one_region:
+            case.split(stream)
+            ev[i][1].record(stream)
         case.prodsum(stream)
         ev[i][2].record(stream)
     torch.cuda.synchronize()
@@ -303,8 +318,8 @@ def time_device(case: Case, steps: int, warmup: int, world: int, flush: bool):
     torch.cuda.synchronize()
     wall = time.perf_counter() - t0
     window = (epoch0, time.time())
-    split_ms = [a.elapsed_time(b) for a, b, _ in ev]
-    prod_ms = [b.elapsed_time(c) for _, b, c in ev]
+    split_ms = [0.0 if one_region else a.elapsed_time(b) for a, b, _ in ev]
+    prod_ms = [a.elapsed_time(c) if one_region else b.elapsed_time(c) for a, b, c in ev]
     step_ms = [a.elapsed_time(c) for a, _, c in ev]
     return {"step_ms": step_ms, "split_ms": split_ms, "prodsum_ms": prod_ms, "wall_s": wall, "window": window}
 
@@ -511,7 +526,7 @@ def variants(args, rank, world, pk):
     # 1024-8192 (16384 is the headline); FP64 4096^3 at 6/10/15/21 products;
     # FP64 8192^3 scaled inputs at 21 and 10 products; the large-K shape
     # 2048 x 2048 x 65536 in FP32 and at every FP64 product count.
-    todo = [("fp32_n256", None), ("fp32_n1024", None), ("fp32_n2048", None), ("fp32_n4096", None),
+    todo = [("fp32_n256", "api"), ("fp32_n1024", "api"), ("fp32_n2048", "api"), ("fp32_n4096", None),
             ("fp32_n8192", None), ("fp64_n4096", 6), ("fp64_n4096", 10), ("fp64_n4096", 15), ("fp64_n4096", 21),
             ("fp64_scaled_phi4_n8192", 21), ("fp64_scaled_phi4_n8192", 10), ("fp64_scaled_phi0.5_n8192", 21),
             ("fp64_scaled_phi2_n8192", 21), ("fp32_largek", None), ("fp64_largek", 6), ("fp64_largek", 10),
@@ -522,14 +537,14 @@ def variants(args, rank, world, pk):
                  ("fp32_cancel_n4096", None), ("fp64_cancel_n4096", 21)]
     torch = __import__("torch")
     for name, nprod in todo:
-        fused = nprod == "fused"
+        fused, api = nprod == "fused", nprod == "api"
         merge_from = nprod[1] if isinstance(nprod, tuple) else None
-        nprod = nprod[0] if isinstance(nprod, tuple) else None if fused else nprod
-        case = Case(name, rank, nprod, fused=fused, merge_from=merge_from)
+        nprod = nprod[0] if isinstance(nprod, tuple) else None if fused or api else nprod
+        case = Case(name, rank, nprod, fused=fused, merge_from=merge_from, api=api)
         res = time_device(case, max(3, args.variant_steps), 2, world, flush=True)
         t = max_over_ranks(sum(res["step_ms"]) / 1e3, world)
         pm = statistics.mean(res["prodsum_ms"])
-        key = f"{name}" + (f"_np{case.nprod}" if case.mode == 64 else "_fused" if fused else "") + \
+        key = f"{name}" + (f"_np{case.nprod}" if case.mode == 64 else "_fused" if fused else "_gemm" if api else "") + \
             (f"_merged{merge_from}" if merge_from else "")
         out[key] = {"tflops": job_throughput(case.flop, len(res["step_ms"]), world, t),
                     "ms_per_step": 1e3 * t / len(res["step_ms"]),
@@ -537,7 +552,7 @@ def variants(args, rank, world, pk):
                     "executed_tflops": case.exec_flop / (pm / 1e3) / 1e12,
                     "frac_of_bf16_peak": case.exec_flop / (pm / 1e3) / 1e12 / pk["bf16_burst"],
                     "kernel": case.kernel,
-                    "traffic": None if fused or merge_from else
+                    "traffic": None if fused or merge_from or api else
                                kernel_traffic(case.kernel, name if case.mode == 32 else f"{name}_np{case.nprod}"),
                     "flags": case.emu.read_flags(case.gemm_ws if case.gemm_ws is not None else case.ws)}
         del case

@@ -160,7 +160,12 @@ size_t emu_gemm_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K);
  * (K x N, ldb), all FP32 row-major.  Splits A and B into the workspace, then
  * runs the tensor-core product-sum: the 6 products of Eq. (fp32six) are
  * accumulated in one FP32 accumulator over all of K (Section 6.3, FP32
- * reconstruction), so C matches the oracle within FP32 reordering error. */
+ * reconstruction), so C matches the oracle within FP32 reordering error.
+ * When the result has too few 128 x 128 tiles to occupy the GPU, K is split
+ * in two: each half has its own FP32 accumulator and the two are added into
+ * C (cleared first) in L2, one rounding, independent of which half finishes
+ * first; FP32 reductions there flush subnormal sums to zero.  C then differs
+ * from the one-accumulator result by FP32 rounding only. */
 emu_status emu_gemm_f32(int64_t M, int64_t N, int64_t K, const float *A, int64_t lda,
                         const float *B, int64_t ldb, float *C, int64_t ldc, void *ws,
                         size_t ws_bytes, emu_stream_t stream);

@@ -160,9 +160,11 @@ emu_status emu_gemm_f32(int64_t M, int64_t N, int64_t K, const float *A, int64_t
     const int64_t ldk = gemm_ldk(K);
     uint16_t *Ap = reinterpret_cast<uint16_t *>(static_cast<char *>(ws) + kWsHeaderBytes);
     uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(3 * M * ldk * 2, 256));
-    e = launch_split_f32(A, M, K, lda, false, Ap, ldk, h, st);
-    if (e == cudaSuccess) e = launch_split_f32(B, K, N, ldb, true, Bp, ldk, h, st);
-    if (e == cudaSuccess) e = launch_prodsum_f32(M, N, K, Ap, Bp, ldk, C, ldc, &h->flags, st);
+    // both splits in one launch; when the product-sum will split K in two
+    // (few output tiles), the same launch clears C for the halves to add into
+    const bool split_k = f32_split_parts(M, N, K) > 1;
+    e = launch_split_f32_gemm(A, M, K, lda, B, N, ldb, Ap, Bp, ldk, h, split_k ? C : nullptr, ldc, st);
+    if (e == cudaSuccess) e = launch_prodsum_f32(M, N, K, Ap, Bp, ldk, C, ldc, &h->flags, st, 0, 0, split_k);
     return cuda_status(e);
 }
 

@@ -57,12 +57,14 @@ __device__ __forceinline__ void prefetch_l2(const void *p)
     asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
 }
 
-// What one of CONV converter threads holds of a 128 x 32 A tile and a 32 x 256
+// What one of CONV converter threads holds of a 128 x 32 A tile and a 32 x BN
 // B tile: float4 number ct % 8 of A rows ct / 8 + (CONV / 8) i, and B column
-// ct % 256 over the K rows KPT (ct / 256) .. + KPT - 1.
-template <int CONV>
+// ct % BN over the K rows KPT (ct / BN) .. + KPT - 1 (KPT >= 8, so that a
+// thread fills whole 16-byte chunks of its transposed B row).
+template <int BN, int CONV>
 struct FusedTiles {
-    static constexpr int NA = 1024 / CONV, KPT = 32 * 256 / CONV;
+    static constexpr int NA = 1024 / CONV, KPT = 32 * BN / CONV;
+    static_assert(KPT >= 8 && KPT % 8 == 0 && CONV % BN == 0, "converter mapping of the B tile");
     float a[NA][4];
     float b[KPT];
 };
@@ -73,8 +75,8 @@ gemm_f32_fused_kernel(const float *__restrict__ A, int64_t lda, const float *__r
                       int N, int K, float *__restrict__ C, int64_t ldc, uint32_t *flags)
 {
     using Cfg = F32Cfg<BN, KB, STAGES>;
-    static_assert(BN == 256 && KB == 32 && (CONV == 256 || CONV == 512), "converter mapping");
-    using Tiles = FusedTiles<CONV>;
+    static_assert(KB == 32 && (CONV == 256 || CONV == 512), "converter mapping");
+    using Tiles = FusedTiles<BN, CONV>;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -106,7 +108,7 @@ gemm_f32_fused_kernel(const float *__restrict__ A, int64_t lda, const float *__r
     } else {
         const int ct = threadIdx.x - 32;
         const int a_c4 = ct & 7, a_r0 = ct >> 3;
-        const int b_col = ct & 255, b_k0 = (ct >> 8) * Tiles::KPT;
+        const int b_col = ct % BN, b_k0 = (ct / BN) * Tiles::KPT;
         const int bn = n0 + b_col;
         const bool avec = ((lda & 3) == 0) && ((reinterpret_cast<uintptr_t>(A) & 15u) == 0);
 
@@ -135,12 +137,14 @@ gemm_f32_fused_kernel(const float *__restrict__ A, int64_t lda, const float *__r
                     t.b[k] = (bn < N && kb0 + k < K) ? __ldg(bsrc + (int64_t)k * ldb) : 0.0f;
             }
         };
-        // one 128-byte line per thread and operand: A row ct, B K row ct / 8 segment ct % 8
+        // one 128-byte line per thread and operand: A row ct, B K row ct / L segment ct % L
+        // (L = BN / 32 lines per K row of the B tile)
         auto prefetch = [&](int kb) {
+            constexpr int L = BN / 32;
             const int k0 = kb * KB;
             if (ct < kBM && m0 + ct < M) prefetch_l2(A + (int64_t)(m0 + ct) * lda + k0);
-            const int k = k0 + (ct >> 3), n = n0 + 32 * (ct & 7);
-            if (ct < 256 && k < K && n < N) prefetch_l2(B + (int64_t)k * ldb + n);
+            const int k = k0 + ct / L, n = n0 + 32 * (ct % L);
+            if (ct < 32 * L && k < K && n < N) prefetch_l2(B + (int64_t)k * ldb + n);
         };
         uint32_t amax = 0;
         auto store = [&](uint32_t st, const Tiles &t) {
@@ -194,6 +198,7 @@ gemm_f32_fused_kernel(const float *__restrict__ A, int64_t lda, const float *__r
         publish_f32_flags(amax, flags);
         // epilogue: CONV / 128 warps per TMEM lane quarter, an equal share of the columns each
         constexpr int kPart = BN / (CONV / 128);
+        static_assert(kPart % 32 == 0, "epilogue columns come in groups of 32");
         const bool ok = mbar_wait(accum_bar, 0, flags);
         __syncwarp();
         const int part = (warp - 1) >> 2;
@@ -210,18 +215,31 @@ gemm_f32_fused_kernel(const float *__restrict__ A, int64_t lda, const float *__r
 
 }  // namespace
 
-// FP32-mode GEMM with the split in the producer (gemm_f32_fused_kernel).
+template <int BN, int STAGES, int CONV>
+cudaError_t run_fused(int64_t M, int64_t N, int64_t K, const float *A, int64_t lda, const float *B, int64_t ldb,
+                      float *C, int64_t ldc, uint32_t *flags, cudaStream_t st)
+{
+    using Cfg = F32Cfg<BN, 32, STAGES>;
+    auto kern = gemm_f32_fused_kernel<BN, 32, STAGES, CONV>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    if (e != cudaSuccess) return e;
+    const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + BN - 1) / BN);
+    kern<<<(unsigned)tiles, 32 + CONV, Cfg::SMEM, st>>>(A, lda, B, ldb, (int)M, (int)N, (int)K, C, ldc, flags);
+    return cudaGetLastError();
+}
+
+// FP32-mode GEMM with the split in the producer (gemm_f32_fused_kernel), on
+// the tile width the product-sum would take for this result size (128 x 256,
+// 128 x 128 or 128 x 64): every width issues the same MMAs in the same order
+// for each output element, so C does not depend on it.
 cudaError_t launch_gemm_f32_fused(int64_t M, int64_t N, int64_t K, const float *A, int64_t lda, const float *B,
                                   int64_t ldb, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st)
 {
-    constexpr int kConv = 512;
-    using Cfg = F32Cfg<256, 32, 3>;
-    auto kern = gemm_f32_fused_kernel<256, 32, 3, kConv>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
-    if (e != cudaSuccess) return e;
-    const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + 255) / 256);
-    kern<<<(unsigned)tiles, 32 + kConv, Cfg::SMEM, st>>>(A, lda, B, ldb, (int)M, (int)N, (int)K, C, ldc, flags);
-    return cudaGetLastError();
+    switch (f32_tile_columns(M, N)) {
+    case 64: return run_fused<64, 4, 256>(M, N, K, A, lda, B, ldb, C, ldc, flags, st);
+    case 128: return run_fused<128, 4, 256>(M, N, K, A, lda, B, ldb, C, ldc, flags, st);
+    default: return run_fused<256, 3, 512>(M, N, K, A, lda, B, ldb, C, ldc, flags, st);
+    }
 }
 
 }  // namespace emu

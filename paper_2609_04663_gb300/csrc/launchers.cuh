@@ -50,9 +50,22 @@ inline size_t rc_scratch_bytes(int64_t plane_rows) { return (size_t)plane_rows *
 // B planes in elements (0 = dense: M * ldcomp / N * ldcomp), so that a row
 // panel of A or a column panel of B in a larger plane set can be multiplied
 // on its own.
+// c_zeroed: C is zero on entry, so when few output tiles would leave SMs idle
+// the product-sum may split K in two and add both halves into C.
 cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
-                               int64_t a_plane = 0, int64_t b_plane = 0);
+                               int64_t a_plane = 0, int64_t b_plane = 0, bool c_zeroed = false);
+// Both operands of an FP32 GEMM (A: M x K row-major planes, B: K x N K-major
+// planes, row pitch ldcomp, B's planes at Bp) split in one launch; with C
+// non-null the launch also sets the M x N result C (ldc) to zero.
+cudaError_t launch_split_f32_gemm(const float *A, int64_t M, int64_t K, int64_t lda, const float *B, int64_t N,
+                                  int64_t ldb, uint16_t *Ap, uint16_t *Bp, int64_t ldcomp, WsHeader *ws, float *C,
+                                  int64_t ldc, cudaStream_t st);
+// Tile width (256, 128 or 64) the FP32 product-sums pick for an M x N result,
+// and the number of K-parts (1 or 2) the product-sum takes when C is cleared
+// first.
+int f32_tile_columns(int64_t M, int64_t N);
+int f32_split_parts(int64_t M, int64_t N, int64_t K);
 // Eq. (fp32split) and the FP32 product-sum in one kernel: A (M x K, lda) and
 // B (K x N, ldb) FP32 row-major are split inside the product-sum's producer;
 // no planes are written.  flags receives the split's domain flags.

@@ -19,7 +19,46 @@ namespace emu {
 
 namespace {
 
-template <int BN, int KB, int STAGES>
+// Epilogue of one warp for a product-sum split along K: accumulator columns
+// [c0, c1) of the warp's TMEM lane quarter added into C (which starts at zero)
+// by FP32 reductions in L2.  With two K-parts the sum is the same in either
+// order of arrival (0 + a, then a + b, rounded once; FP32 reductions flush
+// subnormal inputs and results to zero).
+__device__ __forceinline__ void reduce_tile(uint32_t tmem, int quarter, int c0, int c1, int m0, int n0, int M, int N,
+                                            float *__restrict__ C, int64_t ldc)
+{
+    tc_fence_after();
+    const int row = m0 + quarter * 32 + lane_id();
+    float *crow = C + (int64_t)row * ldc;
+    const bool vec = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15u) == 0);
+#pragma unroll 1
+    for (int c = c0; c < c1; c += 32) {
+        uint32_t v[32];
+        tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)c, v);
+        tmem_ld_wait();
+        const int col = n0 + c;
+        if (row < M) {
+            if (vec && col + 32 <= N) {
+#pragma unroll
+                for (int j = 0; j < 32; j += 4)
+                    asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(crow + col + j),
+                                 "f"(__uint_as_float(v[j])), "f"(__uint_as_float(v[j + 1])),
+                                 "f"(__uint_as_float(v[j + 2])), "f"(__uint_as_float(v[j + 3])) : "memory");
+            } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    if (col + j < N)
+                        asm volatile("red.global.add.f32 [%0], %1;" ::"l"(crow + col + j), "f"(__uint_as_float(v[j]))
+                                     : "memory");
+            }
+        }
+    }
+}
+
+// SPLIT > 1: the grid holds SPLIT CTAs per output tile, each over its own
+// contiguous range of K-blocks, which add their FP32 accumulators into C (set
+// to zero beforehand) instead of storing them.
+template <int BN, int KB, int STAGES, int SPLIT>
 __global__ void __launch_bounds__(192, 1)
 prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    int M, int N, int K, float *__restrict__ C, int64_t ldc, uint32_t *flags)
@@ -36,9 +75,12 @@ prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     const int warp = threadIdx.x >> 5, lane = lane_id();
     const int tiles_m = (M + kBM - 1) / kBM, tiles_n = (N + BN - 1) / BN;
     int tm, tn;
-    tile_coords(blockIdx.x, tiles_m, tiles_n, tm, tn);
+    const int tiles = tiles_m * tiles_n, part = (int)blockIdx.x / tiles;
+    tile_coords((int)blockIdx.x % tiles, tiles_m, tiles_n, tm, tn);
     const int m0 = tm * kBM, n0 = tn * BN;
-    const int nkb = (K + KB - 1) / KB;
+    const int nkb_all = (K + KB - 1) / KB, per = (nkb_all + SPLIT - 1) / SPLIT;
+    const int kb0 = min(nkb_all, part * per);
+    const int nkb = min(nkb_all, kb0 + per) - kb0;     // K-blocks of this CTA
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) { mbar_init(full0 + 8u * s, 1); mbar_init(empty0 + 8u * s, 1); }
@@ -63,9 +105,10 @@ prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
             const uint32_t st = base + (uint32_t)(s * Cfg::STAGE), fb = full0 + 8u * s;
             mbar_arrive_expect_tx(fb, Cfg::STAGE);
 #pragma unroll
-            for (int r = 0; r < 3; ++r) tma_load_3d(st + r * Cfg::A_TILE, &tmA, fb, kb * KB, m0, r);
+            for (int r = 0; r < 3; ++r) tma_load_3d(st + r * Cfg::A_TILE, &tmA, fb, (kb0 + kb) * KB, m0, r);
 #pragma unroll
-            for (int r = 0; r < 3; ++r) tma_load_3d(st + 3 * Cfg::A_TILE + r * Cfg::B_TILE, &tmB, fb, kb * KB, n0, r);
+            for (int r = 0; r < 3; ++r)
+                tma_load_3d(st + 3 * Cfg::A_TILE + r * Cfg::B_TILE, &tmB, fb, (kb0 + kb) * KB, n0, r);
             ++issued;
         }
         if (!ok) drain_inflight(full0, STAGES, issued, flags);
@@ -75,7 +118,8 @@ prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
         // ---------------- epilogue: TMEM -> registers -> C
         const bool ok = mbar_wait(accum_bar, 0, flags);
         __syncwarp();
-        if (ok) store_tile(tmem, warp & 3, 0, BN, m0, n0, M, N, C, ldc);
+        if (ok && SPLIT == 1) store_tile(tmem, warp & 3, 0, BN, m0, n0, M, N, C, ldc);
+        else if (ok && nkb > 0) reduce_tile(tmem, warp & 3, 0, BN, m0, n0, M, N, C, ldc);
     }
     tc_fence_before();
     __syncthreads();
@@ -89,8 +133,11 @@ prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
 // Per-SM rates of the narrower tiles relative to 128 x 256 (measured at 8192^3:
 // 274 and 164 against 316 TFLOP/s for the whole GEMM).
 constexpr double kRate128 = 0.87, kRate64 = 0.52;
+// Cost of splitting K in two (clearing C, adding the halves in L2) as a
+// factor on the per-SM rate.
+constexpr double kSplitCost = 0.95;
 
-template <int BN, int KB, int STAGES>
+template <int BN, int KB, int STAGES, int SPLIT = 1>
 cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
                     float *C, int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane, int64_t b_plane)
 {
@@ -99,17 +146,17 @@ cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
     if (!make_plane_map(&ta, Ap, K, M, 3, ldcomp, KB, kBM, a_plane) ||
         !make_plane_map(&tb, Bp, K, N, 3, ldcomp, KB, BN, b_plane))
         return cudaErrorInvalidValue;
-    auto kern = prodsum_f32_kernel<BN, KB, STAGES>;
+    auto kern = prodsum_f32_kernel<BN, KB, STAGES, SPLIT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
-    const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + BN - 1) / BN);
+    const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + BN - 1) / BN) * SPLIT;
     kern<<<(unsigned)tiles, Cfg::THREADS, Cfg::SMEM, st>>>(ta, tb, (int)M, (int)N, (int)K, C, ldc, flags);
     return cudaGetLastError();
 }
 
 }  // namespace
 
-// FP32 tile shape.  128 x 256 with 32-wide K-blocks (64-byte swizzle, three
+// FP32 tile plan.  128 x 256 with 32-wide K-blocks (64-byte swizzle, three
 // stages) is the fastest per SM; 128 x 128 (64-wide K-blocks, 128-byte
 // swizzle, two stages) and 128 x 64 (64-wide K-blocks, three stages) reach
 // smaller fractions of it but give more CTAs, which pays when there are too
@@ -117,9 +164,7 @@ cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
 // over the waves) x (relative per-SM rate).  Every shape issues the same MMAs
 // in the same order for each output element, so C does not depend on it.
 // EMU_F32_TILE=128x256 / 128x128 / 128x64 forces one.
-cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
-                               int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
-                               int64_t a_plane, int64_t b_plane)
+void f32_tile_plan(int64_t M, int64_t N, int64_t K, bool split_ok, int &bn, int &parts)
 {
     static const int forced = [] {
         const char *e = std::getenv("EMU_F32_TILE");
@@ -127,22 +172,48 @@ cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *
         return (e[4] == '2' && e[5] == '5' && e[6] == '6') ? 256 : (e[4] == '1' && e[5] == '2' && e[6] == '8') ? 128
                : (e[4] == '6' && e[5] == '4') ? 64 : 0;
     }();
-    int bn = forced;
-    if (bn == 0) {
-        int dev = 0, sms = 0;
-        if (cudaGetDevice(&dev) != cudaSuccess ||
-            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
-            sms = 152;
-        const int widths[3] = {256, 128, 64};
-        const double rate[3] = {1.0, kRate128, kRate64};
-        double best = -1.0;
-        for (int i = 0; i < 3; ++i) {
-            const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + widths[i] - 1) / widths[i]);
-            const int64_t waves = (tiles + sms - 1) / sms;
-            const double score = rate[i] * (double)tiles / (double)(waves * sms);
-            if (score > best * 1.02) { best = score; bn = widths[i]; }   // prefer the wider tile on near ties
-        }
+    bn = forced;
+    parts = 1;
+    if (bn != 0) return;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+        sms = 152;
+    // (width, K-parts, relative per-SM rate); the split plan needs C cleared
+    // beforehand and at least two 64-wide K-blocks per part
+    const int widths[4] = {256, 128, 64, 128}, nparts[4] = {1, 1, 1, 2};
+    const double rate[4] = {1.0, kRate128, kRate64, kRate128 * kSplitCost};
+    const int options = (split_ok && K >= 4 * 64) ? 4 : 3;
+    double best = -1.0;
+    for (int i = 0; i < options; ++i) {
+        const int64_t ctas = ((M + kBM - 1) / kBM) * ((N + widths[i] - 1) / widths[i]) * nparts[i];
+        const int64_t waves = (ctas + sms - 1) / sms;
+        const double score = rate[i] * (double)ctas / (double)(waves * sms);
+        if (score > best * 1.02) { best = score; bn = widths[i]; parts = nparts[i]; }   // earlier options win near ties
     }
+}
+
+int f32_tile_columns(int64_t M, int64_t N)
+{
+    int bn, parts;
+    f32_tile_plan(M, N, 0, false, bn, parts);
+    return bn;
+}
+
+int f32_split_parts(int64_t M, int64_t N, int64_t K)
+{
+    int bn, parts;
+    f32_tile_plan(M, N, K, true, bn, parts);
+    return parts;
+}
+
+cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
+                               int64_t ldcomp, float *C, int64_t ldc, uint32_t *flags, cudaStream_t st,
+                               int64_t a_plane, int64_t b_plane, bool c_zeroed)
+{
+    int bn, parts;
+    f32_tile_plan(M, N, K, c_zeroed, bn, parts);
+    if (parts == 2) return run_f32<128, 64, 2, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
     if (bn == 128) return run_f32<128, 64, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
     if (bn == 64) return run_f32<64, 64, 3>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
     return run_f32<256, 32, 3>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);

@@ -12,17 +12,18 @@ namespace {
 // Row-major planes: thread = 8 consecutive elements of a row (two 16-byte
 // loads, one 16-byte store per plane), no shared memory.  Rows advance by
 // the grid's y dimension.
-__global__ void __launch_bounds__(kThreads)
-split_f32_rows_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
-                      uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws)
+// Block (bx, by) of a grid with gy rows of blocks.
+__device__ __forceinline__ void split_f32_rows_body(const float *__restrict__ X, int64_t rows, int64_t cols,
+                                                    int64_t ldx, uint16_t *__restrict__ comps, int64_t ldcomp,
+                                                    int64_t plane, WsHeader *ws, int64_t bx, int64_t by, int64_t gy)
 {
     const bool vin = ((ldx & 3) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
     const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
-    const int64_t j0 = ((int64_t)blockIdx.x * kThreads + threadIdx.x) * 8;
+    const int64_t j0 = (bx * kThreads + threadIdx.x) * 8;
     uint32_t amax = 0;
     if (j0 < cols) {
         const bool full = j0 + 8 <= cols;
-        for (int64_t i = blockIdx.y; i < rows; i += gridDim.y) {
+        for (int64_t i = by; i < rows; i += gy) {
             const float *src = X + i * ldx + j0;
             float x[8];
             if (vin && full) {
@@ -54,16 +55,25 @@ split_f32_rows_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, i
     publish_f32_flags(amax, &ws->flags);
 }
 
+__global__ void __launch_bounds__(kThreads)
+split_f32_rows_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                      uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws)
+{
+    split_f32_rows_body(X, rows, cols, ldx, comps, ldcomp, plane, ws, blockIdx.x, blockIdx.y, gridDim.y);
+}
+
 // Transposed (K-major) planes: a 64 x 64 tile of X.  Warp q takes columns
 // 8q .. 8q+7, lane p rows 2p and 2p+1, so each slice word packs the two
 // elements that are adjacent in the transposed row; the words go to shared
 // memory (one bank per lane: conflict-free) and leave as 16-byte chunks of
 // whole transposed rows.
-__global__ void __launch_bounds__(kThreads)
-split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
-                           uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws)
+// Block bid of nblk blocks (tiles taken with a stride of nblk); sm: the
+// block's [3][kTile][kTile / 2] staging words.
+__device__ __forceinline__ void split_f32_transpose_body(const float *__restrict__ X, int64_t rows, int64_t cols,
+                                                         int64_t ldx, uint16_t *__restrict__ comps, int64_t ldcomp,
+                                                         int64_t plane, WsHeader *ws, int64_t bid, int64_t nblk,
+                                                         uint32_t (*sm)[kTile][kTile / 2])
 {
-    __shared__ __align__(16) uint32_t sm[3][kTile][kTile / 2];   // [plane][transposed row][word]
     const bool vin = ((ldx & 3) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
     const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
     const int q = threadIdx.x >> 5, p = lane_id();
@@ -88,11 +98,11 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
     };
     uint32_t amax = 0;
     float x[2][8];
-    if ((int64_t)blockIdx.x < tiles_r * tiles_c) load_tile(blockIdx.x, x);
-    for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
+    if (bid < tiles_r * tiles_c) load_tile(bid, x);
+    for (int64_t t = bid; t < tiles_r * tiles_c; t += nblk) {
         const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
         float xn[2][8];
-        if (t + gridDim.x < tiles_r * tiles_c) load_tile(t + gridDim.x, xn);
+        if (t + nblk < tiles_r * tiles_c) load_tile(t + nblk, xn);
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
             amax = abs_bits_max(amax, x[0][e], x[1][e]);
@@ -131,6 +141,38 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
     publish_f32_flags(amax, &ws->flags);
 }
 
+__global__ void __launch_bounds__(kThreads)
+split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                           uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws)
+{
+    __shared__ __align__(16) uint32_t sm[3][kTile][kTile / 2];   // [plane][transposed row][word]
+    split_f32_transpose_body(X, rows, cols, ldx, comps, ldcomp, plane, ws, blockIdx.x, gridDim.x, sm);
+}
+
+// Both operands of an FP32 GEMM in one launch: blocks [0, nA) split A into
+// row-major planes (nA = ax * ay blocks as the row kernel's grid), blocks
+// [nA, nA + nB) split B into K-major planes, and blocks from nA + nB on set
+// the M x N result C to zero (a product-sum that adds its K-parts into C
+// needs it cleared).
+__global__ void __launch_bounds__(kThreads)
+split_f32_gemm_kernel(const float *__restrict__ A, int64_t M, int64_t K, int64_t lda, const float *__restrict__ B,
+                      int64_t N, int64_t ldb, uint16_t *__restrict__ Ap, uint16_t *__restrict__ Bp, int64_t ldcomp,
+                      WsHeader *ws, int64_t ax, int64_t ay, int64_t nB, float *__restrict__ C, int64_t ldc,
+                      int64_t nC)
+{
+    __shared__ __align__(16) uint32_t sm[3][kTile][kTile / 2];
+    const int64_t b = blockIdx.x, nA = ax * ay;
+    if (b < nA) {
+        split_f32_rows_body(A, M, K, lda, Ap, ldcomp, M * ldcomp, ws, b % ax, b / ax, ay);
+    } else if (b < nA + nB) {
+        split_f32_transpose_body(B, K, N, ldb, Bp, ldcomp, N * ldcomp, ws, b - nA, nB, sm);
+    } else {
+        const int64_t c = b - nA - nB;
+        for (int64_t i = c; i < M; i += nC)
+            for (int64_t j = threadIdx.x; j < N; j += kThreads) C[i * ldc + j] = 0.0f;
+    }
+}
+
 }  // namespace
 
 // ----------------------------------------------------------- host launchers
@@ -149,6 +191,25 @@ cudaError_t launch_split_f32(const float *X, int64_t rows, int64_t cols, int64_t
         split_f32_rows_kernel<<<dim3((unsigned)bx, (unsigned)by), kThreads, 0, st>>>(X, rows, cols, ldx, comps, ldcomp,
                                                                                      plane, ws);
     }
+    return cudaGetLastError();
+}
+
+// Both operands of an FP32 GEMM (A: M x K, B: K x N) into planes of row
+// pitch ldcomp laid out as the GEMM workspace holds them, in one launch; with
+// C non-null also C <- 0.
+cudaError_t launch_split_f32_gemm(const float *A, int64_t M, int64_t K, int64_t lda, const float *B, int64_t N,
+                                  int64_t ldb, uint16_t *Ap, uint16_t *Bp, int64_t ldcomp, WsHeader *ws, float *C,
+                                  int64_t ldc, cudaStream_t st)
+{
+    if (M == 0 || N == 0 || K == 0) return cudaSuccess;
+    const int64_t ax = (K + 8 * kThreads - 1) / (8 * kThreads);
+    const int64_t want = (152 * 4 + ax - 1) / ax;
+    const int64_t ay = M < want ? M : want;
+    const int64_t tiles = ((K + kTile - 1) / kTile) * ((N + kTile - 1) / kTile);
+    const int64_t nB = grid_for(tiles, 152 * 4);
+    const int64_t nC = C ? (M < 152 ? M : 152) : 0;
+    split_f32_gemm_kernel<<<(unsigned)(ax * ay + nB + nC), kThreads, 0, st>>>(A, M, K, lda, B, N, ldb, Ap, Bp, ldcomp,
+                                                                              ws, ax, ay, nB, C, ldc, nC);
     return cudaGetLastError();
 }
 

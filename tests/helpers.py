@@ -57,3 +57,17 @@ def sample_rows(M, count, seed):
     rng = np.random.default_rng(seed)
     rows = sorted(set(int(r) for r in rng.integers(0, M, size=count)) | {0, M - 1})
     return rows
+
+
+def gemm_f32_one_accumulator(A_d, B_d):
+    """FP32 mode as split + product-sum through the separate C-ABI calls: all
+    of K in one FP32 accumulator per tile.  emu_gemm_f32 itself may split K
+    in two for small results, which changes FP32 rounding; the kernels that
+    must match the one-accumulator sum bit for bit are compared with this.
+    Returns (C, the splits' flag words or-ed)."""
+    M, K = A_d.shape
+    N = B_d.shape[1]
+    Ap, wa = emu.split_f32(A_d, ldcomp=emu.gemm_ldk(K))
+    Bp, wb = emu.split_f32(B_d, transpose=True, ldcomp=emu.gemm_ldk(K))
+    C, _ = emu.prodsum_f32(Ap, Bp, M, N, K)
+    return C, emu.read_flags(wa) | emu.read_flags(wb)

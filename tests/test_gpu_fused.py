@@ -3,7 +3,8 @@ on the GPU, through the C-ABI.
 
 It forms the same slices (Eq. (fp32split)) and issues the same MMAs in the
 same order into the same accumulator as the split + product-sum pair, so C
-must equal emu_gemm_f32 bit for bit, and the oracle within the FP32-mode bar
+must equal split + product-sum bit for bit (all of K in one accumulator;
+emu_gemm_f32 may split K for small results), and the oracle within the FP32-mode bar
 |C - C_oracle| <= 1e-5 (|A||B|).  Its loads take several paths (16-byte
 vectors, scalars for ragged or unaligned rows, zeros past the edges), so the
 cases cover each of them.
@@ -14,7 +15,7 @@ import pytest
 import oracle
 import synth
 import paper_2609_04663_gb300 as emu
-from helpers import device, fp32_within_tolerance, random_finite_f32, sample_rows, to_dev
+from helpers import device, fp32_within_tolerance, gemm_f32_one_accumulator, random_finite_f32, sample_rows, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -25,9 +26,9 @@ def dev():
 
 
 def _both(A_d, B_d):
-    C2, ws2 = emu.gemm_f32(A_d, B_d)
+    C2, f2 = gemm_f32_one_accumulator(A_d, B_d)
     C1, ws1 = emu.gemm_f32_fused(A_d, B_d)
-    return C1, emu.read_flags(ws1), C2, emu.read_flags(ws2)
+    return C1, emu.read_flags(ws1), C2, f2
 
 
 @pytest.mark.parametrize("M,N,K,seed", [
@@ -66,7 +67,7 @@ def test_fused_strided_and_unaligned(dev, pad_a, pad_b, offset_a):
     C = Cbig[:, :N]
     _, ws = emu.gemm_f32_fused(Ad, Bd, C=C)
     assert emu.read_flags(ws) == 0
-    C2, _ = emu.gemm_f32(to_dev(A, dev), to_dev(B, dev))
+    C2, _ = gemm_f32_one_accumulator(to_dev(A, dev), to_dev(B, dev))
     assert np.array_equal(C.cpu().numpy().view(np.uint32), C2.cpu().numpy().view(np.uint32))
     assert not Cbig[:, N:].any()
 
@@ -121,7 +122,7 @@ def test_fused_fullsize_fp32_n16384_sampled(dev):
     Ad, Bd = to_dev(A, dev), to_dev(B, dev)
     C1, ws = emu.gemm_f32_fused(Ad, Bd)
     assert emu.read_flags(ws) == 0
-    C2, _ = emu.gemm_f32(Ad, Bd)
+    C2, _ = gemm_f32_one_accumulator(Ad, Bd)
     assert bool((C1.view(emu._torch().int32) == C2.view(emu._torch().int32)).all())
     del C2
     rows = sample_rows(n, 3, 1)

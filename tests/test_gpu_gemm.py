@@ -371,3 +371,23 @@ def test_fullsize_large_k_sampled(dev):
         Co = oracle.prodsum_f64(Ap[:, rows], Bp, nprod)
         assert np.array_equal(Cg, Co), nprod
         del C, ws
+
+
+@pytest.mark.parametrize("M,N,K,seed", [(1024, 1024, 1024, 41), (300, 333, 700, 42), (256, 1000, 4096, 43),
+                                        (129, 64, 256, 44)])
+def test_gemm_f32_k_split_small_results(M, N, K, seed):
+    """Small results: emu_gemm_f32 splits K in two and adds the halves into C
+    in L2.  Within the FP32-mode bar of the oracle, and the same bits on a
+    second run (two addends: the order of arrival does not matter)."""
+    dev = device()
+    A, B = synth.gemm_inputs("f32", M, N, K, seed)
+    Ad, Bd = to_dev(A, dev), to_dev(B, dev)
+    C1, ws = emu.gemm_f32(Ad, Bd)
+    assert emu.read_flags(ws) == 0
+    C2, _ = emu.gemm_f32(Ad, Bd)
+    C1n = C1.cpu().numpy()
+    assert np.array_equal(C1n.view(np.uint32), C2.cpu().numpy().view(np.uint32))
+    rows = sample_rows(M, 6, seed) if M * N * K > 400 * 400 * 1000 else list(range(M))
+    Co = oracle.prodsum_f32(oracle.split_f32(A[rows])[0], oracle.split_f32(B)[0])
+    ok, worst = fp32_within_tolerance(C1n[rows], Co, A[rows], B)
+    assert ok, worst

@@ -11,7 +11,7 @@ import pytest
 import oracle
 import synth
 import paper_2609_04663_gb300 as emu
-from helpers import device, fp32_within_tolerance, to_dev
+from helpers import device, fp32_within_tolerance, gemm_f32_one_accumulator, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -52,7 +52,7 @@ def test_gemm_f32_host_equals_device_path(dev, M, N, K, seed):
     A, B = synth.gemm_inputs("f32", M, N, K, seed)
     Ch, flags = run_host(A, B, pads=(3, 5, 7))
     assert flags == 0
-    Cd, _ = emu.gemm_f32(to_dev(A, dev), to_dev(B, dev))
+    Cd, _ = gemm_f32_one_accumulator(to_dev(A, dev), to_dev(B, dev))
     np.testing.assert_array_equal(Ch.view(np.uint32), Cd.cpu().numpy().view(np.uint32))
     if M * N * K <= 300 * 200 * 700:
         Co, _ = oracle.gemm_f32(A, B)
@@ -79,7 +79,7 @@ def test_gemm_f64_host_equals_oracle(dev, M, N, K, nprod, seed):
 def test_host_pageable_buffers(dev):
     A, B = synth.gemm_inputs("f32", 200, 100, 300, 41)
     Ch, flags = run_host(A, B, pinned=False)
-    Cd, _ = emu.gemm_f32(to_dev(A, dev), to_dev(B, dev))
+    Cd, _ = gemm_f32_one_accumulator(to_dev(A, dev), to_dev(B, dev))
     np.testing.assert_array_equal(Ch.view(np.uint32), Cd.cpu().numpy().view(np.uint32))
 
 
@@ -112,5 +112,5 @@ def test_host_repeated_calls_and_interleaving(dev):
         outs.append((A, B, Ah, Bh, C, ws))
     torch.cuda.synchronize()
     for A, B, _, _, C, _ in outs:
-        Cd, _ = emu.gemm_f32(to_dev(A, dev), to_dev(B, dev))
+        Cd, _ = gemm_f32_one_accumulator(to_dev(A, dev), to_dev(B, dev))
         np.testing.assert_array_equal(C.numpy().view(np.uint32), Cd.cpu().numpy().view(np.uint32))
