@@ -94,6 +94,9 @@ prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // set-up above overlaps the end of the kernel that wrote the planes (and
+    // cleared C) when this one is launched as its programmatic dependent
+    griddep_wait();
 
     if (warp == 0 && lane == 0) {
         // ---------------- TMA producer
@@ -150,7 +153,21 @@ cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
     const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + BN - 1) / BN) * SPLIT;
-    kern<<<(unsigned)tiles, Cfg::THREADS, Cfg::SMEM, st>>>(ta, tb, (int)M, (int)N, (int)K, C, ldc, flags);
+    // launched as a programmatic dependent of the previous kernel in the
+    // stream: its set-up overlaps that kernel's tail (griddep_wait orders the
+    // rest after it)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)tiles);
+    cfg.blockDim = dim3(Cfg::THREADS);
+    cfg.dynamicSmemBytes = Cfg::SMEM;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, kern, ta, tb, (int)M, (int)N, (int)K, C, ldc, flags);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

@@ -12,8 +12,9 @@ namespace {
 // Row-major planes: thread = 8 consecutive elements of a row (two 16-byte
 // loads, one 16-byte store per plane), no shared memory.  Rows advance by
 // the grid's y dimension.
-// Block (bx, by) of a grid with gy rows of blocks.
-__device__ __forceinline__ void split_f32_rows_body(const float *__restrict__ X, int64_t rows, int64_t cols,
+// Block (bx, by) of a grid with gy rows of blocks; returns the block's part of
+// the flag check (the largest |x| bit pattern seen), for publish_f32_flags.
+__device__ __forceinline__ uint32_t split_f32_rows_body(const float *__restrict__ X, int64_t rows, int64_t cols,
                                                     int64_t ldx, uint16_t *__restrict__ comps, int64_t ldcomp,
                                                     int64_t plane, WsHeader *ws, int64_t bx, int64_t by, int64_t gy)
 {
@@ -52,14 +53,15 @@ __device__ __forceinline__ void split_f32_rows_body(const float *__restrict__ X,
             }
         }
     }
-    publish_f32_flags(amax, &ws->flags);
+    return amax;
 }
 
 __global__ void __launch_bounds__(kThreads)
 split_f32_rows_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
                       uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws)
 {
-    split_f32_rows_body(X, rows, cols, ldx, comps, ldcomp, plane, ws, blockIdx.x, blockIdx.y, gridDim.y);
+    publish_f32_flags(split_f32_rows_body(X, rows, cols, ldx, comps, ldcomp, plane, ws, blockIdx.x, blockIdx.y,
+                                          gridDim.y), &ws->flags);
 }
 
 // Transposed (K-major) planes: a 64 x 64 tile of X.  Warp q takes columns
@@ -68,8 +70,9 @@ split_f32_rows_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, i
 // memory (one bank per lane: conflict-free) and leave as 16-byte chunks of
 // whole transposed rows.
 // Block bid of nblk blocks (tiles taken with a stride of nblk); sm: the
-// block's [3][kTile][kTile / 2] staging words.
-__device__ __forceinline__ void split_f32_transpose_body(const float *__restrict__ X, int64_t rows, int64_t cols,
+// block's [3][kTile][kTile / 2] staging words.  Returns the block's part of
+// the flag check, as the row body does.
+__device__ __forceinline__ uint32_t split_f32_transpose_body(const float *__restrict__ X, int64_t rows, int64_t cols,
                                                          int64_t ldx, uint16_t *__restrict__ comps, int64_t ldcomp,
                                                          int64_t plane, WsHeader *ws, int64_t bid, int64_t nblk,
                                                          uint32_t (*sm)[kTile][kTile / 2])
@@ -138,7 +141,7 @@ __device__ __forceinline__ void split_f32_transpose_body(const float *__restrict
 #pragma unroll
             for (int e = 0; e < 8; ++e) x[h][e] = xn[h][e];
     }
-    publish_f32_flags(amax, &ws->flags);
+    return amax;
 }
 
 __global__ void __launch_bounds__(kThreads)
@@ -146,7 +149,8 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
                            uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws)
 {
     __shared__ __align__(16) uint32_t sm[3][kTile][kTile / 2];   // [plane][transposed row][word]
-    split_f32_transpose_body(X, rows, cols, ldx, comps, ldcomp, plane, ws, blockIdx.x, gridDim.x, sm);
+    publish_f32_flags(split_f32_transpose_body(X, rows, cols, ldx, comps, ldcomp, plane, ws, blockIdx.x, gridDim.x, sm),
+                      &ws->flags);
 }
 
 // Both operands of an FP32 GEMM in one launch: blocks [0, nA) split A into
@@ -162,10 +166,13 @@ split_f32_gemm_kernel(const float *__restrict__ A, int64_t M, int64_t K, int64_t
 {
     __shared__ __align__(16) uint32_t sm[3][kTile][kTile / 2];
     const int64_t b = blockIdx.x, nA = ax * ay;
-    if (b < nA) {
-        split_f32_rows_body(A, M, K, lda, Ap, ldcomp, M * ldcomp, ws, b % ax, b / ax, ay);
-    } else if (b < nA + nB) {
-        split_f32_transpose_body(B, K, N, ldb, Bp, ldcomp, N * ldcomp, ws, b - nA, nB, sm);
+    if (b < nA + nB) {
+        const uint32_t amax = b < nA ? split_f32_rows_body(A, M, K, lda, Ap, ldcomp, M * ldcomp, ws, b % ax, b / ax, ay)
+                                     : split_f32_transpose_body(B, K, N, ldb, Bp, ldcomp, N * ldcomp, ws, b - nA, nB, sm);
+        // the flag word is cleared by the operation before this launch, which
+        // may still be running when this kernel is its programmatic dependent
+        griddep_wait();
+        publish_f32_flags(amax, &ws->flags);
     } else {
         const int64_t c = b - nA - nB;
         for (int64_t i = c; i < M; i += nC)
@@ -208,8 +215,20 @@ cudaError_t launch_split_f32_gemm(const float *A, int64_t M, int64_t K, int64_t 
     const int64_t tiles = ((K + kTile - 1) / kTile) * ((N + kTile - 1) / kTile);
     const int64_t nB = grid_for(tiles, 152 * 4);
     const int64_t nC = C ? (M < 152 ? M : 152) : 0;
-    split_f32_gemm_kernel<<<(unsigned)(ax * ay + nB + nC), kThreads, 0, st>>>(A, M, K, lda, B, N, ldb, Ap, Bp, ldcomp,
-                                                                              ws, ax, ay, nB, C, ldc, nC);
+    // a programmatic dependent of the clearing of the workspace header, which
+    // only its flag publication waits for
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(ax * ay + nB + nC));
+    cfg.blockDim = dim3(kThreads);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, split_f32_gemm_kernel, A, M, K, lda, B, N, ldb, Ap, Bp, ldcomp, ws,
+                                             ax, ay, nB, C, ldc, nC);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
