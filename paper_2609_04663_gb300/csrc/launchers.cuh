@@ -89,11 +89,12 @@ cudaError_t launch_prodsum_tail(int64_t M, int64_t N, int64_t K, const uint16_t 
 // Tile width (128 or 256) the FP64 product-sum picks for an M x N result.
 int f64_tile_columns(int64_t M, int64_t N);
 // The FP64 product-sum on 128 x 256 tiles (prodsum_f64w.cu); launch_prodsum_f64
-// calls it when that tile shape is chosen.  acc: f64_acc_bytes(M, N) bytes.
+// calls it when that tile shape is chosen, for the first ctas tiles in raster
+// order.  acc: f64_acc_bytes(M, N) bytes.
 cudaError_t launch_prodsum_f64_wide(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                     int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
                                     int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
-                                    bool rowcol, const float *T, int64_t ldt);
+                                    bool rowcol, const float *T, int64_t ldt, int64_t ctas);
 
 // Bytes of the FP64 product-sum's accumulator, enough for either tile shape:
 // one FP64 tile of 128 x 128 (narrow kernel) or 128 x 256 (wide kernel) per

@@ -84,7 +84,7 @@ __global__ void __launch_bounds__(F64Cfg::THREADS, 1)
 prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    int M, int N, int K, const int32_t *__restrict__ vA, const int32_t *__restrict__ vB,
                    double *__restrict__ C, int64_t ldc, double *__restrict__ acc, uint32_t *flags,
-                   const float *__restrict__ T, int64_t ldt)
+                   const float *__restrict__ T, int64_t ldt, int wide_first)
 {
     using Cfg = F64Cfg;
     extern __shared__ uint8_t smem_raw[];
@@ -100,7 +100,16 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     const int warp = threadIdx.x >> 5, lane = lane_id();
     const int tiles_m = (M + kBM - 1) / kBM, tiles_n = (N + Cfg::BN - 1) / Cfg::BN;
     int tm, tn;
-    tile_coords(blockIdx.x, tiles_m, tiles_n, tm, tn);
+    if (wide_first < 0) {
+        tile_coords(blockIdx.x, tiles_m, tiles_n, tm, tn);
+    } else {
+        // the two 128-column halves of the 128 x 256 tiles from raster index
+        // wide_first on, which the wide kernel's last, partial wave would have taken
+        int tnw;
+        tile_coords(wide_first + (int)(blockIdx.x >> 1), tiles_m, (N + 255) / 256, tm, tnw);
+        tn = 2 * tnw + (int)(blockIdx.x & 1);
+        if (tn >= tiles_n) return;                    // a half past the last column
+    }
     const int m0 = tm * kBM, n0 = tn * Cfg::BN;
     const int nch = (K + kKChunk - 1) / kKChunk;
 
@@ -398,7 +407,7 @@ constexpr double kF64RateNarrow = 0.76;
 template <int NPROD, bool ROWCOL, bool TAIL = false>
 cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
                     const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, double *acc, uint32_t *flags,
-                    cudaStream_t st, int64_t a_plane, const float *T, int64_t ldt)
+                    cudaStream_t st, int64_t a_plane, const float *T, int64_t ldt, int wide_first, int64_t ctas)
 {
     using Cfg = F64Cfg;
     CUtensorMap ta, tb;
@@ -407,9 +416,9 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
     auto kern = prodsum_f64_kernel<NPROD, ROWCOL, TAIL>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
-    const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + Cfg::BN - 1) / Cfg::BN);
+    const int64_t tiles = wide_first < 0 ? ((M + kBM - 1) / kBM) * ((N + Cfg::BN - 1) / Cfg::BN) : ctas;
     kern<<<(unsigned)tiles, Cfg::THREADS, Cfg::SMEM, st>>>(ta, tb, (int)M, (int)N, (int)K, vA, vB, C, ldc, acc, flags,
-                                                           T, ldt);
+                                                           T, ldt, wide_first);
     return cudaGetLastError();
 }
 
@@ -418,26 +427,26 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
 static cudaError_t launch_prodsum_f64_narrow(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
                                int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
-                               bool rowcol, const float *T, int64_t ldt)
+                               bool rowcol, const float *T, int64_t ldt, int wide_first = -1, int64_t ctas = 0)
 {
     if (T) {                                          // merged tail: whole-matrix levels only
         if (rowcol) return cudaErrorInvalidValue;
         switch (nprod) {
-        case 6: return run_f64<6, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
-        case 10: return run_f64<10, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
-        case 15: return run_f64<15, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
+        case 6: return run_f64<6, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, wide_first, ctas);
+        case 10: return run_f64<10, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, wide_first, ctas);
+        case 15: return run_f64<15, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, wide_first, ctas);
         default: return cudaErrorInvalidValue;
         }
     }
     switch (nprod) {
-    case 6: return rowcol ? run_f64<6, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0)
-                   : run_f64<6, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
-    case 10: return rowcol ? run_f64<10, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0)
-                   : run_f64<10, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
-    case 15: return rowcol ? run_f64<15, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0)
-                   : run_f64<15, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
-    case 21: return rowcol ? run_f64<21, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0)
-                   : run_f64<21, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
+    case 6: return rowcol ? run_f64<6, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas)
+                   : run_f64<6, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas);
+    case 10: return rowcol ? run_f64<10, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas)
+                   : run_f64<10, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas);
+    case 15: return rowcol ? run_f64<15, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas)
+                   : run_f64<15, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas);
+    case 21: return rowcol ? run_f64<21, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas)
+                   : run_f64<21, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas);
     default: return cudaErrorInvalidValue;
     }
 }
@@ -448,14 +457,20 @@ static cudaError_t launch_prodsum_f64_narrow(int64_t M, int64_t N, int64_t K, co
 // x (relative per-SM rate), as for the FP32 product-sum.  Both shapes form
 // the same exact per-product sums and fold them in the same order, so C does
 // not depend on the choice.  EMU_F64_TILE=128x128 / 128x256 forces one.
-int f64_tile_columns(int64_t M, int64_t N)
+// EMU_F64_TILE=128x128 / 128x256: one tile width for every result (0: unset).
+static int f64_tile_forced()
 {
     static const int forced = [] {
         const char *e = std::getenv("EMU_F64_TILE");
         if (!e || std::strncmp(e, "128x", 4) != 0) return 0;
         return std::strcmp(e + 4, "256") == 0 ? 256 : std::strcmp(e + 4, "128") == 0 ? 128 : 0;
     }();
-    int bn = forced;
+    return forced;
+}
+
+int f64_tile_columns(int64_t M, int64_t N)
+{
+    int bn = f64_tile_forced();
     if (bn == 0) {
         int dev = 0, sms = 0;
         if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -479,9 +494,31 @@ cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *
                                int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
                                bool rowcol, const float *T, int64_t ldt)
 {
-    if (f64_tile_columns(M, N) == 256)
+    if (f64_tile_columns(M, N) == 256) {
+        // When the 128 x 256 tiles leave the last wave partly empty, the wide
+        // kernel takes the full waves and the narrow kernel, launched after it,
+        // the remaining tiles as twice as many 128 x 128 halves, if that is
+        // estimated faster (a half takes 0.5 / kF64RateNarrow of a wide tile's
+        // time).  The two kernels run one after the other, so the accumulator
+        // tiles they index differently never overlap in time.
+        int dev = 0, sms = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+            sms = 152;
+        const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + 255) / 256);
+        const int64_t full = (tiles / sms) * sms, rem = tiles - full;
+        const double t_wide = (double)((tiles + sms - 1) / sms);
+        const double t_mixed = (double)(full / sms) + (0.5 / kF64RateNarrow) * (double)((2 * rem + sms - 1) / sms);
+        if (!f64_tile_forced() && full > 0 && rem > 0 && t_mixed < 0.97 * t_wide) {
+            cudaError_t e = launch_prodsum_f64_wide(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st,
+                                                    a_plane, rowcol, T, ldt, full);
+            if (e != cudaSuccess) return e;
+            return launch_prodsum_f64_narrow(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane,
+                                             rowcol, T, ldt, (int)full, 2 * rem);
+        }
         return launch_prodsum_f64_wide(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane,
-                                       rowcol, T, ldt);
+                                       rowcol, T, ldt, tiles);
+    }
     return launch_prodsum_f64_narrow(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane,
                                      rowcol, T, ldt);
 }

@@ -343,10 +343,12 @@ prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     }
 }
 
+// ctas: the first ctas tiles in raster order (all of them, or the full waves
+// when the narrow kernel takes the rest).
 template <int NPROD, bool ROWCOL, bool TAIL>
 cudaError_t run_f64w(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
                      const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, double *acc, uint32_t *flags,
-                     cudaStream_t st, int64_t a_plane, const float *T, int64_t ldt)
+                     cudaStream_t st, int64_t a_plane, const float *T, int64_t ldt, int64_t ctas)
 {
     using Cfg = F64WCfg;
     CUtensorMap ta, tb;
@@ -356,7 +358,7 @@ cudaError_t run_f64w(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const 
     auto kern = prodsum_f64w_kernel<NPROD, ROWCOL, TAIL>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
-    const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + Cfg::BN - 1) / Cfg::BN);
+    const int64_t tiles = ctas;
     kern<<<(unsigned)tiles, Cfg::THREADS, Cfg::SMEM, st>>>(ta, tb, (int)M, (int)N, (int)K, vA, vB, C, ldc, acc, flags,
                                                            T, ldt);
     return cudaGetLastError();
@@ -367,26 +369,26 @@ cudaError_t run_f64w(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const 
 cudaError_t launch_prodsum_f64_wide(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                     int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
                                     int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
-                                    bool rowcol, const float *T, int64_t ldt)
+                                    bool rowcol, const float *T, int64_t ldt, int64_t ctas)
 {
     if (T) {                                          // merged tail: whole-matrix levels only
         if (rowcol) return cudaErrorInvalidValue;
         switch (nprod) {
-        case 6: return run_f64w<6, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
-        case 10: return run_f64w<10, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
-        case 15: return run_f64w<15, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt);
+        case 6: return run_f64w<6, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, ctas);
+        case 10: return run_f64w<10, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, ctas);
+        case 15: return run_f64w<15, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, ctas);
         default: return cudaErrorInvalidValue;
         }
     }
     switch (nprod) {
-    case 6: return rowcol ? run_f64w<6, true, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0)
-                   : run_f64w<6, false, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
-    case 10: return rowcol ? run_f64w<10, true, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0)
-                   : run_f64w<10, false, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
-    case 15: return rowcol ? run_f64w<15, true, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0)
-                   : run_f64w<15, false, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
-    case 21: return rowcol ? run_f64w<21, true, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0)
-                   : run_f64w<21, false, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0);
+    case 6: return rowcol ? run_f64w<6, true, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas)
+                   : run_f64w<6, false, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas);
+    case 10: return rowcol ? run_f64w<10, true, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas)
+                   : run_f64w<10, false, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas);
+    case 15: return rowcol ? run_f64w<15, true, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas)
+                   : run_f64w<15, false, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas);
+    case 21: return rowcol ? run_f64w<21, true, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas)
+                   : run_f64w<21, false, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas);
     default: return cudaErrorInvalidValue;
     }
 }

@@ -73,6 +73,15 @@ for M, N, K, seed, nprod in [(300, 333, 700, 1, 21), (129, 257, 33, 3, 6), (256,
     Cn = C.cpu().numpy()
     assert np.array_equal(Cn, oracle.gemm_f64(A, B, nprod)[0]), (M, N, K, nprod)
     digest((M, N, K, nprod), Cn)
+# a 4096 x 4096 result: 3.4 waves of 128 x 256 tiles, so by default the full
+# waves run wide and the last tiles as 128 x 128 halves
+A, B = synth.gemm_inputs("f64", 4096, 4096, 264, 14)
+C, ws = emu.gemm_f64(to_dev(A, dev), to_dev(B, dev), 10)
+assert emu.read_flags(ws) == 0
+Cn = C.cpu().numpy()
+for r in (0, 1234, 3000, 4095):
+    assert np.array_equal(Cn[r], oracle.gemm_f64(A, B, 10, rows=(r, r + 1))[0][0]), r
+digest("mixed", Cn)
 # positive entries: every running sum passes 2^24 units, so the carries into the low words run
 A, B = synth.gemm_inputs("f64", 200, 300, 8192, 11)
 A, B = np.abs(A), np.abs(B)
@@ -112,9 +121,11 @@ def _run64(tile):
 def test_f64_tile_shapes_parity_and_bit_identity():
     """The FP64 product-sum's tile shapes (EMU_F64_TILE=128x128 / 128x256):
     both form the same exact per-product sums and add them in Algorithm 2's
-    order, so C must equal the oracle bit for bit with either shape, through
-    the plain, carry, per-row/column and merged-tail paths."""
+    order, so C must equal the oracle bit for bit with either shape, and with
+    the default schedule that runs the last partial wave of wide tiles as
+    narrow ones, through the plain, carry, per-row/column and merged-tail
+    paths."""
     ref = _run64(None)
-    assert len(ref) == 7
+    assert len(ref) == 8
     for tile in ("128x256", "128x128"):
         assert _run64(tile) == ref, tile
