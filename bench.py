@@ -229,8 +229,19 @@ class Case:
             "prodsum_f64w" if emu.emu_prodsum_f64_tile_columns(M, N) == 256 else "prodsum_f64"
         self.flop = 2.0 * M * N * K
         self.exec_flop = self.flop * (6 if self.mode == 32 else self.nprod)
-        # kernels of ours per step: FP32 split = 1 launch, FP64 split = 10, product-sum = 1
-        self.launches = 1 if self.fused else (2 * 1 + 1) if self.mode == 32 else (2 * 10 + 1)
+        # kernels of ours per step: FP32 split of both operands = 1 launch; FP64 split of both =
+        # 5 (level maxima of both, then a speculative pass and a verifier per operand);
+        # product-sum = 1 (FP64 with its last partial wave on 128 x 128 tiles: 2)
+        self.launches = 1 if self.fused else 2 if self.mode == 32 else 5 + 1
+        if self.kernel == "prodsum_f64w":
+            # the library's schedule: full waves of 128 x 256 tiles, the rest as 128 x 128
+            # halves in a second launch when that is estimated at least 3 % faster
+            sms = torch.cuda.get_device_properties(0).multi_processor_count
+            tiles = ((M + 127) // 128) * ((N + 255) // 256)
+            full, rem = (tiles // sms) * sms, tiles % sms
+            t_wide, t_mixed = -(-tiles // sms), full // sms + (0.5 / 0.76) * -(-2 * rem // sms)
+            if full > 0 and rem > 0 and t_mixed < 0.97 * t_wide:
+                self.launches += 1
         if self.merge_from is not None:
             self.launches += 1                    # the tail kernel
         if self.api and self.mode == 32:
@@ -243,17 +254,14 @@ class Case:
         if self.fused or self.merge_from is not None or self.api:
             return                                # the whole GEMM runs in prodsum()
         if self.mode == 32:
-            r = emu.emu_split_f32(self.A.data_ptr(), self.M, self.K, self.A.stride(0), 0, self.Ap.data_ptr(),
-                                  self.ldk, ws, n, st)
-            r |= emu.emu_split_f32(self.B.data_ptr(), self.K, self.N, self.B.stride(0), 1, self.Bp.data_ptr(),
-                                   self.ldk, ws, n, st)
+            r = emu.emu_split_f32_pair(self.M, self.N, self.K, self.A.data_ptr(), self.A.stride(0), self.B.data_ptr(),
+                                       self.B.stride(0), self.Ap.data_ptr(), self.Bp.data_ptr(), self.ldk, ws, n, st)
         else:
             # only the d slices the product-sum reads (d = 3, 4, 5, 6 for nprod = 6, 10, 15, 21)
             d = {6: 3, 10: 4, 15: 5, 21: 6}[self.nprod]
-            r = emu.emu_split_f64_slices(self.A.data_ptr(), self.M, self.K, self.A.stride(0), 0, self.Ap.data_ptr(),
-                                         self.ldk, d, self.v.data_ptr(), ws, n, st)
-            r |= emu.emu_split_f64_slices(self.B.data_ptr(), self.K, self.N, self.B.stride(0), 1, self.Bp.data_ptr(),
-                                          self.ldk, d, self.v.data_ptr() + 24, ws, n, st)
+            r = emu.emu_split_f64_pair(self.M, self.N, self.K, self.A.data_ptr(), self.A.stride(0), self.B.data_ptr(),
+                                       self.B.stride(0), self.Ap.data_ptr(), self.Bp.data_ptr(), self.ldk, d,
+                                       self.v.data_ptr(), self.v.data_ptr() + 24, ws, n, st)
         assert r == 0, r
 
     def prodsum(self, stream):

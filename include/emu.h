@@ -156,6 +156,23 @@ emu_status emu_split_f64_slices(const double *X, int64_t rows, int64_t cols, int
  * larger). */
 size_t emu_gemm_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K);
 
+/* The split step of a GEMM C = A . B as one call: A (M x K, lda) into
+ * row-major planes Acomps [s][M][ldcomp] and B (K x N, ldb) into K-major
+ * planes Bcomps [s][N][ldcomp] (ldcomp >= K), exactly as emu_split_f32 /
+ * emu_split_f64_slices split each operand (planes and levels identical), in
+ * fewer launches, as the GEMM entry points run it (FP32: one launch for
+ * both; FP64: the level-0 maxima of both in one launch).  FP64: nslices in 3..6 as for emu_split_f64_slices; vA, vB:
+ * device int32[6] receiving the level exponents of A and of B.  ws: at least
+ * emu_split_workspace_bytes(mode); one flag word covers both operands.
+ * Errors as the single-operand splits. */
+emu_status emu_split_f32_pair(int64_t M, int64_t N, int64_t K, const float *A, int64_t lda,
+                              const float *B, int64_t ldb, uint16_t *Acomps, uint16_t *Bcomps,
+                              int64_t ldcomp, void *ws, size_t ws_bytes, emu_stream_t stream);
+emu_status emu_split_f64_pair(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda,
+                              const double *B, int64_t ldb, uint16_t *Acomps, uint16_t *Bcomps,
+                              int64_t ldcomp, int nslices, int32_t *vA, int32_t *vB, void *ws,
+                              size_t ws_bytes, emu_stream_t stream);
+
 /* FP32-mode emulated GEMM, Algorithm 1: C (M x N, ldc) = A (M x K, lda) . B
  * (K x N, ldb), all FP32 row-major.  Splits A and B into the workspace, then
  * runs the tensor-core product-sum: the 6 products of Eq. (fp32six) are

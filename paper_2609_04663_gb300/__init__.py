@@ -33,6 +33,8 @@ _SIGS = {
     "emu_split_f64": ("i", ["p", "l", "l", "l", "i", "p", "l", "p", "p", "size", "p"]),
     "emu_split_f64_slices": ("i", ["p", "l", "l", "l", "i", "p", "l", "i", "p", "p", "size", "p"]),
     "emu_gemm_workspace_bytes": ("size", ["i", "l", "l", "l"]),
+    "emu_split_f32_pair": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "p", "l", "p", "size", "p"]),
+    "emu_split_f64_pair": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "p", "l", "i", "p", "p", "p", "size", "p"]),
     "emu_gemm_f32": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "p", "size", "p"]),
     "emu_gemm_f64": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "i", "p", "size", "p"]),
     "emu_gemm_f32_fused": ("i", ["l", "l", "l", "p", "l", "p", "l", "p", "l", "p", "size", "p"]),
@@ -100,6 +102,8 @@ emu_split_f32 = _mk("emu_split_f32")
 emu_split_f64 = _mk("emu_split_f64")
 emu_split_f64_slices = _mk("emu_split_f64_slices")
 emu_gemm_workspace_bytes = _mk("emu_gemm_workspace_bytes")
+emu_split_f32_pair = _mk("emu_split_f32_pair")
+emu_split_f64_pair = _mk("emu_split_f64_pair")
 emu_gemm_f32 = _mk("emu_gemm_f32")
 emu_gemm_f64 = _mk("emu_gemm_f64")
 emu_gemm_f32_fused = _mk("emu_gemm_f32_fused")

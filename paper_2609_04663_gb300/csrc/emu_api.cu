@@ -137,6 +137,42 @@ emu_status emu_split_f64_slices(const double *X, int64_t rows, int64_t cols, int
     return cuda_status(e);
 }
 
+emu_status emu_split_f32_pair(int64_t M, int64_t N, int64_t K, const float *A, int64_t lda, const float *B,
+                              int64_t ldb, uint16_t *Acomps, uint16_t *Bcomps, int64_t ldcomp, void *ws,
+                              size_t ws_bytes, emu_stream_t stream)
+{
+    emu_status s = check_gemm_dims(M, N, K, lda, ldb, N > 0 ? N : 1);
+    if (s != EMU_OK) return s;
+    if (!ws || ldcomp < (K > 0 ? K : 1)) return EMU_ERR_INVALID_ARG;
+    if (M > 0 && N > 0 && K > 0 && (!A || !B || !Acomps || !Bcomps)) return EMU_ERR_INVALID_ARG;
+    if (ws_bytes < kWsHeaderBytes) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
+    if (e == cudaSuccess && M > 0 && N > 0 && K > 0)
+        e = launch_split_f32_gemm(A, M, K, lda, B, N, ldb, Acomps, Bcomps, ldcomp, h, nullptr, 0, st);
+    return cuda_status(e);
+}
+
+emu_status emu_split_f64_pair(int64_t M, int64_t N, int64_t K, const double *A, int64_t lda, const double *B,
+                              int64_t ldb, uint16_t *Acomps, uint16_t *Bcomps, int64_t ldcomp, int nslices,
+                              int32_t *vA, int32_t *vB, void *ws, size_t ws_bytes, emu_stream_t stream)
+{
+    emu_status s = check_gemm_dims(M, N, K, lda, ldb, N > 0 ? N : 1);
+    if (s != EMU_OK) return s;
+    if (nslices < 3 || nslices > 6 || !ws || !vA || !vB || ldcomp < (K > 0 ? K : 1)) return EMU_ERR_INVALID_ARG;
+    if (M > 0 && N > 0 && K > 0 && (!A || !B || !Acomps || !Bcomps)) return EMU_ERR_INVALID_ARG;
+    if (ws_bytes < kWsHeaderBytes) return EMU_ERR_WORKSPACE_TOO_SMALL;
+    if (!aligned16(ws)) return EMU_ERR_MISALIGNED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    WsHeader *h = static_cast<WsHeader *>(ws);
+    cudaError_t e = cudaMemsetAsync(h, 0, sizeof(WsHeader), st);
+    if (e == cudaSuccess)
+        e = launch_split_f64_gemm(A, M, K, lda, B, N, ldb, Acomps, Bcomps, ldcomp, vA, vB, h, st, nslices);
+    return cuda_status(e);
+}
+
 size_t emu_gemm_workspace_bytes(int mode, int64_t M, int64_t N, int64_t K)
 {
     if (M < 0 || N < 0 || K < 0) return 0;
@@ -214,8 +250,7 @@ emu_status emu_gemm_f64_merged(int64_t M, int64_t N, int64_t K, const double *A,
     float *T = merge_from < d ? reinterpret_cast<float *>(static_cast<char *>(ws) + gemm_ws_bytes(6, M, N, K)) : nullptr;
     // the product-sum uses slices 0 .. d-1 only
     const int nlev = f64_diagonals(nprod);
-    e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st, nlev);
-    if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st, nlev);
+    e = launch_split_f64_gemm(A, M, K, lda, B, N, ldb, Ap, Bp, ldk, h->vout[0], h->vout[1], h, st, nlev);
     if (e == cudaSuccess && T) e = launch_prodsum_tail(M, N, K, Ap, Bp, ldk, merge_from, d, T, N, &h->flags, st);
     if (e == cudaSuccess)
         e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], merge_from * (merge_from + 1) / 2, C,
@@ -244,8 +279,7 @@ emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_
     uint16_t *Bp = reinterpret_cast<uint16_t *>(reinterpret_cast<char *>(Ap) + round_up(6 * M * ldk * 2, 256));
     // the product-sum uses slices 0 .. d-1 only
     const int nlev = f64_diagonals(nprod);
-    e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st, nlev);
-    if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st, nlev);
+    e = launch_split_f64_gemm(A, M, K, lda, B, N, ldb, Ap, Bp, ldk, h->vout[0], h->vout[1], h, st, nlev);
     if (e == cudaSuccess)
         e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, C, ldc, gemm_acc(ws, M, N, K),
                                &h->flags, st);

@@ -22,6 +22,13 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
                              uint16_t *comps, int64_t ldcomp, int32_t *v_out, WsHeader *ws, int slot,
                              cudaStream_t st, int nlev = 6);
 
+// Both operands of an FP64 GEMM split as launch_split_f64 splits A (rows x
+// cols = M x K, row-major planes, slot 0) and then B (K x N, K-major planes,
+// slot 1), with the level-maximum passes of the two sharing one launch.
+cudaError_t launch_split_f64_gemm(const double *A, int64_t M, int64_t K, int64_t lda, const double *B, int64_t N,
+                                  int64_t ldb, uint16_t *Ap, uint16_t *Bp, int64_t ldcomp, int32_t *vA_out,
+                                  int32_t *vB_out, WsHeader *ws, cudaStream_t st, int nlev);
+
 // Number of diagonals d of an FP64-mode product count (Eq. (fp64productcounts):
 // nprod = d (d + 1) / 2), i.e. the slices 0 .. d-1 a product-sum reads; 0 for
 // any other count.

@@ -75,8 +75,7 @@ extern "C" emu_status emu_gemm_f64_noalloc(int64_t M, int64_t N, int64_t K, cons
         } else {
             uint16_t *Ap = reinterpret_cast<uint16_t *>(scratch + kWsHeaderBytes);
             uint16_t *Bp = reinterpret_cast<uint16_t *>(scratch + kWsHeaderBytes + a_bytes);
-            e = launch_split_f64(A, M, K, lda, false, Ap, ldk, h->vout[0], h, 0, st, nlev);
-            if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldk, h->vout[1], h, 1, st, nlev);
+            e = launch_split_f64_gemm(A, M, K, lda, B, N, ldb, Ap, Bp, ldk, h->vout[0], h->vout[1], h, st, nlev);
             if (e == cudaSuccess)
                 e = launch_prodsum_f64(M, N, K, Ap, Bp, ldk, h->vout[0], h->vout[1], nprod, C, ldc,
                                        reinterpret_cast<double *>(scratch + kWsHeaderBytes + a_bytes + b_bytes),

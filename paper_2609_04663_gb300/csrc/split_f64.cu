@@ -26,23 +26,25 @@ namespace {
 
 // Row-major planes: thread = 4 consecutive entries of a row (two 16-byte
 // loads, one 8-byte store per plane), rows advancing by the grid's y size.
+// Block (bx, by) of a grid with gy rows of blocks; red: 5 * kThreads / 32
+// words of shared memory.
 template <int NLEV>
-__global__ void __launch_bounds__(kThreads)
-f64_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
-                     uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
+__device__ __forceinline__ void f64_spec_rows_body(const double *__restrict__ X, int64_t rows, int64_t cols,
+                                                   int64_t ldx, uint16_t *__restrict__ comps, int64_t ldcomp,
+                                                   int64_t plane, WsHeader *ws, int slot, int64_t bx, int64_t by,
+                                                   int64_t gy, unsigned long long *red)
 {
-    __shared__ unsigned long long red[5 * (kThreads / 32)];
     const int v0 = spec_v0(ws, slot);
     const bool fast = v0 >= -78;
     float P[6] = {};
     if (fast) spec_units(v0 - 50, P);
     const bool vin = ((ldx & 1) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
     const bool vout = ((ldcomp & 3) == 0) && ((plane & 3) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 7u) == 0);
-    const int64_t j0 = ((int64_t)blockIdx.x * kThreads + threadIdx.x) * 4;
+    const int64_t j0 = (bx * kThreads + threadIdx.x) * 4;
     SpecState st;
     if (j0 < cols) {
         const bool full = j0 + 4 <= cols;
-        for (int64_t i = blockIdx.y; i < rows; i += gridDim.y) {
+        for (int64_t i = by; i < rows; i += gy) {
             const double *src = X + i * ldx + j0;
             double x[4];
             if (vin && full) {
@@ -77,17 +79,27 @@ f64_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, i
     spec_publish(st, v0, ws, slot, red);
 }
 
+template <int NLEV>
+__global__ void __launch_bounds__(kThreads)
+f64_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                     uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
+{
+    __shared__ unsigned long long red[5 * (kThreads / 32)];
+    f64_spec_rows_body<NLEV>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, blockIdx.x, blockIdx.y, gridDim.y, red);
+}
+
 // Transposed (K-major) planes: a 64 x 64 tile, warp q on columns 8q .. 8q+7,
 // lane p on rows 2p and 2p+1; each plane word packs the two entries adjacent
 // in the transposed row, staged one bank per lane and written as 16-byte
 // chunks of whole transposed rows.  Shared memory: [6][64][32] words.
+// Block bid of nblk (tiles with a stride of nblk); smw: [6][kTile][kTile / 2]
+// words, red: 5 * kThreads / 32 words of shared memory.
 template <int NLEV>
-__global__ void __launch_bounds__(kThreads)
-f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
-                          uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
+__device__ __forceinline__ void f64_spec_transpose_body(const double *__restrict__ X, int64_t rows, int64_t cols,
+                                                        int64_t ldx, uint16_t *__restrict__ comps, int64_t ldcomp,
+                                                        int64_t plane, WsHeader *ws, int slot, int64_t bid,
+                                                        int64_t nblk, uint32_t *smw, unsigned long long *red)
 {
-    extern __shared__ __align__(16) uint32_t smw[];                  // [6][kTile][kTile / 2]
-    __shared__ unsigned long long red[5 * (kThreads / 32)];
     const int v0 = spec_v0(ws, slot);
     const bool fast = v0 >= -78;
     float P[6] = {};
@@ -97,7 +109,7 @@ f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t co
     const int q = threadIdx.x >> 5, p = lane_id();
     const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
     SpecState st;
-    for (int64_t t = blockIdx.x; t < tiles_r * tiles_c; t += gridDim.x) {
+    for (int64_t t = bid; t < tiles_r * tiles_c; t += nblk) {
         const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
         const int64_t gj = c0 + 8 * q;
         // two adjacent columns per step (one 16-byte load per row), so that
@@ -149,6 +161,41 @@ f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t co
         __syncthreads();
     }
     spec_publish(st, v0, ws, slot, red);
+}
+
+template <int NLEV>
+__global__ void __launch_bounds__(kThreads)
+f64_spec_transpose_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
+                          uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws, int slot)
+{
+    extern __shared__ __align__(16) uint32_t smw[];                  // [6][kTile][kTile / 2]
+    __shared__ unsigned long long red[5 * (kThreads / 32)];
+    f64_spec_transpose_body<NLEV>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, blockIdx.x, gridDim.x, smw, red);
+}
+
+// Block b of a launch that holds nA blocks of one kind and nB of another:
+// the first 2 min(nA, nB) blocks alternate between the kinds (blocks are
+// dispatched roughly in index order, so both kinds run side by side), the
+// rest belong to the larger kind.  Returns the block's index within its kind.
+__device__ __forceinline__ int64_t pair_block(int64_t b, int64_t nA, int64_t nB, bool &is_a)
+{
+    const int64_t m = nA < nB ? nA : nB;
+    if (b < 2 * m) { is_a = (b & 1) == 0; return b >> 1; }
+    is_a = nA > nB;
+    return m + (b - 2 * m);
+}
+
+// The level-0 maxima of both operands of an FP64 GEMM in one launch: nA
+// blocks on A (header slot 0) and nB on B (slot 1), interleaved.
+__global__ void __launch_bounds__(kThreads)
+f64_max_gemm_kernel(const double *__restrict__ A, int64_t M, int64_t K, int64_t lda, const double *__restrict__ B,
+                    int64_t N, int64_t ldb, WsHeader *ws, int64_t nA, int64_t nB)
+{
+    __shared__ unsigned long long red[kThreads / 32];
+    bool is_a;
+    const int64_t i = pair_block(blockIdx.x, nA, nB, is_a);
+    if (is_a) f64_max_pass<0>(A, M, K, lda, ws, 0, i, nA, red);
+    else f64_max_pass<0>(B, K, N, ldb, ws, 1, i, nB, red);
 }
 
 // The fused speculative pass for slices 0 .. NLEV-1.
@@ -203,5 +250,56 @@ cudaError_t launch_split_f64(const double *X, int64_t rows, int64_t cols, int64_
     return launch_f64_fix_empty(ws, slot, v_out, st);
 }
 
+
+// Both operands of an FP64 GEMM (A: M x K into row-major planes, B: K x N
+// into K-major planes, row pitch ldcomp), with the level maxima of A and B in
+// one launch; the speculative passes and verifiers stay one launch per
+// operand.  Results are those of launch_split_f64 on A, then B.
+cudaError_t launch_split_f64_gemm(const double *A, int64_t M, int64_t K, int64_t lda, const double *B, int64_t N,
+                                  int64_t ldb, uint16_t *Ap, uint16_t *Bp, int64_t ldcomp, int32_t *vA_out,
+                                  int32_t *vB_out, WsHeader *ws, cudaStream_t st, int nlev)
+{
+    if (nlev < 3 || nlev > 6) return cudaErrorInvalidValue;
+    if (M == 0 || N == 0 || K == 0) {
+        cudaError_t e = launch_split_f64(A, M, K, lda, false, Ap, ldcomp, vA_out, ws, 0, st, nlev);
+        if (e == cudaSuccess) e = launch_split_f64(B, K, N, ldb, true, Bp, ldcomp, vB_out, ws, 1, st, nlev);
+        return e;
+    }
+    // level-0 maxima: blocks shared in proportion to the entries, at most 152 x 8 in all
+    const int64_t segA = M * ((K + 4 * kThreads - 1) / (4 * kThreads)), segB = K * ((N + 4 * kThreads - 1) / (4 * kThreads));
+    const double fa = (double)(M * K) / (double)(M * K + K * N);
+    int64_t nA = (int64_t)(152 * 8 * fa + 0.5), nB = 152 * 8 - nA;
+    nA = nA < 1 ? 1 : (nA > segA ? segA : nA);
+    nB = nB < 1 ? 1 : (nB > segB ? segB : nB);
+    f64_max_gemm_kernel<<<(unsigned)(nA + nB), kThreads, 0, st>>>(A, M, K, lda, B, N, ldb, ws, nA, nB);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    // the speculative passes stay one launch per operand: in one launch the
+    // row blocks would reserve the transposed blocks' shared memory (measured
+    // 15-25 % slower)
+    const int gB = grid_for(((K + kTile - 1) / kTile) * ((N + kTile - 1) / kTile), 152 * 8);
+    switch (nlev) {
+    case 3:
+        e = launch_spec<3>(A, M, K, lda, false, Ap, ldcomp, M * ldcomp, ws, 0, 0, st);
+        if (e == cudaSuccess) e = launch_spec<3>(B, K, N, ldb, true, Bp, ldcomp, N * ldcomp, ws, 1, gB, st);
+        break;
+    case 4:
+        e = launch_spec<4>(A, M, K, lda, false, Ap, ldcomp, M * ldcomp, ws, 0, 0, st);
+        if (e == cudaSuccess) e = launch_spec<4>(B, K, N, ldb, true, Bp, ldcomp, N * ldcomp, ws, 1, gB, st);
+        break;
+    case 5:
+        e = launch_spec<5>(A, M, K, lda, false, Ap, ldcomp, M * ldcomp, ws, 0, 0, st);
+        if (e == cudaSuccess) e = launch_spec<5>(B, K, N, ldb, true, Bp, ldcomp, N * ldcomp, ws, 1, gB, st);
+        break;
+    default:
+        e = launch_spec<6>(A, M, K, lda, false, Ap, ldcomp, M * ldcomp, ws, 0, 0, st);
+        if (e == cudaSuccess) e = launch_spec<6>(B, K, N, ldb, true, Bp, ldcomp, N * ldcomp, ws, 1, gB, st);
+        break;
+    }
+    if (e == cudaSuccess) e = cudaGetLastError();
+    if (e == cudaSuccess) e = launch_f64_fix(A, M, K, lda, false, Ap, ldcomp, M * ldcomp, ws, 0, vA_out, st, nlev);
+    if (e == cudaSuccess) e = launch_f64_fix(B, K, N, ldb, true, Bp, ldcomp, N * ldcomp, ws, 1, vB_out, st, nlev);
+    return e;
+}
 
 }  // namespace emu

@@ -227,3 +227,57 @@ def test_split_f64_empty_operands(dev, shape, transpose):
         planes, v, ws = emu.split_f64_rowcol(X, transpose=transpose, ldcomp=8)
         assert emu.read_flags(ws) == 0
         assert (v.cpu().numpy() == oracle.ZERO_LEVEL).all()
+
+
+def _gap_matrix(rng, shape, gap_level, scale=3):
+    """Integers times descending powers of two, so that the speculative levels
+    hold below gap_level and fail at it (gap_level 0: they all hold)."""
+    X = rng.integers(-127, 128, size=shape) * 2.0**10
+    for r in range(1, gap_level or 6):
+        X = X + rng.integers(-127, 128, size=shape) * 2.0**(10 - 8 * r)
+    if gap_level:
+        X = X + rng.integers(-127, 128, size=shape) * 2.0**(10 - 8 * gap_level - scale)
+    X[0, 0] = 127 * 2.0**10
+    return X
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 333, 700), (129, 257, 33), (1000, 64, 520), (1, 1, 1)])
+def test_pair_splits_equal_single_operand_splits(dev, M, N, K):
+    """emu_split_f32_pair / emu_split_f64_pair (the split step the GEMMs run,
+    both operands sharing launches): planes and levels identical to the
+    single-operand splits; FP64 with the speculative levels holding, and
+    failing at a level of A only or of B only."""
+    torch = emu._torch()
+    ldk = emu.gemm_ldk(K)
+    A, B = synth.gemm_inputs("f32", M, N, K, 71)
+    Ad, Bd = to_dev(A, dev), to_dev(B, dev)
+    Ap = torch.zeros((3, M, ldk), dtype=torch.int16, device=dev)
+    Bp = torch.zeros((3, N, ldk), dtype=torch.int16, device=dev)
+    ws = emu.workspace(emu.emu_split_workspace_bytes(32), dev)
+    assert emu.emu_split_f32_pair(M, N, K, Ad.data_ptr(), K, Bd.data_ptr(), N, Ap.data_ptr(), Bp.data_ptr(), ldk,
+                                  ws.data_ptr(), ws.numel(), emu._stream(None)) == 0
+    assert emu.read_flags(ws) == 0
+    Ar, _ = emu.split_f32(Ad, ldcomp=ldk)
+    Br, _ = emu.split_f32(Bd, transpose=True, ldcomp=ldk)
+    assert torch.equal(Ap[:, :, :K], Ar[:, :, :K]) and torch.equal(Bp[:, :, :K], Br[:, :, :K])
+    rng = np.random.default_rng(72)
+    for nslices in (3, 6):
+        for ga, gb in ((0, 0), (2, 0), (0, 4)):
+            A64 = _gap_matrix(rng, (M, K), ga)
+            B64 = _gap_matrix(rng, (K, N), gb)
+            Ad, Bd = to_dev(A64, dev), to_dev(B64, dev)
+            Ap = torch.zeros((6, M, ldk), dtype=torch.int16, device=dev)
+            Bp = torch.zeros((6, N, ldk), dtype=torch.int16, device=dev)
+            vA = torch.empty(6, dtype=torch.int32, device=dev)
+            vB = torch.empty(6, dtype=torch.int32, device=dev)
+            ws = emu.workspace(emu.emu_split_workspace_bytes(64), dev)
+            assert emu.emu_split_f64_pair(M, N, K, Ad.data_ptr(), K, Bd.data_ptr(), N, Ap.data_ptr(), Bp.data_ptr(),
+                                          ldk, nslices, vA.data_ptr(), vB.data_ptr(), ws.data_ptr(), ws.numel(),
+                                          emu._stream(None)) == 0
+            Ar, vAr, wa = emu.split_f64(Ad, ldcomp=ldk, nslices=nslices)
+            Br, vBr, wb = emu.split_f64(Bd, transpose=True, ldcomp=ldk, nslices=nslices)
+            assert emu.read_flags(ws) == emu.read_flags(wa) | emu.read_flags(wb)
+            n = nslices
+            assert torch.equal(Ap[:n, :, :K], Ar[:n, :, :K]), (nslices, ga, gb)
+            assert torch.equal(Bp[:n, :, :K], Br[:n, :, :K]), (nslices, ga, gb)
+            assert torch.equal(vA[:n], vAr[:n]) and torch.equal(vB[:n], vBr[:n]), (nslices, ga, gb)
