@@ -109,26 +109,36 @@ __device__ __forceinline__ void f64_spec_transpose_body(const double *__restrict
     const int q = threadIdx.x >> 5, p = lane_id();
     const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
     SpecState st;
+    // this thread's two entries of column pair k of tile t's rows 2p, 2p + 1
+    auto load = [&](int64_t t, int k, double (&x)[2][2]) {
+        const int64_t r0 = (t / tiles_c) * kTile, gj = (t % tiles_c) * kTile + 8 * q;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int64_t gi = r0 + 2 * p + h;
+            const double *src = X + gi * ldx + gj + k;
+            if (gi < rows && vin && gj + 8 <= cols) {
+                const double2 a = *reinterpret_cast<const double2 *>(src);
+                x[h][0] = a.x; x[h][1] = a.y;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 2; ++e) x[h][e] = (gi < rows && gj + k + e < cols) ? src[e] : 0.0;
+            }
+        }
+    };
+    double xn[2][2] = {{0.0, 0.0}, {0.0, 0.0}};
+    if (bid < tiles_r * tiles_c) load(bid, 0, xn);
     for (int64_t t = bid; t < tiles_r * tiles_c; t += nblk) {
         const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
-        const int64_t gj = c0 + 8 * q;
         // two adjacent columns per step (one 16-byte load per row), so that
-        // the element body appears four times in the loop, not sixteen
+        // the element body appears four times in the loop, not sixteen; the
+        // next step's entries are loaded before this step is split
 #pragma unroll 1
         for (int k = 0; k < 8; k += 2) {
             double x[2][2];
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int64_t gi = r0 + 2 * p + h;
-                const double *src = X + gi * ldx + gj + k;
-                if (gi < rows && vin && gj + 8 <= cols) {
-                    const double2 a = *reinterpret_cast<const double2 *>(src);
-                    x[h][0] = a.x; x[h][1] = a.y;
-                } else {
-#pragma unroll
-                    for (int e = 0; e < 2; ++e) x[h][e] = (gi < rows && gj + k + e < cols) ? src[e] : 0.0;
-                }
-            }
+            for (int h = 0; h < 2; ++h) { x[h][0] = xn[h][0]; x[h][1] = xn[h][1]; }
+            if (k + 2 < 8) load(t, k + 2, xn);
+            else if (t + nblk < tiles_r * tiles_c) load(t + nblk, 0, xn);
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
                 uint32_t s0[6], s1[6];
