@@ -224,24 +224,17 @@ class Case:
             self.gemm_ws = emu.workspace(emu.emu_gemm_f64_merged_workspace_bytes(M, N, K), dev)
         if self.api:
             self.gemm_ws = emu.workspace(emu.emu_gemm_workspace_bytes(self.mode, M, N, K), dev)
-        # the product-sum kernel that runs: FP64 mode has a 128 x 128 and a 128 x 256 tile
+        # the product-sum kernel that runs: FP64 mode has 128 x 128 tiles and 256-column tiles
+        # (128 x 256 on one SM, 256 x 256 on a pair of SMs), both kernels named after their file
         self.kernel = "prodsum_f32" if self.mode == 32 else \
             "prodsum_f64w" if emu.emu_prodsum_f64_tile_columns(M, N) == 256 else "prodsum_f64"
         self.flop = 2.0 * M * N * K
         self.exec_flop = self.flop * (6 if self.mode == 32 else self.nprod)
         # kernels of ours per step: FP32 split of both operands = 1 launch; FP64 split of both =
         # 5 (level maxima of both, then a speculative pass and a verifier per operand);
-        # product-sum = 1 (FP64 with its last partial wave on 128 x 128 tiles: 2)
-        self.launches = 1 if self.fused else 2 if self.mode == 32 else 5 + 1
-        if self.kernel == "prodsum_f64w":
-            # the library's schedule: full waves of 128 x 256 tiles, the rest as 128 x 128
-            # halves in a second launch when that is estimated at least 3 % faster
-            sms = torch.cuda.get_device_properties(0).multi_processor_count
-            tiles = ((M + 127) // 128) * ((N + 255) // 256)
-            full, rem = (tiles // sms) * sms, tiles % sms
-            t_wide, t_mixed = -(-tiles // sms), full // sms + (0.5 / 0.76) * -(-2 * rem // sms)
-            if full > 0 and rem > 0 and t_mixed < 0.97 * t_wide:
-                self.launches += 1
+        # product-sum = 1, or in FP64 mode 2 when the library runs the last partial wave of
+        # 256-column tiles as 128 x 128 tiles (it reports its schedule)
+        self.launches = 1 if self.fused else 2 if self.mode == 32 else 5 + emu.emu_prodsum_f64_launches(M, N)
         if self.merge_from is not None:
             self.launches += 1                    # the tail kernel
         if self.api and self.mode == 32:

@@ -305,11 +305,17 @@ emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
  * or another mode. */
 size_t emu_prodsum_workspace_bytes(int mode, int64_t M, int64_t N);
 
-/* Output-tile width (128 or 256 columns; 128 rows either way) that the
- * FP64-mode product-sum picks for an M x N result, unless EMU_F64_TILE
- * forces one.  The paper has no counterpart: both widths give identical
- * results, and the call only reports which kernel runs.  0 for sizes < 1. */
+/* Output-tile shape that the FP64-mode product-sum picks for an M x N
+ * result, unless EMU_F64_TILE (128x128, 128x256 or 256x256) forces one:
+ * width 128 or 256 columns; height 128 rows, or 256 rows where a 256-column
+ * tile runs on a pair of SMs (a cluster of two CTAs sharing each MMA); and
+ * the number of kernel launches (2 when the last, partial wave of 256-column
+ * tiles runs as 128 x 128 tiles in a second launch).  The paper has no
+ * counterpart: every shape gives identical results, and the calls only
+ * report which kernels run.  0 for sizes < 1. */
 int emu_prodsum_f64_tile_columns(int64_t M, int64_t N);
+int emu_prodsum_f64_tile_rows(int64_t M, int64_t N);
+int emu_prodsum_f64_launches(int64_t M, int64_t N);
 
 /* Product-sum alone for FP64 mode, Eq. (fp64reconstruction), summed as in
  * emu_gemm_f64: A planes [6][M][ldcomp], B planes [6][N][ldcomp]; nprod in

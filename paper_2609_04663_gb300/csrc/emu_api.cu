@@ -292,6 +292,18 @@ int emu_prodsum_f64_tile_columns(int64_t M, int64_t N)
     return f64_tile_columns(M, N);
 }
 
+int emu_prodsum_f64_tile_rows(int64_t M, int64_t N)
+{
+    if (M < 1 || N < 1) return 0;
+    return f64_plan(M, N).rows;
+}
+
+int emu_prodsum_f64_launches(int64_t M, int64_t N)
+{
+    if (M < 1 || N < 1) return 0;
+    return f64_plan(M, N).launches;
+}
+
 size_t emu_prodsum_workspace_bytes(int mode, int64_t M, int64_t N)
 {
     if (M < 0 || N < 0 || (mode != 32 && mode != 64)) return 0;

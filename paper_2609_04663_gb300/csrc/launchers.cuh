@@ -93,15 +93,25 @@ cudaError_t launch_prodsum_tail(int64_t M, int64_t N, int64_t K, const uint16_t 
                                 int64_t ldcomp, int L, int d, float *T, int64_t ldt, uint32_t *flags,
                                 cudaStream_t st);
 
+// How the FP64 product-sum covers an M x N result: tiles of rows x cols
+// (128 x 128, 128 x 256, or 256 x 256 on CTA pairs), `tiles` of them in the
+// first launch and, when launches == 2, the remaining rest tiles as 128 x 128
+// parts in a second launch of the 128 x 128 kernel.
+struct F64Plan {
+    int rows = 0, cols = 0, launches = 0;
+    int64_t tiles = 0, rest = 0;
+};
+F64Plan f64_plan(int64_t M, int64_t N);
 // Tile width (128 or 256) the FP64 product-sum picks for an M x N result.
 int f64_tile_columns(int64_t M, int64_t N);
-// The FP64 product-sum on 128 x 256 tiles (prodsum_f64w.cu); launch_prodsum_f64
-// calls it when that tile shape is chosen, for the first ctas tiles in raster
-// order.  acc: f64_acc_bytes(M, N) bytes.
+// The FP64 product-sum on 128 x 256 tiles, or with pair on 256 x 256 tiles
+// computed by clusters of two CTAs (prodsum_f64w.cu); launch_prodsum_f64
+// calls it for the first `tiles` tiles in raster order.  acc:
+// f64_acc_bytes(M, N) bytes.
 cudaError_t launch_prodsum_f64_wide(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                     int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
                                     int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
-                                    bool rowcol, const float *T, int64_t ldt, int64_t ctas);
+                                    bool rowcol, const float *T, int64_t ldt, int64_t tiles, bool pair);
 
 // Bytes of the FP64 product-sum's accumulator, enough for either tile shape:
 // one FP64 tile of 128 x 128 (narrow kernel) or 128 x 256 (wide kernel) per

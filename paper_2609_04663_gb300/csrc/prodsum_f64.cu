@@ -84,7 +84,7 @@ __global__ void __launch_bounds__(F64Cfg::THREADS, 1)
 prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    int M, int N, int K, const int32_t *__restrict__ vA, const int32_t *__restrict__ vB,
                    double *__restrict__ C, int64_t ldc, double *__restrict__ acc, uint32_t *flags,
-                   const float *__restrict__ T, int64_t ldt, int wide_first)
+                   const float *__restrict__ T, int64_t ldt, int wide_first, int wide_rows)
 {
     using Cfg = F64Cfg;
     extern __shared__ uint8_t smem_raw[];
@@ -103,12 +103,17 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     if (wide_first < 0) {
         tile_coords(blockIdx.x, tiles_m, tiles_n, tm, tn);
     } else {
-        // the two 128-column halves of the 128 x 256 tiles from raster index
-        // wide_first on, which the wide kernel's last, partial wave would have taken
-        int tnw;
-        tile_coords(wide_first + (int)(blockIdx.x >> 1), tiles_m, (N + 255) / 256, tm, tnw);
-        tn = 2 * tnw + (int)(blockIdx.x & 1);
-        if (tn >= tiles_n) return;                    // a half past the last column
+        // the 128 x 128 parts of the (128 * wide_rows) x 256 tiles from raster
+        // index wide_first on, which the wide kernel's last, partial wave
+        // would have taken: two column halves per 128-row tile row
+        const int per = 2 * wide_rows;
+        int tw, tnw;
+        tile_coords(wide_first + (int)(blockIdx.x / per), (tiles_m + wide_rows - 1) / wide_rows, (N + 255) / 256,
+                    tw, tnw);
+        const int sub = (int)(blockIdx.x % per);
+        tm = tw * wide_rows + (sub >> 1);
+        tn = 2 * tnw + (sub & 1);
+        if (tm >= tiles_m || tn >= tiles_n) return;   // a part past the last row or column
     }
     const int m0 = tm * kBM, n0 = tn * Cfg::BN;
     const int nch = (K + kKChunk - 1) / kKChunk;
@@ -407,7 +412,8 @@ constexpr double kF64RateNarrow = 0.76;
 template <int NPROD, bool ROWCOL, bool TAIL = false>
 cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
                     const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, double *acc, uint32_t *flags,
-                    cudaStream_t st, int64_t a_plane, const float *T, int64_t ldt, int wide_first, int64_t ctas)
+                    cudaStream_t st, int64_t a_plane, const float *T, int64_t ldt, int wide_first, int wide_rows,
+                    int64_t ctas)
 {
     using Cfg = F64Cfg;
     CUtensorMap ta, tb;
@@ -418,7 +424,7 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
     if (e != cudaSuccess) return e;
     const int64_t tiles = wide_first < 0 ? ((M + kBM - 1) / kBM) * ((N + Cfg::BN - 1) / Cfg::BN) : ctas;
     kern<<<(unsigned)tiles, Cfg::THREADS, Cfg::SMEM, st>>>(ta, tb, (int)M, (int)N, (int)K, vA, vB, C, ldc, acc, flags,
-                                                           T, ldt, wide_first);
+                                                           T, ldt, wide_first, wide_rows);
     return cudaGetLastError();
 }
 
@@ -427,66 +433,116 @@ cudaError_t run_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
 static cudaError_t launch_prodsum_f64_narrow(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
                                int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
-                               bool rowcol, const float *T, int64_t ldt, int wide_first = -1, int64_t ctas = 0)
+                               bool rowcol, const float *T, int64_t ldt, int wide_first = -1, int wide_rows = 1,
+                               int64_t ctas = 0)
 {
+#define EMU_F64N(NP, RC, TL) \
+    run_f64<NP, RC, TL>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, wide_first, \
+                        wide_rows, ctas)
     if (T) {                                          // merged tail: whole-matrix levels only
         if (rowcol) return cudaErrorInvalidValue;
         switch (nprod) {
-        case 6: return run_f64<6, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, wide_first, ctas);
-        case 10: return run_f64<10, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, wide_first, ctas);
-        case 15: return run_f64<15, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, wide_first, ctas);
+        case 6: return EMU_F64N(6, false, true);
+        case 10: return EMU_F64N(10, false, true);
+        case 15: return EMU_F64N(15, false, true);
         default: return cudaErrorInvalidValue;
         }
     }
     switch (nprod) {
-    case 6: return rowcol ? run_f64<6, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas)
-                   : run_f64<6, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas);
-    case 10: return rowcol ? run_f64<10, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas)
-                   : run_f64<10, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas);
-    case 15: return rowcol ? run_f64<15, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas)
-                   : run_f64<15, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas);
-    case 21: return rowcol ? run_f64<21, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas)
-                   : run_f64<21, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, wide_first, ctas);
+    case 6: return rowcol ? EMU_F64N(6, true, false) : EMU_F64N(6, false, false);
+    case 10: return rowcol ? EMU_F64N(10, true, false) : EMU_F64N(10, false, false);
+    case 15: return rowcol ? EMU_F64N(15, true, false) : EMU_F64N(15, false, false);
+    case 21: return rowcol ? EMU_F64N(21, true, false) : EMU_F64N(21, false, false);
     default: return cudaErrorInvalidValue;
     }
+#undef EMU_F64N
 }
 
-// Tile shape of the FP64 product-sum.  128 x 256 (prodsum_f64w.cu) takes in
-// 0.75x the operand bytes per FLOP of 128 x 128 and is faster per SM, but
-// gives half as many CTAs; the choice maximises (SMs kept busy over the waves)
-// x (relative per-SM rate), as for the FP32 product-sum.  Both shapes form
-// the same exact per-product sums and fold them in the same order, so C does
-// not depend on the choice.  EMU_F64_TILE=128x128 / 128x256 forces one.
-// EMU_F64_TILE=128x128 / 128x256: one tile width for every result (0: unset).
+// Tile shape of the FP64 product-sum.  Every shape forms the same exact
+// per-product sums and folds them in the same order, so C does not depend on
+// the choice.
+// - 128 x 256 tiles (prodsum_f64w.cu) take in 0.75x the operand bytes per FLOP
+//   of 128 x 128 and are faster per SM, but give half as many CTAs; the width
+//   maximises (SMs kept busy over the waves) x (relative per-SM rate), as for
+//   the FP32 product-sum.
+// - With two or more 128-row tile rows, the 256-column tiles run as 256 x 256
+//   tiles on CTA pairs (the same kernel with cta_group::2 MMAs): each SM then
+//   stages 8 KB of operands per 2^20 FLOP instead of 12 KB.
+// - When those tiles leave the last wave partly empty, the full waves run as
+//   such and the narrow kernel, launched after them, takes the remaining
+//   tiles as 128 x 128 parts, if that is estimated faster (a part takes
+//   0.5 / kF64RateNarrow of a 128 x 256 tile's time).  The two kernels run one
+//   after the other, so the accumulator tiles they index differently never
+//   overlap in time.
+// EMU_F64_TILE=128x128 / 128x256 / 256x256 forces one shape for every result
+// (and no mixed last wave).
 static int f64_tile_forced()
 {
     static const int forced = [] {
         const char *e = std::getenv("EMU_F64_TILE");
-        if (!e || std::strncmp(e, "128x", 4) != 0) return 0;
-        return std::strcmp(e + 4, "256") == 0 ? 256 : std::strcmp(e + 4, "128") == 0 ? 128 : 0;
+        if (!e) return 0;
+        if (std::strcmp(e, "128x128") == 0) return 1;
+        if (std::strcmp(e, "128x256") == 0) return 2;
+        if (std::strcmp(e, "256x256") == 0) return 3;
+        return 0;
     }();
     return forced;
 }
 
-int f64_tile_columns(int64_t M, int64_t N)
+static int device_sms()
 {
-    int bn = f64_tile_forced();
-    if (bn == 0) {
-        int dev = 0, sms = 0;
-        if (cudaGetDevice(&dev) != cudaSuccess ||
-            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
-            sms = 152;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 2)
+        sms = 152;
+    return sms;
+}
+
+F64Plan f64_plan(int64_t M, int64_t N)
+{
+    F64Plan p;
+    if (M < 1 || N < 1) return p;
+    const int forced = f64_tile_forced();
+    const int sms = device_sms();
+    const int64_t tiles_m = (M + kBM - 1) / kBM;
+    int cols = forced == 1 ? 128 : forced >= 2 ? 256 : 0;
+    if (cols == 0) {
         const int widths[2] = {256, 128};
         const double rate[2] = {1.0, kF64RateNarrow};
         double best = -1.0;
         for (int i = 0; i < 2; ++i) {
-            const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + widths[i] - 1) / widths[i]);
+            const int64_t tiles = tiles_m * ((N + widths[i] - 1) / widths[i]);
             const int64_t waves = (tiles + sms - 1) / sms;
             const double score = rate[i] * (double)tiles / (double)(waves * sms);
-            if (score > best * 1.02) { best = score; bn = widths[i]; }   // prefer the wider tile on near ties
+            if (score > best * 1.02) { best = score; cols = widths[i]; }   // prefer the wider tile on near ties
         }
     }
-    return bn;
+    p.cols = cols;
+    p.rows = kBM;
+    p.launches = 1;
+    if (cols == 128) {
+        p.tiles = tiles_m * ((N + 127) / 128);
+        return p;
+    }
+    const bool pair = forced == 3 || (forced == 0 && tiles_m >= 2);
+    const int rows_per = pair ? 2 : 1, slots = pair ? sms / 2 : sms;
+    p.rows = kBM * rows_per;
+    const int64_t tiles = ((tiles_m + rows_per - 1) / rows_per) * ((N + 255) / 256);
+    const int64_t full = (tiles / slots) * slots, rem = tiles - full;
+    const double t_wide = (double)((tiles + slots - 1) / slots);
+    const double t_mixed = (double)(full / slots) + (0.5 / kF64RateNarrow) * (double)((2 * rows_per * rem + sms - 1) / sms);
+    p.tiles = tiles;
+    if (forced == 0 && full > 0 && rem > 0 && t_mixed < 0.97 * t_wide) {
+        p.tiles = full;
+        p.rest = 2 * rows_per * rem;
+        p.launches = 2;
+    }
+    return p;
+}
+
+int f64_tile_columns(int64_t M, int64_t N)
+{
+    return f64_plan(M, N).cols;
 }
 
 cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
@@ -494,33 +550,16 @@ cudaError_t launch_prodsum_f64(int64_t M, int64_t N, int64_t K, const uint16_t *
                                int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
                                bool rowcol, const float *T, int64_t ldt)
 {
-    if (f64_tile_columns(M, N) == 256) {
-        // When the 128 x 256 tiles leave the last wave partly empty, the wide
-        // kernel takes the full waves and the narrow kernel, launched after it,
-        // the remaining tiles as twice as many 128 x 128 halves, if that is
-        // estimated faster (a half takes 0.5 / kF64RateNarrow of a wide tile's
-        // time).  The two kernels run one after the other, so the accumulator
-        // tiles they index differently never overlap in time.
-        int dev = 0, sms = 0;
-        if (cudaGetDevice(&dev) != cudaSuccess ||
-            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
-            sms = 152;
-        const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + 255) / 256);
-        const int64_t full = (tiles / sms) * sms, rem = tiles - full;
-        const double t_wide = (double)((tiles + sms - 1) / sms);
-        const double t_mixed = (double)(full / sms) + (0.5 / kF64RateNarrow) * (double)((2 * rem + sms - 1) / sms);
-        if (!f64_tile_forced() && full > 0 && rem > 0 && t_mixed < 0.97 * t_wide) {
-            cudaError_t e = launch_prodsum_f64_wide(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st,
-                                                    a_plane, rowcol, T, ldt, full);
-            if (e != cudaSuccess) return e;
-            return launch_prodsum_f64_narrow(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane,
-                                             rowcol, T, ldt, (int)full, 2 * rem);
-        }
-        return launch_prodsum_f64_wide(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane,
-                                       rowcol, T, ldt, tiles);
-    }
-    return launch_prodsum_f64_narrow(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane,
-                                     rowcol, T, ldt);
+    const F64Plan p = f64_plan(M, N);
+    if (p.cols == 128)
+        return launch_prodsum_f64_narrow(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane,
+                                         rowcol, T, ldt);
+    const bool pair = p.rows == 2 * kBM;
+    cudaError_t e = launch_prodsum_f64_wide(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane,
+                                            rowcol, T, ldt, p.tiles, pair);
+    if (e != cudaSuccess || p.rest == 0) return e;
+    return launch_prodsum_f64_narrow(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane, rowcol,
+                                     T, ldt, (int)p.tiles, pair ? 2 : 1, p.rest);
 }
 
 }  // namespace emu

@@ -48,12 +48,19 @@ namespace emu {
 
 namespace {
 
-struct F64WCfg {
-    static constexpr int BN = 256, KB = 64, STAGES = 4, NBUF = 2;
-    static constexpr int A_TILE = kBM * KB * 2, B_TILE = BN * KB * 2;    // 16 KB + 32 KB
+// PAIR: a cluster of two CTAs computes a 256 x 256 tile with cta_group::2
+// MMAs (M = 256); each CTA stages its 128 rows of the A slice and its 128-row
+// half of the B slice and holds its 128 x 256 part of the partials, so a CTA
+// takes in 8 KB of operands per 2^20 FLOP instead of 12 KB.
+template <bool PAIR>
+struct F64WCfgT {
+    static constexpr int BN = 256, KB = 64, NBUF = 2;
+    static constexpr int BH = PAIR ? BN / 2 : BN;                       // B rows staged by this CTA
+    static constexpr int STAGES = PAIR ? 6 : 4;
+    static constexpr int A_TILE = kBM * KB * 2, B_TILE = BH * KB * 2;   // 16 KB + 32 KB (pair: 16 KB)
     static constexpr int STAGE = A_TILE + B_TILE;
     static constexpr uint32_t SWZ = 2u, SBO = 1024u;                     // 128-byte swizzle
-    static constexpr int BAR_OFF = STAGES * STAGE;
+    static constexpr int BAR_OFF = STAGES * STAGE + (PAIR ? 16384 : 0);
     // barriers: full/empty per stage, tfull/tempty per buffer, done; then the TMEM address slot
     static constexpr int NBARS = 2 * STAGES + 2 * NBUF + 1;
     static constexpr int SMEM = BAR_OFF + 256 + 1024;
@@ -65,14 +72,15 @@ struct F64WCfg {
     // 512 x 112 (drain) = 61440 = 640 x 96.
     static constexpr int REG_CTRL = 32, REG_DRAIN = 112, REG_LAUNCH = 96;
     static constexpr int TILE_ELEMS = kBM * BN;
+    static_assert(NBUF * BN == 512, "TMEM budget: two 256-column partial buffers");
+    static_assert(kKChunk % KB == 0, "a K-chunk is a whole number of stages");
+    static_assert(8 * NBARS + 8 <= 256, "barrier area");
+    static_assert(SMEM <= 232448, "shared memory per CTA");
+    static_assert(128 * REG_CTRL + 512 * REG_DRAIN <= THREADS * REG_LAUNCH,
+                  "setmaxnreg split exceeds the registers reserved at launch");
+    static_assert(COLS % 16 == 0, "drain columns come in groups of 16");
 };
-static_assert(F64WCfg::NBUF * F64WCfg::BN == 512, "TMEM budget: two 256-column partial buffers");
-static_assert(kKChunk % F64WCfg::KB == 0, "a K-chunk is a whole number of stages");
-static_assert(8 * F64WCfg::NBARS + 8 <= 256, "barrier area");
-static_assert(F64WCfg::SMEM <= 232448, "shared memory per CTA");
-static_assert(128 * F64WCfg::REG_CTRL + 512 * F64WCfg::REG_DRAIN <= F64WCfg::THREADS * F64WCfg::REG_LAUNCH,
-              "setmaxnreg split exceeds the registers reserved at launch");
-static_assert(F64WCfg::COLS % 16 == 0, "drain columns come in groups of 16");
+using F64WCfg = F64WCfgT<false>;
 
 // FP64 reduction in L2: *p <- fl64(*p + x), round to nearest even.
 __device__ __forceinline__ void red_add_f64(double *p, double x)
@@ -88,14 +96,14 @@ __device__ __forceinline__ double ld_cg_f64(const double *p)
 }
 
 // TAIL: add the merged tail T (an M x N FP32 matrix) once after the last product.
-template <int NPROD, bool ROWCOL, bool TAIL>
+template <int NPROD, bool ROWCOL, bool TAIL, bool PAIR>
 __global__ void __launch_bounds__(F64WCfg::THREADS, 1)
 prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     int M, int N, int K, const int32_t *__restrict__ vA, const int32_t *__restrict__ vB,
                     double *__restrict__ C, int64_t ldc, double *__restrict__ acc, uint32_t *flags,
                     const float *__restrict__ T, int64_t ldt)
 {
-    using Cfg = F64WCfg;
+    using Cfg = F64WCfgT<PAIR>;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -106,21 +114,39 @@ prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(base_ptr + Cfg::BAR_OFF + 8 * Cfg::NBARS);
 
     const int warp = threadIdx.x >> 5, lane = lane_id();
-    const int tiles_m = (M + kBM - 1) / kBM, tiles_n = (N + Cfg::BN - 1) / Cfg::BN;
+    const uint32_t rank = PAIR ? cluster_rank() : 0u;
+    const int tiles_n = (N + Cfg::BN - 1) / Cfg::BN;
     int tm, tn;
-    tile_coords(blockIdx.x, tiles_m, tiles_n, tm, tn);
+    if constexpr (PAIR) {                             // the pair's 256 rows: this CTA takes half `rank`
+        int tp;
+        tile_coords((int)(blockIdx.x >> 1), (M + 2 * kBM - 1) / (2 * kBM), tiles_n, tp, tn);
+        tm = 2 * tp + (int)rank;
+    } else {
+        tile_coords(blockIdx.x, (M + kBM - 1) / kBM, tiles_n, tm, tn);
+    }
     const int m0 = tm * kBM, n0 = tn * Cfg::BN;
     const int nch = (K + kKChunk - 1) / kKChunk;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < Cfg::STAGES; ++s) { mbar_init(full0 + 8u * s, 1); mbar_init(empty0 + 8u * s, 1); }
-        for (int b = 0; b < Cfg::NBUF; ++b) { mbar_init(tfull0 + 8u * b, 1); mbar_init(tempty0 + 8u * b, Cfg::DRAIN_WARPS); }
+        // a pair's TMEM buffers are released by the drain warps of both CTAs,
+        // on the leader's barriers
+        for (int b = 0; b < Cfg::NBUF; ++b) {
+            mbar_init(tfull0 + 8u * b, 1);
+            mbar_init(tempty0 + 8u * b, (PAIR ? 2 : 1) * Cfg::DRAIN_WARPS);
+        }
         mbar_init(done_bar, 1);
         fence_mbar_init();
         tma_prefetch_desc(&tmA);
         tma_prefetch_desc(&tmB);
     }
-    if (warp == 1) { tmem_alloc(smem_u32((const void *)tmem_slot), 512); tmem_relinquish(); }
+    if constexpr (PAIR) {
+        __syncthreads();
+        cluster_sync();                               // both CTAs' barriers initialised
+        if (warp == 1) tmem_alloc_pair(smem_u32((const void *)tmem_slot), 512);
+    } else {
+        if (warp == 1) { tmem_alloc(smem_u32((const void *)tmem_slot), 512); tmem_relinquish(); }
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -141,17 +167,34 @@ prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     if (!(ok = mbar_wait(empty0 + 8u * s, ph ^ 1u, flags))) break;
                     const uint32_t st = base + (uint32_t)(s * Cfg::STAGE), fb = full0 + 8u * s;
                     const int k0 = c * kKChunk + u * Cfg::KB;
-                    mbar_arrive_expect_tx(fb, Cfg::STAGE);
-                    tma_load_3d(st, &tmA, fb, k0, m0, ia);
-                    tma_load_3d(st + Cfg::A_TILE, &tmB, fb, k0, n0, jb);
+                    if constexpr (PAIR) {
+                        // both CTAs' copies are counted on the leader's full barrier
+                        const uint32_t fl = peer_addr(fb, 0);
+                        if (rank == 0) mbar_arrive_expect_tx(fb, 2 * Cfg::STAGE);
+                        tma_load_3d_pair(st, &tmA, fl, k0, m0, ia);
+                        tma_load_3d_pair(st + Cfg::A_TILE, &tmB, fl, k0, n0 + (int)rank * Cfg::BH, jb);
+                    } else {
+                        mbar_arrive_expect_tx(fb, Cfg::STAGE);
+                        tma_load_3d(st, &tmA, fb, k0, m0, ia);
+                        tma_load_3d(st + Cfg::A_TILE, &tmB, fb, k0, n0, jb);
+                    }
                     if (++s == Cfg::STAGES) { s = 0; ph ^= 1u; }
                 }
             }
         }
-        if (!ok) drain_inflight(full0, Cfg::STAGES, L, flags);
-      } else if (warp == 1 && lane == 0) {
-        // ---------------- MMA issuer: one chunk partial into buffer t % NBUF
-        constexpr uint32_t idesc = make_idesc_bf16(kBM, Cfg::BN);
+        if (!ok) {
+            if (rank == 0) {
+                drain_inflight(full0, Cfg::STAGES, L, flags);
+            } else {
+                // the peer's copies complete on the leader's barriers, which it
+                // cannot observe: give them 200 us before the CTA winds down
+                const unsigned long long t0 = globaltimer_ns();
+                while (globaltimer_ns() - t0 < 200000ull) {}
+            }
+        }
+      } else if (warp == 1 && lane == 0 && rank == 0) {
+        // ---------------- MMA issuer (a pair's leader): one chunk partial into buffer t % NBUF
+        constexpr uint32_t idesc = make_idesc_bf16(PAIR ? 2 * kBM : kBM, Cfg::BN);
         int s = 0, b = 0;
         uint32_t ph = 0, tph = 0;
         bool ok = true;
@@ -169,15 +212,21 @@ prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                 for (int kk = 0; kk < Cfg::KB / 16; ++kk) {
                     const uint64_t ad = make_sdesc(st + kk * 32, Cfg::SBO, Cfg::SWZ);
                     const uint64_t bd = make_sdesc(st + Cfg::A_TILE + kk * 32, Cfg::SBO, Cfg::SWZ);
-                    mma_bf16(d, ad, bd, idesc, (u | kk) != 0);
+                    if constexpr (PAIR) mma_bf16_pair(d, ad, bd, idesc, (u | kk) != 0);
+                    else mma_bf16(d, ad, bd, idesc, (u | kk) != 0);
                 }
-                mma_commit(empty0 + 8u * s);
+                if constexpr (PAIR) mma_commit_pair(empty0 + 8u * s);
+                else mma_commit(empty0 + 8u * s);
                 if (++s == Cfg::STAGES) { s = 0; ph ^= 1u; }
             }
-            if (ok) mma_commit(tfull0 + 8u * b);
+            if (ok) {
+                if constexpr (PAIR) mma_commit_pair(tfull0 + 8u * b);
+                else mma_commit(tfull0 + 8u * b);
+            }
             if (++b == Cfg::NBUF) { b = 0; tph ^= 1u; }
         }
-        mma_commit(done_bar);
+        if constexpr (PAIR) mma_commit_pair(done_bar);
+        else mma_commit(done_bar);
         (void)mbar_wait(done_bar, 0, flags);
       }
     } else {
@@ -192,6 +241,9 @@ prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         const int lim = row < M ? N - (n0 + cq * Cfg::COLS) : 0;        // valid columns of this thread
         // this thread's elements of the tile's accumulator (column-major)
         double *tacc = acc + ((size_t)tm * tiles_n + tn) * Cfg::TILE_ELEMS + (size_t)(cq * Cfg::COLS) * kBM + r;
+        // a pair's second CTA may lie wholly below the last row, past the
+        // accumulator's tiles: its threads touch neither the accumulator nor C
+        const bool live = !PAIR || row < M;
         // the low words live in one half of this thread's C words until their product is reduced
         float *lrow = reinterpret_cast<float *>(crow);
         float hi[Cfg::COLS];
@@ -289,7 +341,10 @@ prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     if (h + 16 == Cfg::COLS) {                   // buffer free: all values are in registers
                         tc_fence_before();
                         __syncwarp();
-                        if (lane == 0) mbar_arrive(tempty0 + 8u * b);
+                        if (lane == 0) {
+                            if constexpr (PAIR) mbar_arrive_peer(peer_addr(tempty0 + 8u * b, 0));
+                            else mbar_arrive(tempty0 + 8u * b);
+                        }
                     }
                 }
             }
@@ -299,15 +354,17 @@ prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             // elements, 2^-24 bound; when that unit is a normal FP32 number so is
             // every nonzero sum, and the short widening is exact.
             const bool normal_sums = bound >= 0x1p-102f;
+            if (live) {
 #pragma unroll
-            for (int j = 0; j < Cfg::COLS; ++j) {
-                double sq = normal_sums ? widen_normal(hi[j]) : widen_exact(hi[j]);
-                if (((dirty >> (j >> 4)) & 1u) && j < lim) sq = __dadd_rn(sq, widen_exact(lrow[2 * j]));   // exact
-                if (q == 0) tacc[j * kBM] = sq;
-                else red_add_f64(tacc + j * kBM, sq);
+                for (int j = 0; j < Cfg::COLS; ++j) {
+                    double sq = normal_sums ? widen_normal(hi[j]) : widen_exact(hi[j]);
+                    if (((dirty >> (j >> 4)) & 1u) && j < lim) sq = __dadd_rn(sq, widen_exact(lrow[2 * j]));   // exact
+                    if (q == 0) tacc[j * kBM] = sq;
+                    else red_add_f64(tacc + j * kBM, sq);
+                }
             }
         }
-        if (ok) {
+        if (ok && live) {
             // the accumulator holds every product now (this thread's own reductions,
             // same addresses, so they precede these loads): C <- acc (+ the merged tail)
             const float *trow = TAIL ? T + (int64_t)(row < M ? row : 0) * ldt + n0 + cq * Cfg::COLS : nullptr;
@@ -336,32 +393,73 @@ prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     }
     tc_fence_before();
     __syncthreads();
+    if constexpr (PAIR) cluster_sync();               // the leader's MMAs are done with both CTAs
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
-        tmem_dealloc(tmem, 512);
+        if constexpr (PAIR) tmem_dealloc_pair(tmem, 512);
+        else tmem_dealloc(tmem, 512);
     }
 }
 
-// ctas: the first ctas tiles in raster order (all of them, or the full waves
-// when the narrow kernel takes the rest).
-template <int NPROD, bool ROWCOL, bool TAIL>
+// tiles: the first `tiles` tiles in raster order (all of them, or the full
+// waves when the narrow kernel takes the rest): 128 x 256 tiles, one CTA
+// each, or with PAIR 256 x 256 tiles, one cluster of two CTAs each.
+template <int NPROD, bool ROWCOL, bool TAIL, bool PAIR>
 cudaError_t run_f64w(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
                      const int32_t *vA, const int32_t *vB, double *C, int64_t ldc, double *acc, uint32_t *flags,
-                     cudaStream_t st, int64_t a_plane, const float *T, int64_t ldt, int64_t ctas)
+                     cudaStream_t st, int64_t a_plane, const float *T, int64_t ldt, int64_t tiles)
 {
-    using Cfg = F64WCfg;
+    using Cfg = F64WCfgT<PAIR>;
     CUtensorMap ta, tb;
     if (!make_plane_map(&ta, Ap, K, M, 6, ldcomp, Cfg::KB, kBM, a_plane) ||
-        !make_plane_map(&tb, Bp, K, N, 6, ldcomp, Cfg::KB, Cfg::BN))
+        !make_plane_map(&tb, Bp, K, N, 6, ldcomp, Cfg::KB, Cfg::BH))
         return cudaErrorInvalidValue;
-    auto kern = prodsum_f64w_kernel<NPROD, ROWCOL, TAIL>;
+    auto kern = prodsum_f64w_kernel<NPROD, ROWCOL, TAIL, PAIR>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
-    const int64_t tiles = ctas;
-    kern<<<(unsigned)tiles, Cfg::THREADS, Cfg::SMEM, st>>>(ta, tb, (int)M, (int)N, (int)K, vA, vB, C, ldc, acc, flags,
-                                                           T, ldt);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((PAIR ? 2 : 1) * tiles));
+    cfg.blockDim = dim3(Cfg::THREADS);
+    cfg.dynamicSmemBytes = Cfg::SMEM;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = PAIR ? 2 : 1;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = PAIR ? 1 : 0;
+    e = cudaLaunchKernelEx(&cfg, kern, ta, tb, (int)M, (int)N, (int)K, vA, vB, C, ldc, acc, flags, T, ldt);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
+}
+
+template <bool PAIR>
+cudaError_t dispatch_f64w(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
+                          const int32_t *vA, const int32_t *vB, int nprod, double *C, int64_t ldc, double *acc,
+                          uint32_t *flags, cudaStream_t st, int64_t a_plane, bool rowcol, const float *T, int64_t ldt,
+                          int64_t tiles)
+{
+#define EMU_F64W(NP, RC, TL) \
+    run_f64w<NP, RC, TL, PAIR>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, tiles)
+    if (T) {                                          // merged tail: whole-matrix levels only
+        if (rowcol) return cudaErrorInvalidValue;
+        switch (nprod) {
+        case 6: return EMU_F64W(6, false, true);
+        case 10: return EMU_F64W(10, false, true);
+        case 15: return EMU_F64W(15, false, true);
+        default: return cudaErrorInvalidValue;
+        }
+    }
+    switch (nprod) {
+    case 6: return rowcol ? EMU_F64W(6, true, false) : EMU_F64W(6, false, false);
+    case 10: return rowcol ? EMU_F64W(10, true, false) : EMU_F64W(10, false, false);
+    case 15: return rowcol ? EMU_F64W(15, true, false) : EMU_F64W(15, false, false);
+    case 21: return rowcol ? EMU_F64W(21, true, false) : EMU_F64W(21, false, false);
+    default: return cudaErrorInvalidValue;
+    }
+#undef EMU_F64W
 }
 
 }  // namespace
@@ -369,28 +467,12 @@ cudaError_t run_f64w(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const 
 cudaError_t launch_prodsum_f64_wide(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp,
                                     int64_t ldcomp, const int32_t *vA, const int32_t *vB, int nprod, double *C,
                                     int64_t ldc, double *acc, uint32_t *flags, cudaStream_t st, int64_t a_plane,
-                                    bool rowcol, const float *T, int64_t ldt, int64_t ctas)
+                                    bool rowcol, const float *T, int64_t ldt, int64_t tiles, bool pair)
 {
-    if (T) {                                          // merged tail: whole-matrix levels only
-        if (rowcol) return cudaErrorInvalidValue;
-        switch (nprod) {
-        case 6: return run_f64w<6, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, ctas);
-        case 10: return run_f64w<10, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, ctas);
-        case 15: return run_f64w<15, false, true>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, T, ldt, ctas);
-        default: return cudaErrorInvalidValue;
-        }
-    }
-    switch (nprod) {
-    case 6: return rowcol ? run_f64w<6, true, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas)
-                   : run_f64w<6, false, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas);
-    case 10: return rowcol ? run_f64w<10, true, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas)
-                   : run_f64w<10, false, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas);
-    case 15: return rowcol ? run_f64w<15, true, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas)
-                   : run_f64w<15, false, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas);
-    case 21: return rowcol ? run_f64w<21, true, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas)
-                   : run_f64w<21, false, false>(M, N, K, Ap, Bp, ldcomp, vA, vB, C, ldc, acc, flags, st, a_plane, nullptr, 0, ctas);
-    default: return cudaErrorInvalidValue;
-    }
+    return pair ? dispatch_f64w<true>(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane, rowcol,
+                                      T, ldt, tiles)
+                : dispatch_f64w<false>(M, N, K, Ap, Bp, ldcomp, vA, vB, nprod, C, ldc, acc, flags, st, a_plane, rowcol,
+                                       T, ldt, tiles);
 }
 
 }  // namespace emu

@@ -142,4 +142,15 @@ def test_f64_tile_width_report(lib):
     assert emu.emu_prodsum_f64_tile_columns(8192, 8192) == 256
     assert emu.emu_prodsum_f64_tile_columns(1024, 1024) == 128
     assert emu.emu_prodsum_f64_tile_columns(0, 8) == 0
+    # 256-column tiles run on CTA pairs (256 rows) when there are two tile rows
+    assert emu.emu_prodsum_f64_tile_rows(8192, 8192) == 256
+    assert emu.emu_prodsum_f64_tile_rows(1024, 1024) == 128
+    assert emu.emu_prodsum_f64_tile_rows(128, 65536) == 128
+    assert emu.emu_prodsum_f64_tile_rows(8, 0) == 0
+    # 8192^2: 1024 pair tiles on 76 pairs, 13.5 waves, one launch; 4096^2:
+    # 256 pair tiles, 3.4 waves, the last 28 tiles as 112 128 x 128 tiles
+    assert emu.emu_prodsum_f64_launches(8192, 8192) == 1
+    assert emu.emu_prodsum_f64_launches(4096, 4096) == 2
+    assert emu.emu_prodsum_f64_launches(1024, 1024) == 1
+    assert emu.emu_prodsum_f64_launches(0, 1) == 0
 

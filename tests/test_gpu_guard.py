@@ -107,8 +107,8 @@ def test_gemm_f64_guard_bands(M, N, K, nprod):
     if M * N * K * nprod <= 4e9:
         assert np.array_equal(Cn, oracle.gemm_f64(A, B, nprod)[0])
     else:
-        # the 128 x 256 kernel at a ragged size: sampled rows against the oracle
-        assert emu.emu_prodsum_f64_tile_columns(M, N) == 256
+        # 256 x 256 tiles on CTA pairs at a ragged size: sampled rows against the oracle
+        assert emu.emu_prodsum_f64_tile_columns(M, N) == 256 and emu.emu_prodsum_f64_tile_rows(M, N) == 256
         for r in sample_rows(M, 4, 5):
             assert np.array_equal(Cn[r], oracle.gemm_f64(A, B, nprod, rows=(r, r + 1))[0][0]), r
 

@@ -65,16 +65,18 @@ def digest(tag, C):
     print("digest", tag, hashlib.sha256(C.tobytes()).hexdigest())
 
 # whole-matrix levels, Algorithm 2: ragged tiles, tiny and multi-chunk K, every product count
+# (with 256 x 256 tiles on CTA pairs: 300 rows leave the second CTA of the
+# last pair below the matrix, 129 rows leave it one row, 100 rows need no pair)
 for M, N, K, seed, nprod in [(300, 333, 700, 1, 21), (129, 257, 33, 3, 6), (256, 512, 1024, 8, 10),
-                             (520, 130, 300, 5, 15)]:
+                             (520, 130, 300, 5, 15), (100, 600, 500, 9, 6)]:
     A, B = synth.gemm_inputs("f64", M, N, K, seed)
     C, ws = emu.gemm_f64(to_dev(A, dev), to_dev(B, dev), nprod)
     assert emu.read_flags(ws) == 0
     Cn = C.cpu().numpy()
     assert np.array_equal(Cn, oracle.gemm_f64(A, B, nprod)[0]), (M, N, K, nprod)
     digest((M, N, K, nprod), Cn)
-# a 4096 x 4096 result: 3.4 waves of 128 x 256 tiles, so by default the full
-# waves run wide and the last tiles as 128 x 128 halves
+# a 4096 x 4096 result: 3.4 waves of 256 x 256 tiles on CTA pairs, so by
+# default the full waves run as pairs and the last tiles as 128 x 128 parts
 A, B = synth.gemm_inputs("f64", 4096, 4096, 264, 14)
 C, ws = emu.gemm_f64(to_dev(A, dev), to_dev(B, dev), 10)
 assert emu.read_flags(ws) == 0
@@ -119,13 +121,13 @@ def _run64(tile):
 
 
 def test_f64_tile_shapes_parity_and_bit_identity():
-    """The FP64 product-sum's tile shapes (EMU_F64_TILE=128x128 / 128x256):
-    both form the same exact per-product sums and add them in Algorithm 2's
-    order, so C must equal the oracle bit for bit with either shape, and with
-    the default schedule that runs the last partial wave of wide tiles as
-    narrow ones, through the plain, carry, per-row/column and merged-tail
-    paths."""
+    """The FP64 product-sum's tile shapes (EMU_F64_TILE=128x128 / 128x256 /
+    256x256, the last on CTA pairs): all form the same exact per-product sums
+    and add them in Algorithm 2's order, so C must equal the oracle bit for bit
+    with any shape, and with the default schedule that runs the last partial
+    wave of 256-column tiles as 128 x 128 ones, through the plain, carry,
+    per-row/column and merged-tail paths."""
     ref = _run64(None)
-    assert len(ref) == 8
-    for tile in ("128x256", "128x128"):
+    assert len(ref) == 9
+    for tile in ("256x256", "128x256", "128x128"):
         assert _run64(tile) == ref, tile
