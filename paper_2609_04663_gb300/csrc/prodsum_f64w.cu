@@ -1,12 +1,20 @@
-// FP64-mode tensor-core product-sum on 128 x 256 output tiles, Eq.
+// FP64-mode tensor-core product-sum on 256-column output tiles, Eq.
 // (fp64reconstruction) / Algorithm 2: the same arithmetic as the 128 x 128
-// kernel (prodsum_f64.cu), bit for bit, with twice the output columns per CTA.
+// kernel (prodsum_f64.cu), bit for bit, with twice the output columns per CTA,
+// and optionally (PAIR) twice the rows per MMA on a pair of SMs.
 //
 // Why wider: every MMA brings its A and B operands into the SM through shared
 // memory, and for one product at a time nothing is reused across MMAs.  A
 // 128 x 256 x 16 MMA takes in 12 KB of operands for 2^20 FLOP, a 128 x 128 x 16
 // one 8 KB for 2^19, so this tile moves 0.75x the bytes per FLOP, the quantity
-// that bounds the narrower kernel.
+// that bounds the narrower kernel.  With PAIR a cluster of two CTAs on one TPC
+// computes a 256 x 256 tile with cta_group::2 MMAs (M = 256): each CTA stages
+// its 128 rows of the A slice and half of the B slice's 256 rows, the leader
+// (cluster rank 0) issues the MMAs for both, and each CTA's TMEM receives its
+// 128 x 256 part of the partials; per SM that is 8 KB of operands per 2^20
+// FLOP.  Both CTAs' copies complete on the leader's stage barriers, the MMA
+// commits arrive on both CTAs' barriers (multicast), and both CTAs' drain
+// warps release a TMEM buffer on the leader's barrier.
 //
 // Products are taken in Algorithm 2's diagonal order (outer loop); for each
 // product K is walked in chunks of 256 (B_K of Section 6.1), every chunk
@@ -38,9 +46,10 @@
 // product-outer order.
 //
 // Warp roles: warp 0 lane 0 issues TMA loads (four 48 KB stages, one 64-wide
-// K-block of the A slice and the B slice each), warp 1 owns TMEM and lane 0
-// issues the MMAs (M = 128, N = 256), warps 4-19 drain and reduce.  Every wait
-// is bounded and reports EMU_FLAG_TIMEOUT instead of hanging.
+// K-block of the A slice and the B slice each; PAIR: six 32 KB stages), warp
+// 1 owns TMEM and lane 0 issues the MMAs (M = 128, N = 256; PAIR: the
+// leader's, M = 256), warps 4-19 drain and reduce.  Every wait is bounded and
+// reports EMU_FLAG_TIMEOUT instead of hanging.
 #include "launchers.cuh"
 #include "prodsum_f64_common.cuh"
 
