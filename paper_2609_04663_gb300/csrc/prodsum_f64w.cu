@@ -362,8 +362,21 @@ prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             // The sums are integer multiples of the smallest unit of this thread's
             // elements, 2^-24 bound; when that unit is a normal FP32 number so is
             // every nonzero sum, and the short widening is exact.
+            // The common case (no low words, normal unit) is a branch of its own
+            // with integer widening only: written as selects, the rare path's
+            // FP64 additions and general widening would run for every element
+            // (GB300's FP64 pipe does about one warp-wide add per 32 clocks per
+            // SM sub-partition).
             const bool normal_sums = bound >= 0x1p-102f;
-            if (live) {
+            if (live && dirty == 0 && normal_sums) {
+                if (q == 0) {
+#pragma unroll
+                    for (int j = 0; j < Cfg::COLS; ++j) tacc[j * kBM] = widen_normal(hi[j]);
+                } else {
+#pragma unroll
+                    for (int j = 0; j < Cfg::COLS; ++j) red_add_f64(tacc + j * kBM, widen_normal(hi[j]));
+                }
+            } else if (live) {
 #pragma unroll
                 for (int j = 0; j < Cfg::COLS; ++j) {
                     double sq = normal_sums ? widen_normal(hi[j]) : widen_exact(hi[j]);
