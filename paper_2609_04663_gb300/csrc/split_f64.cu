@@ -107,21 +107,23 @@ __device__ __forceinline__ void f64_spec_transpose_body(const double *__restrict
     const bool vin = ((ldx & 1) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
     const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
     const int q = threadIdx.x >> 5, p = lane_id();
+    const int rp = 4 * q + (p >> 3), cg = p & 7;       // rows 2rp, 2rp + 1; columns 16j + 2cg + {0, 1}
     const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
     SpecState st;
-    // this thread's two entries of column pair k of tile t's rows 2p, 2p + 1
-    auto load = [&](int64_t t, int k, double (&x)[2][2]) {
-        const int64_t r0 = (t / tiles_c) * kTile, gj = (t % tiles_c) * kTile + 8 * q;
+    // this thread's two entries in step j of tile t: eight lanes read 128
+    // contiguous bytes of one row
+    auto load = [&](int64_t t, int j, double (&x)[2][2]) {
+        const int64_t r0 = (t / tiles_c) * kTile, gj = (t % tiles_c) * kTile + 16 * j + 2 * cg;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-            const int64_t gi = r0 + 2 * p + h;
-            const double *src = X + gi * ldx + gj + k;
-            if (gi < rows && vin && gj + 8 <= cols) {
+            const int64_t gi = r0 + 2 * rp + h;
+            const double *src = X + gi * ldx + gj;
+            if (gi < rows && vin && gj + 2 <= cols) {
                 const double2 a = *reinterpret_cast<const double2 *>(src);
                 x[h][0] = a.x; x[h][1] = a.y;
             } else {
 #pragma unroll
-                for (int e = 0; e < 2; ++e) x[h][e] = (gi < rows && gj + k + e < cols) ? src[e] : 0.0;
+                for (int e = 0; e < 2; ++e) x[h][e] = (gi < rows && gj + e < cols) ? src[e] : 0.0;
             }
         }
     };
@@ -133,19 +135,22 @@ __device__ __forceinline__ void f64_spec_transpose_body(const double *__restrict
         // the element body appears four times in the loop, not sixteen; the
         // next step's entries are loaded before this step is split
 #pragma unroll 1
-        for (int k = 0; k < 8; k += 2) {
+        for (int j = 0; j < 4; ++j) {
             double x[2][2];
 #pragma unroll
             for (int h = 0; h < 2; ++h) { x[h][0] = xn[h][0]; x[h][1] = xn[h][1]; }
-            if (k + 2 < 8) load(t, k + 2, xn);
+            if (j + 1 < 4) load(t, j + 1, xn);
             else if (t + nblk < tiles_r * tiles_c) load(t + nblk, 0, xn);
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
                 uint32_t s0[6], s1[6];
                 spec_element<NLEV>(x[0][e], v0, fast, P, s0, st);
                 spec_element<NLEV>(x[1][e], v0, fast, P, s1, st);
+                // transposed row col, K-chunk rp / 4 stored at chunk (rp / 4) ^ cg: conflict-free
+                const int col = 16 * j + 2 * cg + e;
 #pragma unroll
-                for (int r = 0; r < NLEV; ++r) smw[(r * kTile + 8 * q + k + e) * (kTile / 2) + p] = pack2(s0[r], s1[r]);
+                for (int r = 0; r < NLEV; ++r)
+                    smw[(r * kTile + col) * (kTile / 2) + (((q ^ cg) << 2) | (p >> 3))] = pack2(s0[r], s1[r]);
             }
         }
         __syncthreads();
@@ -156,7 +161,7 @@ __device__ __forceinline__ void f64_spec_transpose_body(const double *__restrict
             const int r = c >> 9, orow = (c >> 3) & 63, ch = c & 7;
             const int64_t go = c0 + orow, gk = r0 + 8 * ch;
             if (go < cols && gk < rows) {
-                const uint4 v = *reinterpret_cast<const uint4 *>(&smw[(r * kTile + orow) * (kTile / 2) + 4 * ch]);
+                const uint4 v = *reinterpret_cast<const uint4 *>(&smw[(r * kTile + orow) * (kTile / 2) + 4 * (ch ^ ((orow >> 1) & 7))]);
                 uint16_t *dst = comps + r * plane + go * ldcomp + gk;
                 if (vout && gk + 8 <= rows) {
                     *reinterpret_cast<uint4 *>(dst) = v;
