@@ -64,11 +64,13 @@ split_f32_rows_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, i
                                           gridDim.y), &ws->flags);
 }
 
-// Transposed (K-major) planes: a 64 x 64 tile of X.  Warp q takes columns
-// 8q .. 8q+7, lane p rows 2p and 2p+1, so each slice word packs the two
-// elements that are adjacent in the transposed row; the words go to shared
-// memory (one bank per lane: conflict-free) and leave as 16-byte chunks of
-// whole transposed rows.
+// Transposed (K-major) planes: a 64 x 64 tile of X.  Lane p of warp q takes
+// rows 2rp and 2rp+1 (rp = 4q + p / 8) and columns 32j + 4(p % 8) + {0..3},
+// j = 0, 1, so eight lanes read 128 contiguous bytes of a row and each slice
+// word packs the two elements that are adjacent in the transposed row; the
+// words go to shared memory, each transposed row's 16-byte K-chunks permuted
+// by an XOR with its column (so a warp's stores hit 32 different banks), and
+// leave as 16-byte chunks of whole transposed rows.
 // Block bid of nblk blocks (tiles taken with a stride of nblk); sm: the
 // block's [3][kTile][kTile / 2] staging words.  Returns the block's part of
 // the flag check, as the row body does.
@@ -80,22 +82,27 @@ __device__ __forceinline__ uint32_t split_f32_transpose_body(const float *__rest
     const bool vin = ((ldx & 3) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
     const bool vout = ((ldcomp & 7) == 0) && ((plane & 7) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 15u) == 0);
     const int q = threadIdx.x >> 5, p = lane_id();
+    const int rp = 4 * q + (p >> 3), cg = p & 7;       // rows 2rp, 2rp + 1; columns 32j + 4cg + {0..3}
     const int64_t tiles_r = (rows + kTile - 1) / kTile, tiles_c = (cols + kTile - 1) / kTile;
     // the next tile's rows are loaded before this tile is split and stored,
-    // so that the loads of a block overlap its own stores
+    // so that the loads of a block overlap its own stores; eight lanes read
+    // 128 contiguous bytes of one row
     auto load_tile = [&](int64_t t, float (&x)[2][8]) {
-        const int64_t r0 = (t / tiles_c) * kTile, gj = (t % tiles_c) * kTile + 8 * q;
+        const int64_t r0 = (t / tiles_c) * kTile, c0 = (t % tiles_c) * kTile;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-            const int64_t gi = r0 + 2 * p + h;
-            const float *src = X + gi * ldx + gj;
-            if (gi < rows && vin && gj + 8 <= cols) {
-                const float4 a = reinterpret_cast<const float4 *>(src)[0], b = reinterpret_cast<const float4 *>(src)[1];
-                x[h][0] = a.x; x[h][1] = a.y; x[h][2] = a.z; x[h][3] = a.w;
-                x[h][4] = b.x; x[h][5] = b.y; x[h][6] = b.z; x[h][7] = b.w;
-            } else {
+            const int64_t gi = r0 + 2 * rp + h;
 #pragma unroll
-                for (int e = 0; e < 8; ++e) x[h][e] = (gi < rows && gj + e < cols) ? src[e] : 0.0f;
+            for (int j = 0; j < 2; ++j) {
+                const int64_t gj = c0 + 32 * j + 4 * cg;
+                const float *src = X + gi * ldx + gj;
+                if (gi < rows && vin && gj + 4 <= cols) {
+                    const float4 a = *reinterpret_cast<const float4 *>(src);
+                    x[h][4 * j] = a.x; x[h][4 * j + 1] = a.y; x[h][4 * j + 2] = a.z; x[h][4 * j + 3] = a.w;
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) x[h][4 * j + e] = (gi < rows && gj + e < cols) ? src[e] : 0.0f;
+                }
             }
         }
     };
@@ -111,9 +118,11 @@ __device__ __forceinline__ uint32_t split_f32_transpose_body(const float *__rest
             amax = abs_bits_max(amax, x[0][e], x[1][e]);
             uint32_t w0, w1, w2;
             split_pair(x[0][e], x[1][e], w0, w1, w2);
-            sm[0][8 * q + e][p] = w0;
-            sm[1][8 * q + e][p] = w1;
-            sm[2][8 * q + e][p] = w2;
+            // transposed row col, K-chunk rp / 4 stored at chunk (rp / 4) ^ cg: conflict-free
+            const int col = 32 * (e >> 2) + 4 * cg + (e & 3), w = ((q ^ cg) << 2) | (p >> 3);
+            sm[0][col][w] = w0;
+            sm[1][col][w] = w1;
+            sm[2][col][w] = w2;
         }
         __syncthreads();
         // 3 planes x 64 transposed rows x 8 chunks of 16 bytes
@@ -123,7 +132,7 @@ __device__ __forceinline__ uint32_t split_f32_transpose_body(const float *__rest
             const int r = c >> 9, orow = (c >> 3) & 63, ch = c & 7;
             const int64_t go = c0 + orow, gk = r0 + 8 * ch;
             if (go < cols && gk < rows) {
-                const uint4 v = *reinterpret_cast<const uint4 *>(&sm[r][orow][4 * ch]);
+                const uint4 v = *reinterpret_cast<const uint4 *>(&sm[r][orow][4 * (ch ^ ((orow >> 2) & 7))]);
                 uint16_t *dst = comps + r * plane + go * ldcomp + gk;
                 if (vout && gk + 8 <= rows) {
                     *reinterpret_cast<uint4 *>(dst) = v;

@@ -88,9 +88,12 @@ f64_spec_rows_kernel(const double *__restrict__ X, int64_t rows, int64_t cols, i
     f64_spec_rows_body<NLEV>(X, rows, cols, ldx, comps, ldcomp, plane, ws, slot, blockIdx.x, blockIdx.y, gridDim.y, red);
 }
 
-// Transposed (K-major) planes: a 64 x 64 tile, warp q on columns 8q .. 8q+7,
-// lane p on rows 2p and 2p+1; each plane word packs the two entries adjacent
-// in the transposed row, staged one bank per lane and written as 16-byte
+// Transposed (K-major) planes: a 64 x 64 tile; lane p of warp q takes rows
+// 2rp and 2rp+1 (rp = 4q + p / 8) and columns 16j + 2(p % 8) + {0, 1},
+// j = 0..3, so eight lanes read 128 contiguous bytes of a row.  Each plane
+// word packs the two entries adjacent in the transposed row; it is staged
+// with each transposed row's 16-byte K-chunks permuted by an XOR with the
+// column (a warp's stores hit 32 different banks) and written as 16-byte
 // chunks of whole transposed rows.  Shared memory: [6][64][32] words.
 // Block bid of nblk (tiles with a stride of nblk); smw: [6][kTile][kTile / 2]
 // words, red: 5 * kThreads / 32 words of shared memory.
