@@ -409,8 +409,8 @@ __device__ __forceinline__ void f64_max_pass(const double *__restrict__ X, int64
     unsigned long long m = 0;
     uint32_t flagbits = 0;
     const int64_t segs = (cols + 4 * kThreads - 1) / (4 * kThreads);
-    for (int64_t it = bid; it < rows * segs; it += nblk) {
-        const int64_t i = it / segs, j0 = (it % segs) * (4 * kThreads) + 4 * threadIdx.x;
+    // four entries of row i from column j0 on
+    auto body = [&](int64_t i, int64_t j0) {
         const double *src = X + i * ldx + j0;
         double x[4];
         if (j0 + 4 <= cols && ((reinterpret_cast<uintptr_t>(src) & 15u) == 0)) {
@@ -438,6 +438,18 @@ __device__ __forceinline__ void f64_max_pass(const double *__restrict__ X, int64
                 m = ab > m ? ab : m;
             }
         }
+    };
+    if (nblk >= segs) {
+        // block bid walks rows bid / segs, + rstride, ... of column segment
+        // bid % segs (no division in the loop); blocks past rstride * segs idle
+        const int64_t rstride = nblk / segs;
+        if (bid < rstride * segs) {
+            const int64_t j0 = (bid % segs) * (4 * kThreads) + 4 * threadIdx.x;
+#pragma unroll 2
+            for (int64_t i = bid / segs; i < rows; i += rstride) body(i, j0);
+        }
+    } else {
+        for (int64_t it = bid; it < rows * segs; it += nblk) body(it / segs, (it % segs) * (4 * kThreads) + 4 * threadIdx.x);
     }
     if constexpr (LEVEL == 0) {
         flagbits = __reduce_or_sync(0xFFFFFFFFu, flagbits);
