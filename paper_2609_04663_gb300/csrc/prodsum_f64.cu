@@ -369,13 +369,26 @@ prodsum_f64_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                 asm volatile("ld.shared.u8 %0, [%1];" : "=r"(mask) : "r"(hmask + (uint32_t)(r * 4 + (col >> 5))) : "memory");
                 const bool dg = (mask >> ((col >> 4) & 1)) & 1u;   // 16-column group of these 8 columns
                 tmem_ld_wait();
+                // the common case (no low words, not the first product) is a
+                // branch of its own: written as selects, the rare cases' FP64
+                // additions would run for every element (GB300's FP64 pipe does
+                // about one warp-wide add per 32 clocks per sub-partition)
                 double out[8];
+                if (!dg && !first) {
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    double sq = widen_exact(__uint_as_float(hv[j]));
-                    if (dg && col + j < lim) sq = __dadd_rn(sq, widen_exact(lrow[2 * (col + j)]));   // exact
-                    out[j] = first ? sq : __dadd_rn(cur[j], sq);
-                    if (TAIL && last && col + j < lim) out[j] = __dadd_rn(out[j], widen_exact(trow[col + j]));
+                    for (int j = 0; j < 8; ++j) out[j] = __dadd_rn(cur[j], widen_exact(__uint_as_float(hv[j])));
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        double sq = widen_exact(__uint_as_float(hv[j]));
+                        if (dg && col + j < lim) sq = __dadd_rn(sq, widen_exact(lrow[2 * (col + j)]));   // exact
+                        out[j] = first ? sq : __dadd_rn(cur[j], sq);
+                    }
+                }
+                if (TAIL && last) {
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        if (col + j < lim) out[j] = __dadd_rn(out[j], widen_exact(trow[col + j]));
                 }
                 if (!last) {
 #pragma unroll
