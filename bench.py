@@ -542,7 +542,9 @@ def variants(args, rank, world, pk):
         merge_from = nprod[1] if isinstance(nprod, tuple) else None
         nprod = nprod[0] if isinstance(nprod, tuple) else None if fused or api else nprod
         case = Case(name, rank, nprod, fused=fused, merge_from=merge_from, api=api)
-        res = time_device(case, max(3, args.variant_steps), 2, world, flush=True)
+        # steps of a few microseconds vary by some microseconds: many more of them
+        steps = 50 if case.flop < 2e11 else max(3, args.variant_steps)
+        res = time_device(case, steps, 5 if case.flop < 2e11 else 2, world, flush=True)
         t = max_over_ranks(sum(res["step_ms"]) / 1e3, world)
         pm = statistics.mean(res["prodsum_ms"])
         key = f"{name}" + (f"_np{case.nprod}" if case.mode == 64 else "_fused" if fused else "_gemm" if api else "") + \

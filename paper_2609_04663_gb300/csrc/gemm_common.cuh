@@ -107,4 +107,24 @@ inline bool make_plane_map(CUtensorMap *map, const uint16_t *planes, int64_t K, 
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Tensor map over an FP32 matrix C [M][ldc] for 32 x 32 boxes (128-byte rows,
+// 128-byte swizzle), the unit of the product-sum's reduction epilogue.
+// False when C cannot be described (base not 16-byte aligned, row pitch not
+// a multiple of 16 bytes) or when N is not a multiple of 4: a bulk tensor
+// reduction clips a box at the end of a row only to whole 16-byte pieces
+// (on GB300 a box over columns 320-351 of a 333-column C also wrote columns
+// 333-335), which would reach into the padding of C.
+inline bool make_c_map_f32(CUtensorMap *map, float *C, int64_t M, int64_t N, int64_t ldc)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc || (reinterpret_cast<uintptr_t>(C) & 15u) != 0 || (ldc & 3) != 0 || (N & 3) != 0) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)N, (cuuint64_t)M};
+    cuuint64_t strides[1] = {(cuuint64_t)ldc * 4};
+    cuuint32_t box[2] = {32, 32};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, C, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace emu

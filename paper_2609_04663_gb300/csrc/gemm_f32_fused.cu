@@ -38,20 +38,6 @@ namespace {
 // and leave the tensor pipe idle 28 % of the time.
 constexpr int kFusedPrefetch = 4;        // K-blocks between the L2 prefetch and the loads
 
-__device__ __forceinline__ void st_shared_v2(uint32_t addr, uint32_t a, uint32_t b)
-{
-    asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
-}
-__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d)
-{
-    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
-}
-// Makes this thread's shared-memory stores visible to the tensor cores
-// (async proxy) before it signals the stage as full.
-__device__ __forceinline__ void fence_proxy_async_smem()
-{
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
 __device__ __forceinline__ void prefetch_l2(const void *p)
 {
     asm volatile("prefetch.global.L2 [%0];" ::"l"(p));

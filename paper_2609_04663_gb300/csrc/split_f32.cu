@@ -56,6 +56,72 @@ __device__ __forceinline__ uint32_t split_f32_rows_body(const float *__restrict_
     return amax;
 }
 
+// Row-major planes by 64 x 64 tiles (the GEMM's one-launch split of A):
+// thread t takes rows t / 16 + 16 i (i = 0..3) and columns 4 (t % 16) .. + 3
+// of a tile, so a warp reads two whole 256-byte row segments per load and
+// writes 128 contiguous bytes of two plane rows per store; the next tile's
+// entries are loaded before this tile is split and stored, so every thread
+// has four to eight 16-byte loads in flight.  Block bid of nblk (tiles with a
+// stride of nblk).  Returns the block's part of the flag check.
+__device__ __forceinline__ uint32_t split_f32_rowtile_body(const float *__restrict__ X, int64_t rows, int64_t cols,
+                                                       int64_t ldx, uint16_t *__restrict__ comps, int64_t ldcomp,
+                                                       int64_t plane, int64_t bid, int64_t nblk)
+{
+    const bool vin = ((ldx & 3) == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
+    const bool vout = ((ldcomp & 3) == 0) && ((plane & 3) == 0) && ((reinterpret_cast<uintptr_t>(comps) & 7u) == 0);
+    const int tr = threadIdx.x >> 4, tc = 4 * (threadIdx.x & 15);
+    const int64_t tiles_c = (cols + kTile - 1) / kTile, ntiles = ((rows + kTile - 1) / kTile) * tiles_c;
+    auto load_tile = [&](int64_t t, float (&x)[4][4]) {
+        const int64_t r0 = (t / tiles_c) * kTile, gj = (t % tiles_c) * kTile + tc;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int64_t gi = r0 + tr + 16 * i;
+            const float *src = X + gi * ldx + gj;
+            if (gi < rows && vin && gj + 4 <= cols) {
+                const float4 a = *reinterpret_cast<const float4 *>(src);
+                x[i][0] = a.x; x[i][1] = a.y; x[i][2] = a.z; x[i][3] = a.w;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) x[i][e] = (gi < rows && gj + e < cols) ? src[e] : 0.0f;
+            }
+        }
+    };
+    uint32_t amax = 0;
+    float x[4][4];
+    if (bid < ntiles) load_tile(bid, x);
+    for (int64_t t = bid; t < ntiles; t += nblk) {
+        float xn[4][4];
+        if (t + nblk < ntiles) load_tile(t + nblk, xn);
+        const int64_t r0 = (t / tiles_c) * kTile, gj = (t % tiles_c) * kTile + tc;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int64_t gi = r0 + tr + 16 * i;
+            uint32_t w[3][2];
+            amax = abs_bits_max(abs_bits_max(amax, x[i][0], x[i][1]), x[i][2], x[i][3]);
+            split_pair(x[i][0], x[i][1], w[0][0], w[1][0], w[2][0]);
+            split_pair(x[i][2], x[i][3], w[0][1], w[1][1], w[2][1]);
+            if (gi < rows) {
+                uint16_t *dst = comps + gi * ldcomp + gj;
+#pragma unroll
+                for (int r = 0; r < 3; ++r) {
+                    if (vout && gj + 4 <= cols) {
+                        *reinterpret_cast<uint2 *>(dst + r * plane) = make_uint2(w[r][0], w[r][1]);
+                    } else {
+#pragma unroll
+                        for (int e = 0; e < 4; ++e)
+                            if (gj + e < cols) dst[r * plane + e] = (uint16_t)(w[r][e >> 1] >> (16 * (e & 1)));
+                    }
+                }
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) x[i][e] = xn[i][e];
+    }
+    return amax;
+}
+
 __global__ void __launch_bounds__(kThreads)
 split_f32_rows_kernel(const float *__restrict__ X, int64_t rows, int64_t cols, int64_t ldx,
                       uint16_t *__restrict__ comps, int64_t ldcomp, int64_t plane, WsHeader *ws)
@@ -163,29 +229,44 @@ split_f32_transpose_kernel(const float *__restrict__ X, int64_t rows, int64_t co
 }
 
 // Both operands of an FP32 GEMM in one launch: blocks [0, nA) split A into
-// row-major planes (nA = ax * ay blocks as the row kernel's grid), blocks
-// [nA, nA + nB) split B into K-major planes, and blocks from nA + nB on set
-// the M x N result C to zero (a product-sum that adds its K-parts into C
-// needs it cleared).
+// row-major planes (by rows on an ax x (nA / ax) grid when ax > 0, else by
+// 64 x 64 tiles), blocks [nA, nA + nB) split B into K-major planes, and
+// blocks from nA + nB on set the M x N result C to zero (a product-sum that
+// adds its K-parts into C needs it cleared).
 __global__ void __launch_bounds__(kThreads)
 split_f32_gemm_kernel(const float *__restrict__ A, int64_t M, int64_t K, int64_t lda, const float *__restrict__ B,
                       int64_t N, int64_t ldb, uint16_t *__restrict__ Ap, uint16_t *__restrict__ Bp, int64_t ldcomp,
-                      WsHeader *ws, int64_t ax, int64_t ay, int64_t nB, float *__restrict__ C, int64_t ldc,
-                      int64_t nC)
+                      WsHeader *ws, int64_t ax, int64_t nA, int64_t nB, float *__restrict__ C, int64_t ldc, int64_t nC)
 {
     __shared__ __align__(16) uint32_t sm[3][kTile][kTile / 2];
-    const int64_t b = blockIdx.x, nA = ax * ay;
+    // the product-sum launched after this kernel may start its set-up as soon
+    // as every block of this one is running (it waits for all of it before
+    // reading planes or C)
+    griddep_launch_dependents();
+    const int64_t b = blockIdx.x;
     if (b < nA + nB) {
-        const uint32_t amax = b < nA ? split_f32_rows_body(A, M, K, lda, Ap, ldcomp, M * ldcomp, ws, b % ax, b / ax, ay)
-                                     : split_f32_transpose_body(B, K, N, ldb, Bp, ldcomp, N * ldcomp, ws, b - nA, nB, sm);
+        const uint32_t amax =
+            b >= nA ? split_f32_transpose_body(B, K, N, ldb, Bp, ldcomp, N * ldcomp, ws, b - nA, nB, sm)
+            : ax > 0 ? split_f32_rows_body(A, M, K, lda, Ap, ldcomp, M * ldcomp, ws, b % ax, b / ax, nA / ax)
+                     : split_f32_rowtile_body(A, M, K, lda, Ap, ldcomp, M * ldcomp, b, nA);
         // the flag word is cleared by the operation before this launch, which
         // may still be running when this kernel is its programmatic dependent
         griddep_wait();
         publish_f32_flags(amax, &ws->flags);
     } else {
         const int64_t c = b - nA - nB;
-        for (int64_t i = c; i < M; i += nC)
-            for (int64_t j = threadIdx.x; j < N; j += kThreads) C[i * ldc + j] = 0.0f;
+        const bool vec = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15u) == 0);
+        for (int64_t i = c; i < M; i += nC) {
+            float *row = C + i * ldc;
+            if (vec) {
+                for (int64_t j = 4 * (int64_t)threadIdx.x; j < N; j += 4 * kThreads) {
+                    if (j + 4 <= N) *reinterpret_cast<float4 *>(row + j) = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+                    else for (int64_t e = j; e < N; ++e) row[e] = 0.0f;
+                }
+            } else {
+                for (int64_t j = threadIdx.x; j < N; j += kThreads) row[j] = 0.0f;
+            }
+        }
     }
 }
 
@@ -218,16 +299,29 @@ cudaError_t launch_split_f32_gemm(const float *A, int64_t M, int64_t K, int64_t 
                                   int64_t ldc, cudaStream_t st)
 {
     if (M == 0 || N == 0 || K == 0) return cudaSuccess;
-    const int64_t ax = (K + 8 * kThreads - 1) / (8 * kThreads);
-    const int64_t want = (152 * 4 + ax - 1) / ax;
-    const int64_t ay = M < want ? M : want;
-    const int64_t tiles = ((K + kTile - 1) / kTile) * ((N + kTile - 1) / kTile);
-    const int64_t nB = grid_for(tiles, 152 * 4);
-    const int64_t nC = C ? (M < 152 ? M : 152) : 0;
+    // Operands of at most 256 tiles of 64 x 64 each: one block per tile, A by
+    // tiles too, and at most 96 blocks clearing C, so that the launch is one
+    // wave (608 blocks: four 256-thread blocks per SM at the kernel's 64
+    // registers) and its time one round trip to DRAM.  Larger operands: rows
+    // of A on 608 blocks, 608 blocks of B tiles (measured faster there).
+    const int64_t tiles_a = ((M + kTile - 1) / kTile) * ((K + kTile - 1) / kTile);
+    const int64_t tiles_b = ((K + kTile - 1) / kTile) * ((N + kTile - 1) / kTile);
+    const bool small = tiles_a <= 256 && tiles_b <= 256;
+    int64_t ax = 0, nA = tiles_a, nB = tiles_b, nC = 0;
+    if (small) {
+        nC = C ? (M < 96 ? M : 96) : 0;
+    } else {
+        ax = (K + 8 * kThreads - 1) / (8 * kThreads);
+        const int64_t want = (152 * 4 + ax - 1) / ax;
+        nA = ax * (M < want ? M : want);
+        nB = grid_for(tiles_b, 152 * 4);
+        nC = C ? (M < 152 ? M : 152) : 0;
+    }
+    cudaError_t e;
     // a programmatic dependent of the clearing of the workspace header, which
     // only its flag publication waits for
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(ax * ay + nB + nC));
+    cfg.gridDim = dim3((unsigned)(nA + nB + nC));
     cfg.blockDim = dim3(kThreads);
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
@@ -235,8 +329,8 @@ cudaError_t launch_split_f32_gemm(const float *A, int64_t M, int64_t K, int64_t 
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, split_f32_gemm_kernel, A, M, K, lda, B, N, ldb, Ap, Bp, ldcomp, ws,
-                                             ax, ay, nB, C, ldc, nC);
+    e = cudaLaunchKernelEx(&cfg, split_f32_gemm_kernel, A, M, K, lda, B, N, ldb, Ap, Bp, ldcomp, ws, ax, nA, nB, C,
+                           ldc, nC);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

@@ -59,15 +59,18 @@ def _band_intact(buf, nbytes):
     return bool(np.all(buf[nbytes:].cpu().numpy() == CANARY8))
 
 
-@pytest.mark.parametrize("M,N,K", [(300, 333, 700), (129, 257, 33)])
-def test_gemm_f32_guard_bands(M, N, K):
+@pytest.mark.parametrize("M,N,K,cpad", [(300, 333, 700, 7), (129, 257, 33, 7), (300, 336, 700, 8), (1000, 1024, 512, 4)])
+def test_gemm_f32_guard_bands(M, N, K, cpad):
+    """cpad: padding columns of C.  The last two shapes have N and the row
+    pitch of C multiples of 4, so the product-sum, which splits K for these
+    few-tile results, adds its K-parts into C by bulk tensor reductions."""
     dev = device()
     torch = _torch()
     A, B = synth.gemm_inputs("f32", M, N, K, 21)
     Ad, Abig = _padded(A, dev, 5, 2, CANARY32)
     Bd, Bbig = _padded(B, dev, 3, 1, CANARY32)
     Abefore, Bbefore = Abig.clone(), Bbig.clone()
-    Cbig = torch.full((M + 3, N + 7), CANARY32, dtype=torch.int32, device=dev)
+    Cbig = torch.full((M + 3, N + cpad), CANARY32, dtype=torch.int32, device=dev)
     C = Cbig.view(torch.float32)
     need = emu.emu_gemm_workspace_bytes(32, M, N, K)
     ws = _ws(need, dev)
