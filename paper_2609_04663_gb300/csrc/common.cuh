@@ -172,6 +172,13 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
     asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
 
+// Orders this thread's earlier global-memory accesses (generic proxy) before
+// its later bulk copies (async proxy) to the same addresses.
+__device__ __forceinline__ void fence_proxy_async_global()
+{
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
 // Makes this thread's shared-memory stores visible to the async proxy (the
 // tensor cores, TMA) before they are signalled to it.
 __device__ __forceinline__ void fence_proxy_async_smem()

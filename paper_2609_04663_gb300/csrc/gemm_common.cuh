@@ -127,4 +127,19 @@ inline bool make_c_map_f32(CUtensorMap *map, float *C, int64_t M, int64_t N, int
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The same for an FP64 C [M][ldc], boxes of 32 rows x 16 columns (128-byte
+// rows); N must be even for the same reason.
+inline bool make_c_map_f64(CUtensorMap *map, double *C, int64_t M, int64_t N, int64_t ldc)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc || (reinterpret_cast<uintptr_t>(C) & 15u) != 0 || (ldc & 1) != 0 || (N & 1) != 0) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)N, (cuuint64_t)M};
+    cuuint64_t strides[1] = {(cuuint64_t)ldc * 8};
+    cuuint32_t box[2] = {16, 32};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT64, 2, C, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace emu

@@ -66,14 +66,16 @@ __device__ __forceinline__ void reduce_tile(uint32_t tmem, int quarter, int c0, 
 // per row, and those epilogues took 4.7 us per 128 x 256 tile and 2.0 us per
 // 128 x 128 tile on GB300.
 template <bool REDUCE>
-__device__ __forceinline__ void epilogue_tma(uint32_t tmem, int quarter, int ncols, int m0, int n0,
+__device__ __forceinline__ void epilogue_tma(uint32_t tmem, int quarter, int ncols, int m0, int n0, int M, int N,
                                              const CUtensorMap *cmap, uint32_t stage)
 {
     tc_fence_after();
     const uint32_t lane = lane_id();
     const uint32_t slots = stage + (uint32_t)(quarter * ncols) * 128u;     // 32 rows x 4 bytes per column
+    // pieces wholly past the last row or column are neither staged nor copied
+    const int cols = m0 + quarter * 32 < M ? min(ncols, N - n0) : 0;
 #pragma unroll 1
-    for (int c = 0; c < ncols; c += 32) {
+    for (int c = 0; c < cols; c += 32) {
         uint32_t v[32];
         tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)c, v);
         tmem_ld_wait();
@@ -164,12 +166,12 @@ prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     } else if (warp == 1 && lane == 0) {
         mma_loop<BN, KB, STAGES>(tmem, base, full0, empty0, accum_bar, nkb, flags);
     } else if (warp >= 2) {
-        // ---------------- epilogue: TMEM -> registers -> C
-        const bool ok = mbar_wait(accum_bar, 0, flags);
-        __syncwarp();
-        if (ok && SPLIT == 1 && c_tma) epilogue_tma<false>(tmem, warp & 3, BN, m0, n0, &tmC, base);
+        // ---------------- epilogue: TMEM -> registers -> C (tcgen05.ld needs the
+        // whole warp, so a timeout in any lane skips the warp's epilogue)
+        const bool ok = __all_sync(0xFFFFFFFFu, mbar_wait(accum_bar, 0, flags));
+        if (ok && SPLIT == 1 && c_tma) epilogue_tma<false>(tmem, warp & 3, BN, m0, n0, M, N, &tmC, base);
         else if (ok && SPLIT == 1) store_tile(tmem, warp & 3, 0, BN, m0, n0, M, N, C, ldc);
-        else if (ok && nkb > 0 && c_tma) epilogue_tma<true>(tmem, warp & 3, BN, m0, n0, &tmC, base);
+        else if (ok && nkb > 0 && c_tma) epilogue_tma<true>(tmem, warp & 3, BN, m0, n0, M, N, &tmC, base);
         else if (ok && nkb > 0) reduce_tile(tmem, warp & 3, 0, BN, m0, n0, M, N, C, ldc);
     }
     tc_fence_before();

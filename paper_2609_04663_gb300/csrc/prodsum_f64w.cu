@@ -108,9 +108,9 @@ __device__ __forceinline__ double ld_cg_f64(const double *p)
 template <int NPROD, bool ROWCOL, bool TAIL, bool PAIR>
 __global__ void __launch_bounds__(F64WCfg::THREADS, 1)
 prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                    int M, int N, int K, const int32_t *__restrict__ vA, const int32_t *__restrict__ vB,
-                    double *__restrict__ C, int64_t ldc, double *__restrict__ acc, uint32_t *flags,
-                    const float *__restrict__ T, int64_t ldt)
+                    const __grid_constant__ CUtensorMap tmC, int c_tma, int M, int N, int K,
+                    const int32_t *__restrict__ vA, const int32_t *__restrict__ vB, double *__restrict__ C,
+                    int64_t ldc, double *__restrict__ acc, uint32_t *flags, const float *__restrict__ T, int64_t ldt)
 {
     using Cfg = F64WCfgT<PAIR>;
     extern __shared__ uint8_t smem_raw[];
@@ -386,7 +386,55 @@ prodsum_f64w_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                 }
             }
         }
-        if (ok && live) {
+        // The warp takes the bulk-copy branch together (its __syncwarp and the
+        // copies lane 0 issues need every lane) when no lane's wait timed out and
+        // one of its rows is live (a pair's second CTA may reach past the last
+        // row).  Lanes of rows past M read their accumulator elements (inside the
+        // tile, never written) and the copies leave those rows out.
+        const bool warp_ok = __all_sync(0xFFFFFFFFu, ok), warp_live = __any_sync(0xFFFFFFFFu, live);
+        if (warp_ok && warp_live && c_tma && !TAIL) {
+            // the accumulator holds every product now (this thread's own reductions,
+            // same addresses, so they precede these loads): C <- acc through the TMA
+            // engine.  Each 32 x 16 piece of the warp's rows (4 KB, two alternating
+            // buffers per warp in the stage memory, which every MMA has finished
+            // reading) is staged in the 128-byte-swizzled layout of the C map and
+            // written by one bulk tensor store: whole 128-byte row segments, where
+            // the per-lane stores below touch one cache line per row and lane.
+            const uint32_t bufs = base + (uint32_t)(warp - Cfg::FIRST_DRAIN) * 8192u;
+            fence_proxy_async_global();       // this thread's low-word writes to C precede the copies
+            __syncwarp();
+#pragma unroll 1
+            // pieces wholly past the last column are neither staged nor copied
+            for (int j0 = 0, g = 0; j0 < Cfg::COLS && n0 + cq * Cfg::COLS + j0 < N; j0 += 16, ++g) {
+                const uint32_t buf = bufs + (uint32_t)(g & 1) * 4096u;
+                if (g >= 2) {                 // the copy that last read this buffer
+                    if (lane == 0) bulk_wait_read<1>();
+                    __syncwarp();
+                }
+                const uint32_t srow = buf + (uint32_t)lane * 128u;
+#pragma unroll
+                for (int h = 0; h < 16; h += 8) {         // eight columns at a time: few live registers
+                    double out[8];
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) out[j] = ld_cg_f64(tacc + (j0 + h + j) * kBM);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const unsigned long long a = (unsigned long long)__double_as_longlong(out[2 * k]);
+                        const unsigned long long b = (unsigned long long)__double_as_longlong(out[2 * k + 1]);
+                        st_shared_v4(srow + ((uint32_t)((h / 2 + k) ^ (lane & 7)) << 4), (uint32_t)a,
+                                     (uint32_t)(a >> 32), (uint32_t)b, (uint32_t)(b >> 32));
+                    }
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_2d(&tmC, buf, n0 + cq * Cfg::COLS + j0, m0 + quarter * 32);
+                    bulk_commit();
+                }
+            }
+            if (lane == 0) bulk_wait_read<0>();
+            __syncwarp();
+        } else if (ok && live && !(c_tma && !TAIL)) {
             // the accumulator holds every product now (this thread's own reductions,
             // same addresses, so they precede these loads): C <- acc (+ the merged tail)
             const float *trow = TAIL ? T + (int64_t)(row < M ? row : 0) * ldt + n0 + cq * Cfg::COLS : nullptr;
@@ -437,6 +485,9 @@ cudaError_t run_f64w(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const 
     if (!make_plane_map(&ta, Ap, K, M, 6, ldcomp, Cfg::KB, kBM, a_plane) ||
         !make_plane_map(&tb, Bp, K, N, 6, ldcomp, Cfg::KB, Cfg::BH))
         return cudaErrorInvalidValue;
+    static_assert(Cfg::DRAIN_WARPS * 8192 <= Cfg::STAGES * Cfg::STAGE, "TMA epilogue staging exceeds the stages");
+    CUtensorMap tc = {};
+    const int c_tma = make_c_map_f64(&tc, C, M, N, ldc) ? 1 : 0;
     auto kern = prodsum_f64w_kernel<NPROD, ROWCOL, TAIL, PAIR>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
@@ -452,7 +503,7 @@ cudaError_t run_f64w(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const 
     at[0].val.clusterDim.z = 1;
     cfg.attrs = at;
     cfg.numAttrs = PAIR ? 1 : 0;
-    e = cudaLaunchKernelEx(&cfg, kern, ta, tb, (int)M, (int)N, (int)K, vA, vB, C, ldc, acc, flags, T, ldt);
+    e = cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, c_tma, (int)M, (int)N, (int)K, vA, vB, C, ldc, acc, flags, T, ldt);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

@@ -86,15 +86,19 @@ def test_gemm_f32_guard_bands(M, N, K, cpad):
     assert ok, worst
 
 
-@pytest.mark.parametrize("M,N,K,nprod", [(300, 333, 700, 21), (129, 257, 520, 6), (3000, 3000, 300, 21)])
-def test_gemm_f64_guard_bands(M, N, K, nprod):
+@pytest.mark.parametrize("M,N,K,nprod,cpad", [(300, 333, 700, 21, 7), (129, 257, 520, 6, 7), (3000, 3000, 300, 21, 7),
+                                               (3000, 3000, 300, 6, 8)])
+def test_gemm_f64_guard_bands(M, N, K, nprod, cpad):
+    """cpad: padding columns of C.  In the last shape N and the row pitch of C
+    are even, so the product-sum on 256-column tiles writes C by bulk tensor
+    stores."""
     dev = device()
     torch = _torch()
     A, B = synth.gemm_inputs("f64", M, N, K, 22)
     Ad, Abig = _padded(A, dev, 5, 2, CANARY64)
     Bd, Bbig = _padded(B, dev, 3, 1, CANARY64)
     Abefore, Bbefore = Abig.clone(), Bbig.clone()
-    Cbig = torch.full((M + 3, N + 7), CANARY64, dtype=torch.int64, device=dev)
+    Cbig = torch.full((M + 3, N + cpad), CANARY64, dtype=torch.int64, device=dev)
     C = Cbig.view(torch.float64)
     need = emu.emu_gemm_workspace_bytes(64, M, N, K)
     ws = _ws(need, dev)
