@@ -465,6 +465,32 @@ def reference_arm(args, rank, world):
     return 0
 
 
+def capture_run(args, local):
+    """--capture W[:P],W[:P],...: run each workload's split and product-sum
+    --warmup + --steps times in one process and print, for each, the name of
+    the product-sum kernel and the number of product-sum launches per step, so
+    that one profiler run (its kernel filter on "prodsum") yields the counters
+    of every workload in order.  Prints no JSON line."""
+    import torch
+    torch.cuda.set_device(local)
+    import __graft_entry__
+    __graft_entry__.build()
+    for item in args.capture.split(","):
+        name, _, nprod = item.partition(":")
+        case = Case(name, 0, int(nprod) if nprod else None)
+        stream = torch.cuda.current_stream()
+        for _ in range(args.warmup + args.steps):
+            case.split(stream)
+            case.prodsum(stream)
+        torch.cuda.synchronize()
+        per_step = 1 if case.mode == 32 else case.emu.emu_prodsum_f64_launches(case.M, case.N)
+        print(f"capture {name}" + (f"_np{case.nprod}" if case.mode == 64 else "") +
+              f" {case.kernel} launches_per_step={per_step} steps={args.warmup + args.steps}", flush=True)
+        del case
+        torch.cuda.empty_cache()
+    return 0
+
+
 def gpu_arm(args, rank, world, local):
     import torch
     torch.cuda.set_device(local)
@@ -581,12 +607,16 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--ref-seconds", type=float, default=15.0)
+    ap.add_argument("--capture", default=None,
+                    help="W[:P],...: only run these workloads' steps for a profiler (see capture_run); no JSON")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "ours":
         ap.error("--warmup must be at least 3")
     rank, world, local = dist_init()
     if args.impl == "reference":
         return reference_arm(args, rank, world)
+    if args.capture:
+        return capture_run(args, local)
     return gpu_arm(args, rank, world, local)
 
 
