@@ -13,6 +13,7 @@
 #include <cstdlib>
 
 #include "launchers.cuh"
+#include "pair_common.cuh"
 #include "prodsum_f32_common.cuh"
 
 namespace emu {
@@ -183,6 +184,145 @@ prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     }
 }
 
+// The FP32 product-sum on CTA pairs: a cluster of two CTAs on one TPC computes
+// a 256 x BN tile with tcgen05 cta_group::2 MMAs (M = 256) issued by the
+// leader (cluster rank 0).  Each CTA stages its 128 rows of the three A
+// slices and its BN / 2-row half of the three B slices, both CTAs' copies
+// counted on the leader's stage barrier; the MMA commits arrive on both CTAs'
+// barriers, and each CTA's TMEM receives its 128 x BN part of the
+// accumulator, which its own epilogue warps write into C.  An SM then takes
+// in 128 + BN / 2 rows of operands per K-block for 128 x BN results instead
+// of 128 + BN: with BN = 256 a third fewer bytes cross from L2 into shared
+// memory, which at 16384^3 (a step held by the power cap) took the
+// product-sum from 26.6 to 25.0 ms.  The MMAs and their order per output
+// element are those of prodsum_f32_kernel; C is bit-identical to it.
+// Timeouts: a peer whose wait gave up cannot see the leader's barriers, so
+// it lets its copies land for 200 us before winding down.
+template <int BN, int KB, int STAGES>
+struct F32PairCfg {
+    static constexpr int BH = BN / 2;                          // B rows staged by each CTA
+    static constexpr int A_TILE = kBM * KB * 2;
+    static constexpr int B_TILE = BH * KB * 2;
+    static constexpr int STAGE = 3 * A_TILE + 3 * B_TILE;
+    static constexpr uint32_t SWZ = (KB == 64) ? 2u : 4u;
+    static constexpr uint32_t SBO = 8u * KB * 2u;
+    static constexpr int BAR_OFF = STAGES * STAGE;
+    static constexpr int SMEM = BAR_OFF + 256 + 1024;
+    static_assert(KB == 32 || KB == 64, "K-block must fill one 64 B or 128 B swizzle row");
+    static_assert(BN % 32 == 0 && BN >= 64 && BN <= 256, "UMMA N of a pair");
+    static_assert(SMEM <= 232448, "shared memory per CTA");
+};
+
+template <int BN, int KB, int STAGES, int SPLIT>
+__global__ void __launch_bounds__(192, 1)
+prodsum_f32_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                        const __grid_constant__ CUtensorMap tmC, int c_tma, int M, int N, int K,
+                        float *__restrict__ C, int64_t ldc, uint32_t *flags)
+{
+    using Cfg = F32PairCfg<BN, KB, STAGES>;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    uint8_t *base_ptr = smem_raw + (base - raw);
+    const uint32_t full0 = base + Cfg::BAR_OFF, empty0 = full0 + 8u * STAGES;
+    const uint32_t accum_bar = empty0 + 8u * STAGES;
+    volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(base_ptr + Cfg::BAR_OFF + 16 * STAGES + 8);
+    const int warp = threadIdx.x >> 5, lane = lane_id();
+    const uint32_t rank = cluster_rank();
+    const int pm = ((M + kBM - 1) / kBM + 1) / 2, tiles_n = (N + BN - 1) / BN;   // pair tile rows, tile columns
+    const int ptiles = pm * tiles_n, cl = (int)(blockIdx.x >> 1), part = cl / ptiles;
+    int tp, tn;
+    tile_coords(cl % ptiles, pm, tiles_n, tp, tn);
+    const int m0 = (2 * tp + (int)rank) * kBM, n0 = tn * BN;   // this CTA's 128 rows of the pair's 256
+    const int nkb_all = (K + KB - 1) / KB, per = (nkb_all + SPLIT - 1) / SPLIT;
+    const int kb0 = min(nkb_all, part * per);
+    const int nkb = min(nkb_all, kb0 + per) - kb0;     // K-blocks of this pair
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) { mbar_init(full0 + 8u * s, 1); mbar_init(empty0 + 8u * s, 1); }
+        mbar_init(accum_bar, 1);
+        fence_mbar_init();
+        tma_prefetch_desc(&tmA);
+        tma_prefetch_desc(&tmB);
+    }
+    __syncthreads();
+    cluster_sync();                                   // both CTAs' barriers initialised
+    if (warp == 1) tmem_alloc_pair(smem_u32((const void *)tmem_slot), BN);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    // set-up above overlaps the end of the kernel that wrote the planes when
+    // this one is launched as its programmatic dependent
+    griddep_wait();
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer of this CTA: its A rows and its half of B,
+        // counted on the leader's full barrier
+        long issued = 0;
+        bool ok = true;
+        for (int kb = 0; kb < nkb && ok; ++kb) {
+            const int s = kb % STAGES;
+            if (!(ok = mbar_wait(empty0 + 8u * s, ((kb / STAGES) & 1) ^ 1, flags))) break;
+            const uint32_t st = base + (uint32_t)(s * Cfg::STAGE), fb = full0 + 8u * s, fl = peer_addr(fb, 0);
+            if (rank == 0) mbar_arrive_expect_tx(fb, 2 * Cfg::STAGE);
+            const int k0 = (kb0 + kb) * KB;
+#pragma unroll
+            for (int r = 0; r < 3; ++r) tma_load_3d_pair(st + r * Cfg::A_TILE, &tmA, fl, k0, m0, r);
+#pragma unroll
+            for (int r = 0; r < 3; ++r)
+                tma_load_3d_pair(st + 3 * Cfg::A_TILE + r * Cfg::B_TILE, &tmB, fl, k0, n0 + (int)rank * Cfg::BH, r);
+            ++issued;
+        }
+        if (!ok) {
+            if (rank == 0) {
+                drain_inflight(full0, STAGES, issued, flags);
+            } else {
+                const unsigned long long t0 = globaltimer_ns();
+                while (globaltimer_ns() - t0 < 200000ull) {}
+            }
+        }
+    } else if (warp == 1 && lane == 0 && rank == 0) {
+        // ---------------- MMA issuer (the leader): the six products of Eq.
+        // (fp32reuseorder) per 16-wide K step, M = 256 over the pair
+        constexpr uint32_t idesc = make_idesc_bf16(2 * kBM, BN);
+        for (int kb = 0; kb < nkb; ++kb) {
+            const int s = kb % STAGES;
+            if (!mbar_wait(full0 + 8u * s, (kb / STAGES) & 1, flags)) break;
+            tc_fence_after();
+            const uint32_t st = base + (uint32_t)(s * Cfg::STAGE);
+#pragma unroll
+            for (int kk = 0; kk < KB / 16; ++kk) {
+#pragma unroll
+                for (int q = 0; q < 6; ++q) {
+                    const uint64_t ad = make_sdesc(st + kChain[q][0] * Cfg::A_TILE + kk * 32, Cfg::SBO, Cfg::SWZ);
+                    const uint64_t bd = make_sdesc(st + 3 * Cfg::A_TILE + kChain[q][1] * Cfg::B_TILE + kk * 32,
+                                                   Cfg::SBO, Cfg::SWZ);
+                    mma_bf16_pair(tmem, ad, bd, idesc, (kb | kk | q) != 0);
+                }
+            }
+            mma_commit_pair(empty0 + 8u * s);         // both CTAs' stages reusable once these finish
+        }
+        mma_commit_pair(accum_bar);                   // both CTAs' accumulator parts complete
+    } else if (warp >= 2) {
+        // ---------------- epilogue of this CTA's 128 rows (tcgen05.ld needs the
+        // whole warp, so a timeout in any lane skips the warp's epilogue)
+        const bool ok = __all_sync(0xFFFFFFFFu, mbar_wait(accum_bar, 0, flags));
+        if (ok && SPLIT == 1 && c_tma) epilogue_tma<false>(tmem, warp & 3, BN, m0, n0, M, N, &tmC, base);
+        else if (ok && SPLIT == 1) store_tile(tmem, warp & 3, 0, BN, m0, n0, M, N, C, ldc);
+        else if (ok && nkb > 0 && c_tma) epilogue_tma<true>(tmem, warp & 3, BN, m0, n0, M, N, &tmC, base);
+        else if (ok && nkb > 0) reduce_tile(tmem, warp & 3, 0, BN, m0, n0, M, N, C, ldc);
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();                                   // the leader's MMAs are done with both CTAs
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc_pair(tmem, BN);
+    }
+}
+
 // Per-SM rates of the narrower tiles relative to 128 x 256 (measured at 8192^3:
 // 274 and 164 against 316 TFLOP/s for the whole GEMM).
 constexpr double kRate128 = 0.87, kRate64 = 0.52;
@@ -220,6 +360,41 @@ cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, c_tma, (int)M, (int)N, (int)K, C, ldc, flags);
+    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+}
+
+template <int BN, int KB, int STAGES, int SPLIT>
+cudaError_t run_f32_pair(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
+                         float *C, int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane, int64_t b_plane)
+{
+    using Cfg = F32PairCfg<BN, KB, STAGES>;
+    CUtensorMap ta, tb;
+    if (!make_plane_map(&ta, Ap, K, M, 3, ldcomp, KB, kBM, a_plane) ||
+        !make_plane_map(&tb, Bp, K, N, 3, ldcomp, KB, Cfg::BH, b_plane))
+        return cudaErrorInvalidValue;
+    static_assert(4 * BN * 128 <= STAGES * Cfg::STAGE, "TMA epilogue staging exceeds the stage memory");
+    CUtensorMap tc = {};
+    const int c_tma = make_c_map_f32(&tc, C, M, N, ldc) ? 1 : 0;
+    auto kern = prodsum_f32_pair_kernel<BN, KB, STAGES, SPLIT>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    if (e != cudaSuccess) return e;
+    const int64_t pairs = (((M + kBM - 1) / kBM + 1) / 2) * ((N + BN - 1) / BN) * SPLIT;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(2 * pairs));
+    cfg.blockDim = dim3(192);
+    cfg.dynamicSmemBytes = Cfg::SMEM;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
     e = cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, c_tma, (int)M, (int)N, (int)K, C, ldc, flags);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
@@ -284,6 +459,16 @@ cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *
 {
     int bn, parts;
     f32_tile_plan(M, N, K, c_zeroed, bn, parts);
+    // 128 x 256 tiles run as 256 x 256 tiles on CTA pairs (64-wide K-blocks,
+    // two 96 KB stages: at 16384^3 25.0 ms against 25.5 with 32-wide K-blocks
+    // in four stages) wherever there are two or more 128-row tile rows;
+    // EMU_F32_PAIR=0 keeps one CTA per tile
+    static const bool pair_ok = [] {
+        const char *e = std::getenv("EMU_F32_PAIR");
+        return !(e && e[0] == '0');
+    }();
+    if (bn == 256 && parts == 1 && pair_ok && M > kBM)
+        return run_f32_pair<256, 64, 2, 1>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
     if (parts == 2) return run_f32<128, 64, 2, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
     if (bn == 128) return run_f32<128, 64, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
     if (bn == 64) return run_f32<64, 64, 3>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);

@@ -59,11 +59,14 @@ def _band_intact(buf, nbytes):
     return bool(np.all(buf[nbytes:].cpu().numpy() == CANARY8))
 
 
-@pytest.mark.parametrize("M,N,K,cpad", [(300, 333, 700, 7), (129, 257, 33, 7), (300, 336, 700, 8), (1000, 1024, 512, 4)])
+@pytest.mark.parametrize("M,N,K,cpad", [(300, 333, 700, 7), (129, 257, 33, 7), (300, 336, 700, 8), (1000, 1024, 512, 4),
+                                        (4000, 1000, 64, 4)])
 def test_gemm_f32_guard_bands(M, N, K, cpad):
-    """cpad: padding columns of C.  The last two shapes have N and the row
-    pitch of C multiples of 4, so the product-sum, which splits K for these
-    few-tile results, adds its K-parts into C by bulk tensor reductions."""
+    """cpad: padding columns of C.  From the third shape on N and the row
+    pitch of C are multiples of 4, so the product-sum writes C by bulk tensor
+    copies: the few-tile results split K and add their K-parts into C by
+    bulk tensor reductions; the last one (4000 rows: the second CTA of the
+    last pair holds 32 of them) runs 256 x 256 tiles on CTA pairs."""
     dev = device()
     torch = _torch()
     A, B = synth.gemm_inputs("f32", M, N, K, 21)

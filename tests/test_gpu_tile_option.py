@@ -1,8 +1,10 @@
 """The product-sums' tile shapes. FP32 (EMU_F32_TILE=128x256 / 128x128 /
-128x64 forces one; unset, the library picks by tile count): every shape
+128x64 forces one; unset, the library picks by tile count; 128 x 256 tiles
+run as 256 x 256 tiles on CTA pairs unless EMU_F32_PAIR=0): every shape
 issues the same MMAs in the same order for each output element, so C must
 be bit-identical across shapes and within the FP32-mode bar of the oracle.
-The switch is read once per process, so each shape runs in a child process."""
+The switches are read once per process, so each shape runs in a child
+process."""
 import os
 import subprocess
 import sys
@@ -33,11 +35,14 @@ for M, N, K, seed in [(300, 333, 700, 1), (129, 257, 33, 3), (256, 512, 1024, 8)
 """
 
 
-def _run(tile):
+def _run(tile, pair=True):
     env = dict(os.environ)
     env.pop("EMU_F32_TILE", None)
+    env.pop("EMU_F32_PAIR", None)
     if tile:
         env["EMU_F32_TILE"] = tile
+    if not pair:
+        env["EMU_F32_PAIR"] = "0"
     code = CHILD.format(root=ROOT, tests=os.path.join(ROOT, "tests"))
     r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-2000:]
@@ -49,6 +54,9 @@ def test_f32_tile_shapes_parity_and_bit_identity():
     assert len(ref) == 4
     for tile in ("128x256", "128x128", "128x64"):
         assert _run(tile) == ref, tile
+    # 128 x 256 tiles with one CTA each instead of pairs (129 and 300 rows
+    # leave the second CTA of the last pair wholly or partly below the matrix)
+    assert _run("128x256", pair=False) == ref
 
 
 CHILD64 = r"""
