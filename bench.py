@@ -232,9 +232,10 @@ class Case:
         self.exec_flop = self.flop * (6 if self.mode == 32 else self.nprod)
         # kernels of ours per step: FP32 split of both operands = 1 launch; FP64 split of both =
         # 5 (level maxima of both, then a speculative pass and a verifier per operand);
-        # product-sum = 1, or in FP64 mode 2 when the library runs the last partial wave of
-        # 256-column tiles as 128 x 128 tiles (it reports its schedule)
-        self.launches = 1 if self.fused else 2 if self.mode == 32 else 5 + emu.emu_prodsum_f64_launches(M, N)
+        # product-sum = 1, or 2 when the library runs the last partial wave of 256-column
+        # tiles as 128 x 128 tiles (it reports its schedule)
+        self.launches = 1 if self.fused else 1 + emu.emu_prodsum_f32_launches(M, N) if self.mode == 32 else \
+            5 + emu.emu_prodsum_f64_launches(M, N)
         if self.merge_from is not None:
             self.launches += 1                    # the tail kernel
         if self.api and self.mode == 32:
@@ -483,7 +484,8 @@ def capture_run(args, local):
             case.split(stream)
             case.prodsum(stream)
         torch.cuda.synchronize()
-        per_step = 1 if case.mode == 32 else case.emu.emu_prodsum_f64_launches(case.M, case.N)
+        per_step = (case.emu.emu_prodsum_f32_launches if case.mode == 32 else
+                    case.emu.emu_prodsum_f64_launches)(case.M, case.N)
         print(f"capture {name}" + (f"_np{case.nprod}" if case.mode == 64 else "") +
               f" {case.kernel} launches_per_step={per_step} steps={args.warmup + args.steps}", flush=True)
         del case

@@ -305,6 +305,14 @@ emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
  * or another mode. */
 size_t emu_prodsum_workspace_bytes(int mode, int64_t M, int64_t N);
 
+/* Number of kernel launches of the FP32-mode product-sum for an M x N result
+ * (emu_prodsum_f32, and emu_gemm_f32 when it does not split K): 1, or 2 when
+ * the 256 x 256 tiles on pairs of SMs leave the last wave partly empty and
+ * its tiles run as 128 x 128 quarters in a second launch.  The paper has no
+ * counterpart: every schedule gives identical results, and the call only
+ * reports which kernels run.  0 for sizes < 1. */
+int emu_prodsum_f32_launches(int64_t M, int64_t N);
+
 /* Output-tile shape that the FP64-mode product-sum picks for an M x N
  * result, unless EMU_F64_TILE (128x128, 128x256 or 256x256) forces one:
  * width 128 or 256 columns; height 128 rows, or 256 rows where a 256-column

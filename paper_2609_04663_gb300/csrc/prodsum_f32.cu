@@ -105,12 +105,14 @@ __device__ __forceinline__ void epilogue_tma(uint32_t tmem, int quarter, int nco
 // SPLIT > 1: the grid holds SPLIT CTAs per output tile, each over its own
 // contiguous range of K-blocks, which add their FP32 accumulators into C (set
 // to zero beforehand) instead of storing them.  c_tma: C is written through
-// the tensor map tmC.
+// the tensor map tmC.  pair_first >= 0 (BN = 128): CTA b computes quarter
+// b % 4 of 256 x 256 tile pair_first + b / 4 in the raster order of
+// prodsum_f32_pair_kernel, which ran the tiles before it.
 template <int BN, int KB, int STAGES, int SPLIT>
 __global__ void __launch_bounds__(192, 1)
 prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmC, int c_tma, int M, int N, int K, float *__restrict__ C,
-                   int64_t ldc, uint32_t *flags)
+                   int64_t ldc, uint32_t *flags, int pair_first)
 {
     using Cfg = F32Cfg<BN, KB, STAGES>;
     extern __shared__ uint8_t smem_raw[];
@@ -124,8 +126,15 @@ prodsum_f32_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     const int warp = threadIdx.x >> 5, lane = lane_id();
     const int tiles_m = (M + kBM - 1) / kBM, tiles_n = (N + BN - 1) / BN;
     int tm, tn;
-    const int tiles = tiles_m * tiles_n, part = (int)blockIdx.x / tiles;
-    tile_coords((int)blockIdx.x % tiles, tiles_m, tiles_n, tm, tn);
+    const int tiles = tiles_m * tiles_n, part = pair_first >= 0 ? 0 : (int)blockIdx.x / tiles;
+    if (pair_first >= 0) {
+        int tp, tq;
+        tile_coords(pair_first + (int)(blockIdx.x >> 2), (tiles_m + 1) / 2, (N + 255) / 256, tp, tq);
+        tm = 2 * tp + (int)(blockIdx.x & 1);
+        tn = 2 * tq + (int)((blockIdx.x >> 1) & 1);
+    } else {
+        tile_coords((int)blockIdx.x % tiles, tiles_m, tiles_n, tm, tn);
+    }
     const int m0 = tm * kBM, n0 = tn * BN;
     const int nkb_all = (K + KB - 1) / KB, per = (nkb_all + SPLIT - 1) / SPLIT;
     const int kb0 = min(nkb_all, part * per);
@@ -332,7 +341,8 @@ constexpr double kSplitCost = 0.95;
 
 template <int BN, int KB, int STAGES, int SPLIT = 1>
 cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
-                    float *C, int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane, int64_t b_plane)
+                    float *C, int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane, int64_t b_plane,
+                    int pair_first = -1, int64_t pair_tiles = 0)
 {
     using Cfg = F32Cfg<BN, KB, STAGES>;
     CUtensorMap ta, tb;
@@ -346,7 +356,7 @@ cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
     auto kern = prodsum_f32_kernel<BN, KB, STAGES, SPLIT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
-    const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + BN - 1) / BN) * SPLIT;
+    const int64_t tiles = pair_first >= 0 ? 4 * pair_tiles : ((M + kBM - 1) / kBM) * ((N + BN - 1) / BN) * SPLIT;
     // launched as a programmatic dependent of the previous kernel in the
     // stream: its set-up overlaps that kernel's tail (griddep_wait orders the
     // rest after it)
@@ -360,14 +370,15 @@ cudaError_t run_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const u
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, c_tma, (int)M, (int)N, (int)K, C, ldc, flags);
+    e = cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, c_tma, (int)M, (int)N, (int)K, C, ldc, flags, pair_first);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
 template <int BN, int KB, int STAGES, int SPLIT>
 cudaError_t run_f32_pair(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, const uint16_t *Bp, int64_t ldcomp,
-                         float *C, int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane, int64_t b_plane)
+                         float *C, int64_t ldc, uint32_t *flags, cudaStream_t st, int64_t a_plane, int64_t b_plane,
+                         int64_t pair_tiles)
 {
     using Cfg = F32PairCfg<BN, KB, STAGES>;
     CUtensorMap ta, tb;
@@ -380,7 +391,7 @@ cudaError_t run_f32_pair(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, co
     auto kern = prodsum_f32_pair_kernel<BN, KB, STAGES, SPLIT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
-    const int64_t pairs = (((M + kBM - 1) / kBM + 1) / 2) * ((N + BN - 1) / BN) * SPLIT;
+    const int64_t pairs = pair_tiles * SPLIT;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(2 * pairs));
     cfg.blockDim = dim3(192);
@@ -439,6 +450,52 @@ void f32_tile_plan(int64_t M, int64_t N, int64_t K, bool split_ok, int &bn, int 
     }
 }
 
+// Per-SM rate of a 128 x 128 tile relative to the 256 x 256 tiles on pairs.
+constexpr double kRateQuarter = 0.85;
+
+static bool f32_pair_ok()
+{
+    static const bool ok = [] {
+        const char *e = std::getenv("EMU_F32_PAIR");
+        return !(e && e[0] == '0');
+    }();
+    return ok;
+}
+
+// Schedule of the 128 x 256 plan: 256 x 256 tiles on CTA pairs wherever there
+// are two or more 128-row tile rows (EMU_F32_PAIR=0 keeps one CTA per tile).
+// When the pair tiles leave the last wave partly empty and its tiles fit one
+// wave as 128 x 128 quarters, those run in a second launch of the one-CTA
+// kernel if that is estimated at least 2 % faster (a quarter takes
+// 0.5 / kRateQuarter of a pair wave).  pairs: pair tiles in the first launch;
+// rest: pair tiles left to the quarters launch (0: none).  false: no pairs.
+static bool f32_pair_plan(int64_t M, int64_t N, int64_t &pairs, int64_t &rest)
+{
+    if (!f32_pair_ok() || M <= kBM) return false;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 2)
+        sms = 152;
+    const int64_t total = (((M + kBM - 1) / kBM + 1) / 2) * ((N + 255) / 256), per_wave = sms / 2;
+    const int64_t full = total / per_wave, left = total % per_wave;
+    pairs = total;
+    rest = 0;
+    if (full >= 1 && left > 0 && 4 * left <= sms &&
+        (double)full + 0.5 / kRateQuarter <= 0.98 * (double)(full + 1)) {
+        pairs = total - left;
+        rest = left;
+    }
+    return true;
+}
+
+int f32_prodsum_launches(int64_t M, int64_t N)
+{
+    int bn, parts;
+    f32_tile_plan(M, N, 0, false, bn, parts);
+    int64_t pairs, rest;
+    return (bn == 256 && f32_pair_plan(M, N, pairs, rest) && rest > 0) ? 2 : 1;
+}
+
 int f32_tile_columns(int64_t M, int64_t N)
 {
     int bn, parts;
@@ -461,14 +518,15 @@ cudaError_t launch_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *
     f32_tile_plan(M, N, K, c_zeroed, bn, parts);
     // 128 x 256 tiles run as 256 x 256 tiles on CTA pairs (64-wide K-blocks,
     // two 96 KB stages: at 16384^3 25.0 ms against 25.5 with 32-wide K-blocks
-    // in four stages) wherever there are two or more 128-row tile rows;
-    // EMU_F32_PAIR=0 keeps one CTA per tile
-    static const bool pair_ok = [] {
-        const char *e = std::getenv("EMU_F32_PAIR");
-        return !(e && e[0] == '0');
-    }();
-    if (bn == 256 && parts == 1 && pair_ok && M > kBM)
-        return run_f32_pair<256, 64, 2, 1>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
+    // in four stages), the last partial wave possibly as 128 x 128 quarters
+    int64_t pairs, rest;
+    if (bn == 256 && parts == 1 && f32_pair_plan(M, N, pairs, rest)) {
+        cudaError_t e = run_f32_pair<256, 64, 2, 1>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane,
+                                                    pairs);
+        if (e == cudaSuccess && rest > 0)
+            e = run_f32<128, 64, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane, (int)pairs, rest);
+        return e;
+    }
     if (parts == 2) return run_f32<128, 64, 2, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
     if (bn == 128) return run_f32<128, 64, 2>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);
     if (bn == 64) return run_f32<64, 64, 3>(M, N, K, Ap, Bp, ldcomp, C, ldc, flags, st, a_plane, b_plane);

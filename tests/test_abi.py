@@ -154,3 +154,17 @@ def test_f64_tile_width_report(lib):
     assert emu.emu_prodsum_f64_launches(1024, 1024) == 1
     assert emu.emu_prodsum_f64_launches(0, 1) == 0
 
+
+def test_f32_launch_report(lib):
+    # no GPU here: the launcher assumes 152 SMs (76 pairs per wave)
+    if os.environ.get("EMU_F32_TILE") or os.environ.get("EMU_F32_PAIR"):
+        pytest.skip("EMU_F32_TILE / EMU_F32_PAIR force a schedule")
+    # 4096^2: 256 pair tiles, 3.4 waves, the last 28 as 112 128 x 128 quarters;
+    # 8192^2: 1024 pair tiles, 13.5 waves, the last 36 as 144 quarters;
+    # 16384^2: 53.9 waves, the last 68 pair tiles would need 272 quarters
+    assert emu.emu_prodsum_f32_launches(4096, 4096) == 2
+    assert emu.emu_prodsum_f32_launches(8192, 8192) == 2
+    assert emu.emu_prodsum_f32_launches(16384, 16384) == 1
+    assert emu.emu_prodsum_f32_launches(1024, 1024) == 1
+    assert emu.emu_prodsum_f32_launches(0, 5) == 0
+
