@@ -228,6 +228,9 @@ class Case:
         # (128 x 256 on one SM, 256 x 256 on a pair of SMs), both kernels named after their file
         self.kernel = "prodsum_f32" if self.mode == 32 else \
             "prodsum_f64w" if emu.emu_prodsum_f64_tile_columns(M, N) == 256 else "prodsum_f64"
+        # the kernel's own name (FP32: 256 x 256 tiles on CTA pairs have a kernel of their own)
+        self.kernel_name = "prodsum_f32_pair_kernel" if self.mode == 32 and emu.emu_prodsum_f32_tile_rows(M, N) == 256 \
+            else self.kernel + "_kernel"
         self.flop = 2.0 * M * N * K
         self.exec_flop = self.flop * (6 if self.mode == 32 else self.nprod)
         # kernels of ours per step: FP32 split of both operands = 1 launch; FP64 split of both =
@@ -515,7 +518,7 @@ def gpu_arm(args, rank, world, local):
     roofline = {"bound": "tensor", "achieved": achieved, "peak": pk["bf16_burst"], "unit": "TFLOP/s",
                 "frac": achieved / pk["bf16_burst"],
                 "peak_source": f"{pk['source']} bf16 burst (cuBLAS 8192^3); sustained {pk['bf16_sustained']}",
-                "kernel": "gemm_f32_fused_kernel" if case.fused else case.kernel + "_kernel",
+                "kernel": "gemm_f32_fused_kernel" if case.fused else case.kernel_name,
                 "traffic": None if case.fused or case.merge_from else
                            kernel_traffic(case.kernel, name if case.mode == 32 else f"{name}_np{case.nprod}")}
     flags = case.emu.read_flags(case.gemm_ws if case.gemm_ws is not None else case.ws)

@@ -305,12 +305,17 @@ emu_status emu_prodsum_f32(int64_t M, int64_t N, int64_t K, const uint16_t *Acom
  * or another mode. */
 size_t emu_prodsum_workspace_bytes(int mode, int64_t M, int64_t N);
 
-/* Number of kernel launches of the FP32-mode product-sum for an M x N result
- * (emu_prodsum_f32, and emu_gemm_f32 when it does not split K): 1, or 2 when
- * the 256 x 256 tiles on pairs of SMs leave the last wave partly empty and
- * its tiles run as 128 x 128 quarters in a second launch.  The paper has no
- * counterpart: every schedule gives identical results, and the call only
- * reports which kernels run.  0 for sizes < 1. */
+/* Output tiles of the FP32-mode product-sum for an M x N result
+ * (emu_prodsum_f32, and emu_gemm_f32 when it does not split K), unless
+ * EMU_F32_TILE (128x256, 128x128 or 128x64) or EMU_F32_PAIR=0 forces a
+ * shape: width 256, 128 or 64 columns; height 128 rows, or 256 rows where
+ * 256-column tiles run on a pair of SMs (a cluster of two CTAs sharing each
+ * MMA); and the number of kernel launches, 1, or 2 when the pair tiles leave
+ * the last wave partly empty and its tiles run as 128 x 128 quarters in a
+ * second launch.  The paper has no counterpart: every shape gives identical
+ * results, and the calls only report which kernels run.  0 for sizes < 1. */
+int emu_prodsum_f32_tile_columns(int64_t M, int64_t N);
+int emu_prodsum_f32_tile_rows(int64_t M, int64_t N);
 int emu_prodsum_f32_launches(int64_t M, int64_t N);
 
 /* Output-tile shape that the FP64-mode product-sum picks for an M x N

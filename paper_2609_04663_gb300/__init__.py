@@ -50,6 +50,8 @@ _SIGS = {
     "emu_prodsum_f64_tile_rows": ("i", ["l", "l"]),
     "emu_prodsum_f64_launches": ("i", ["l", "l"]),
     "emu_prodsum_f32_launches": ("i", ["l", "l"]),
+    "emu_prodsum_f32_tile_columns": ("i", ["l", "l"]),
+    "emu_prodsum_f32_tile_rows": ("i", ["l", "l"]),
     "emu_split_f64_rowcol_workspace_bytes": ("size", ["l"]),
     "emu_split_f64_rowcol": ("i", ["p", "l", "l", "l", "i", "p", "l", "p", "p", "size", "p"]),
     "emu_gemm_f64_rowcol_workspace_bytes": ("size", ["l", "l", "l"]),
@@ -122,6 +124,8 @@ emu_prodsum_f64_tile_columns = _mk("emu_prodsum_f64_tile_columns")
 emu_prodsum_f64_tile_rows = _mk("emu_prodsum_f64_tile_rows")
 emu_prodsum_f64_launches = _mk("emu_prodsum_f64_launches")
 emu_prodsum_f32_launches = _mk("emu_prodsum_f32_launches")
+emu_prodsum_f32_tile_columns = _mk("emu_prodsum_f32_tile_columns")
+emu_prodsum_f32_tile_rows = _mk("emu_prodsum_f32_tile_rows")
 emu_split_f64_rowcol_workspace_bytes = _mk("emu_split_f64_rowcol_workspace_bytes")
 emu_split_f64_rowcol = _mk("emu_split_f64_rowcol")
 emu_gemm_f64_rowcol_workspace_bytes = _mk("emu_gemm_f64_rowcol_workspace_bytes")

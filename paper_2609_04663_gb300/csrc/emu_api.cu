@@ -286,6 +286,18 @@ emu_status emu_gemm_f64(int64_t M, int64_t N, int64_t K, const double *A, int64_
     return cuda_status(e);
 }
 
+int emu_prodsum_f32_tile_columns(int64_t M, int64_t N)
+{
+    if (M < 1 || N < 1) return 0;
+    return f32_tile_columns(M, N);
+}
+
+int emu_prodsum_f32_tile_rows(int64_t M, int64_t N)
+{
+    if (M < 1 || N < 1) return 0;
+    return f32_tile_rows(M, N);
+}
+
 int emu_prodsum_f32_launches(int64_t M, int64_t N)
 {
     if (M < 1 || N < 1) return 0;

@@ -73,6 +73,7 @@ cudaError_t launch_split_f32_gemm(const float *A, int64_t M, int64_t K, int64_t 
 // first.
 int f32_tile_columns(int64_t M, int64_t N);
 int f32_prodsum_launches(int64_t M, int64_t N);
+int f32_tile_rows(int64_t M, int64_t N);
 int f32_split_parts(int64_t M, int64_t N, int64_t K);
 // Eq. (fp32split) and the FP32 product-sum in one kernel: A (M x K, lda) and
 // B (K x N, ldb) FP32 row-major are split inside the product-sum's producer;

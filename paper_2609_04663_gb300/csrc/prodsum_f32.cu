@@ -496,6 +496,14 @@ int f32_prodsum_launches(int64_t M, int64_t N)
     return (bn == 256 && f32_pair_plan(M, N, pairs, rest) && rest > 0) ? 2 : 1;
 }
 
+int f32_tile_rows(int64_t M, int64_t N)
+{
+    int bn, parts;
+    f32_tile_plan(M, N, 0, false, bn, parts);
+    int64_t pairs, rest;
+    return (bn == 256 && f32_pair_plan(M, N, pairs, rest)) ? 256 : 128;
+}
+
 int f32_tile_columns(int64_t M, int64_t N)
 {
     int bn, parts;

@@ -167,4 +167,11 @@ def test_f32_launch_report(lib):
     assert emu.emu_prodsum_f32_launches(16384, 16384) == 1
     assert emu.emu_prodsum_f32_launches(1024, 1024) == 1
     assert emu.emu_prodsum_f32_launches(0, 5) == 0
+    # 256-column tiles, on CTA pairs where there are two tile rows
+    assert emu.emu_prodsum_f32_tile_columns(16384, 16384) == 256
+    assert emu.emu_prodsum_f32_tile_rows(16384, 16384) == 256
+    assert emu.emu_prodsum_f32_tile_rows(128, 65536) == 128
+    assert emu.emu_prodsum_f32_tile_columns(1024, 1024) in (64, 128)
+    assert emu.emu_prodsum_f32_tile_rows(1024, 1024) == 128
+    assert emu.emu_prodsum_f32_tile_rows(0, 4) == 0
 
