@@ -9,7 +9,9 @@
 // the operand-reuse order of Eq. (fp32reuseorder).  The accumulator is read
 // once at the end.  Warp roles: warp 0 lane 0 issues TMA loads, warp 1 owns
 // TMEM and lane 0 issues the MMAs, warps 2-5 run the epilogue.  Every wait is
-// bounded and reports EMU_FLAG_TIMEOUT instead of hanging.
+// bounded and reports EMU_FLAG_TIMEOUT instead of hanging.  The 128 x 256
+// plan runs on CTA pairs (prodsum_f32_pair_kernel: 256 x 256 tiles, the same
+// MMAs per output element).
 #include <cstdlib>
 
 #include "launchers.cuh"
@@ -420,7 +422,8 @@ cudaError_t run_f32_pair(int64_t M, int64_t N, int64_t K, const uint16_t *Ap, co
 // few 128 x 256 tiles to fill the GPU.  The choice maximises (SMs kept busy
 // over the waves) x (relative per-SM rate).  Every shape issues the same MMAs
 // in the same order for each output element, so C does not depend on it.
-// EMU_F32_TILE=128x256 / 128x128 / 128x64 forces one.
+// EMU_F32_TILE=128x256 / 128x128 / 128x64 forces one.  The 128 x 256 plan
+// runs on CTA pairs where it can (f32_pair_plan below).
 void f32_tile_plan(int64_t M, int64_t N, int64_t K, bool split_ok, int &bn, int &parts)
 {
     static const int forced = [] {
