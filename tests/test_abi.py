@@ -175,3 +175,28 @@ def test_f32_launch_report(lib):
     assert emu.emu_prodsum_f32_tile_rows(1024, 1024) == 128
     assert emu.emu_prodsum_f32_tile_rows(0, 4) == 0
 
+
+def test_f32_schedule_rule(lib):
+    """The FP32 schedule over a range of result sizes (152 SMs assumed, as
+    without a GPU): a second launch of 128 x 128 quarters exactly when the
+    pair tiles leave a partial last wave after at least one full one, its
+    tiles fit one wave as quarters (4 per pair tile), and that is estimated
+    at least 2 % faster (a quarter wave costs 0.5 / 0.85 of a pair wave)."""
+    if os.environ.get("EMU_F32_TILE") or os.environ.get("EMU_F32_PAIR"):
+        pytest.skip("EMU_F32_TILE / EMU_F32_PAIR force a schedule")
+    seen = set()
+    for M in (256, 1000, 2048, 3000, 4096, 5120, 6144, 8192, 10240, 12288, 16384):
+        for N in (512, 2048, 4096, 8192, 12288, 16384):
+            cols, rows = emu.emu_prodsum_f32_tile_columns(M, N), emu.emu_prodsum_f32_tile_rows(M, N)
+            launches = emu.emu_prodsum_f32_launches(M, N)
+            assert cols in (64, 128, 256) and rows in (128, 256) and launches in (1, 2)
+            if rows == 256:
+                assert cols == 256 and M > 128
+            pairs = ((M + 127) // 128 + 1) // 2 * ((N + 255) // 256)
+            full, left = divmod(pairs, 76)
+            mixed = rows == 256 and full >= 1 and 0 < left and 4 * left <= 152 and \
+                full + 0.5 / 0.85 <= 0.98 * (full + 1)
+            assert launches == (2 if mixed else 1), (M, N, pairs)
+            seen.add(launches)
+    assert seen == {1, 2}
+
